@@ -1,0 +1,57 @@
+"""Plant plausible mistakes in copies of the oracle; each must trip some pin.
+
+Every mutation is a literal source edit of oracle/taskpress_oracle.py, loaded
+as a separate module on the CPU.  A mutation that no pin catches would mean
+the pins leave that part of the oracle unchecked.
+"""
+import inspect
+import types
+
+import pytest
+
+from oracle import taskpress_oracle as O
+from tests import oracle_pins
+
+SRC = inspect.getsource(O)
+
+MUTATIONS = {
+    "softmax over the wrong axis": ("z = np.sum(e, axis=1, keepdims=True)", "z = np.sum(e, axis=0, keepdims=True)"),
+    "scale 1/d instead of 1/sqrt(d)": ("1.0 / math.sqrt(d)\n    gamma", "1.0 / d\n    gamma"),
+    "no max subtraction": ("e = np.exp(x - m)", "e = np.exp(x)"),
+    "sum over the GQA group": ("return a.sum(axis=0) / g", "return a.sum(axis=0)"),
+    "mean over guide tokens": ("return a.sum(axis=0) / g", "return a.mean(axis=0)"),
+    "interleaved GQA heads": ("qg = q[b, h * g:(h + 1) * g]", "qg = q[b, h::n_heads_kv]"),
+    "pool renormalised at edges": ("return out / kernel", "return out / np.convolve(np.ones(n), np.ones(kernel), 'same')"),
+    "pool window one short": ("for off in range(-half, half + 1):", "for off in range(-half, half):"),
+    "pool accepts even kernels": ("if kernel < 1 or kernel % 2 == 0:", "if kernel < 1:"),
+    "quant divisor 2^(b-1)": ("qmax = (1 << (quant_bits - 1)) - 1", "qmax = (1 << (quant_bits - 1))"),
+    "quant rounds half away from zero": ("q = np.clip(np.rint(quot), -qmax, qmax)", "q = np.clip(np.trunc(quot + np.copysign(0.5, quot)), -qmax, qmax)"),
+    "quant truncates": ("q = np.clip(np.rint(quot), -qmax, qmax)", "q = np.clip(np.trunc(quot), -qmax, qmax)"),
+    "quant uses mean |v|": ("a = np.max(np.abs(v), axis=-1)", "a = np.mean(np.abs(v), axis=-1)"),
+    "additive combine": ("return pooled * np.asarray(gamma, dtype=np.float64)", "return pooled + np.asarray(gamma, dtype=np.float64)"),
+    "ties keep the higher index": ("order = np.lexsort((np.arange(n), -scores))", "order = np.lexsort((-np.arange(n), -scores))"),
+    "selects the smallest scores": ("order = np.lexsort((np.arange(n), -scores))", "order = np.lexsort((np.arange(n), scores))"),
+    "kept indices not ascending": ("return np.sort(order[:k]).astype(np.int64)", "return order[:k].astype(np.int64)"),
+    "naive ceil budget": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.ceil(keep_ratio * float(n))"),
+    "budget rounds down": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.floor(keep_ratio * float(n))"),
+    "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma)", "s_key = key_scores(qg, k_all[h, 0:n], sigma)"),
+}
+
+
+def _mutant(old, new):
+    assert SRC.count(old) == 1, f"mutation anchor not unique/found: {old!r}"
+    mod = types.ModuleType("oracle_mutant")
+    exec(compile(SRC.replace(old, new), "oracle_mutant", "exec"), mod.__dict__)
+    return mod
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_mutation_is_caught(name):
+    mod = _mutant(*MUTATIONS[name])
+    caught = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(mod)
+        except Exception as e:  # AssertionError or a crash both count as caught
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches mutation: {name}"
