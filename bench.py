@@ -1,0 +1,444 @@
+#!/usr/bin/env python3
+"""Benchmark of the TaskPress compression path on GB300.
+
+One step = the fused per-layer compression (tp_compress_layer: V scales,
+guide scores, per-head top-budget selection, compaction) over every layer of
+the workload, with K/V already resident in HBM.  The metric is context tokens
+compressed per second per layer (all heads): value = n_tokens * layers / t_step.
+
+Default workload: the Llama-3-8B-shaped 32-layer stack at 128K context with a
+128-token guide (32 q / 8 KV heads, d = 128, keep 10%).  `--config 2` runs the
+32K single layer.  Each layer's K+V (512 MiB at 128K) exceeds the 129 MB L2,
+and consecutive layers use different buffers, so no L2 flush is needed.
+
+Also reported on the same JSON line:
+  roofline      the dominant kernel, timed per launch with CUDA events over a
+                staged pass of the same workload (the fused call's kernels
+                launched one entry point at a time);
+  hbm_fused     algorithmic bytes of the fused layer / its time / HBM peak;
+  e2e           the same metric through the public API with the inputs in
+                pinned host memory, H2D and D2H copies inside the timed region;
+  cpu_baseline  the CPU oracle on a bounded sample of one layer;
+  clocks        nvidia-smi samples taken during the timed region.
+
+`--impl reference` times the CPU oracle (the only other implementation of
+this path) on the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "context tokens compressed/s per layer (all heads) at 32K/128K; % of HBM roofline"
+UNIT = "tokens/s/layer"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", type=int, default=3, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-layers", type=int, default=4)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-heads", type=int, default=0, help="0: every KV head of one layer")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, val in zip(names, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(nm)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic bytes / flops (per layer)
+# ---------------------------------------------------------------------------
+def layer_algorithmic(w, kept_total_tokens):
+    """K + V read once, the compressed cache written once (Kc, Vc, int8 Vc, scale,
+    index per kept token and head), the guide queries read once."""
+    d = w.head_dim
+    n = w.n_total
+    read = 4 * d * n * w.n_heads_kv + 2 * d * w.batch * w.n_heads_q * w.guide_len
+    write = (2 * d + 2 * d + d + 4 + 4) * kept_total_tokens
+    flops_one_pass = 2 * w.rows * d * n * w.n_heads_kv
+    return read, write, flops_one_pass
+
+
+def traffic_record(kernel: str, workload: str):
+    """Per-launch DRAM bytes of a kernel from the committed ncu summary, if the
+    kernel source has not changed since the capture (else None)."""
+    src = os.path.join(ROOT, "paper_2608_03276_gb300", "csrc", "score_tc.cu")
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:12]
+        with open(os.path.join(ROOT, "profiles", "ncu_traffic.txt")) as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) >= 4 and not line.startswith("#") and parts[0] == kernel \
+                        and parts[1] == workload and parts[2] == sha:
+                    return float(parts[3])
+    except Exception:
+        pass
+    return None
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle sample (the cpu_baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+def _oracle_unit(args):
+    q, k, v, g, n_heads_q, keep_ratio, budget = args
+    from oracle import taskpress_oracle as O
+    t0 = time.perf_counter()
+    O.compress_layer(q, k, v, [0, k.shape[1]], n_heads_q=g, n_heads_kv=1,
+                     keep_ratio=keep_ratio, fixed_budget=budget)
+    return time.perf_counter() - t0
+
+
+def oracle_inputs(w):
+    """Host inputs of layer 0, document 0 of the workload (what the oracle sample sees)."""
+    from paper_2608_03276_gb300 import synth
+    one_doc = w.with_(doc_lens=(w.doc_lens[0],))
+    return one_doc, synth.make_layer(one_doc)
+
+
+def oracle_sample(w, sample, heads, workers):
+    """Times the oracle on `heads` KV heads of layer 0 of document 0 (one
+    process per head, BLAS single-threaded).  Returns (tokens/s/layer, detail, cores)."""
+    import multiprocessing as mp
+    one_doc, x = sample
+    n = one_doc.n_total
+    g = w.group
+    units = [(x.q[:, h * g:(h + 1) * g].copy(), x.k[h:h + 1].copy(), x.v[h:h + 1].copy(), g, g,
+              w.keep_ratio, w.budget) for h in heads]
+    os.environ["OPENBLAS_NUM_THREADS"] = "1"
+    os.environ["OMP_NUM_THREADS"] = "1"
+    ctx = mp.get_context("spawn")
+    t0 = time.perf_counter()
+    with ctx.Pool(processes=min(workers, len(units))) as pool:
+        per_unit = pool.map(_oracle_unit, units)
+    wall = time.perf_counter() - t0
+    # heads of one layer are independent: the sample covers len(heads)/H_kv of a layer
+    frac = len(heads) / w.n_heads_kv
+    value = n * frac / wall
+    detail = (f"layer 0 of {w.name}: {len(heads)} of {w.n_heads_kv} KV heads of document 0 "
+              f"(n={n}), one process per head, fp64 numpy; wall {wall:.1f}s, "
+              f"CPU {sum(per_unit):.1f}s")
+    return value, detail, min(workers, len(units))
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    cores = os.cpu_count() or 1
+    times = []
+    heads = list(range(min(w.n_heads_kv, cores)))
+    sample = oracle_inputs(w)
+    for i in range(args.warmup + args.steps):
+        v, detail, used = oracle_sample(w, sample, heads, cores)
+        if i >= args.warmup:
+            times.append(v)
+    value = statistics.median(times)
+    n_units = len(heads)
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "layers_sampled": 1, "heads_sampled": n_units},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": used, "kind": "oracle",
+                         "sample": detail},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_ours(args, w):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2608_03276_gb300 import binding, synth
+
+    hbm_peak, tf_burst, tf_sust, peak_src = measured_peaks()
+    stream = torch.cuda.current_stream()
+    L = w.layers
+    p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, w.doc_offsets())
+    # each rank compresses its own stack (weak scaling; no data-path collective)
+    wr = w.with_(seed=w.seed + 7919 * rank)
+    layers = [synth.make_layer_torch(wr, l, dev) for l in range(L)]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, dev, with_scores=False)
+            for _ in range(L)]
+    ws = outs[0].ws
+    for o in outs[1:]:
+        o.ws = ws
+    cap = outs[0].cap
+    kept_tokens = sum(int(min(w.budget, n)) if w.budget >= 0 else binding.tp_budget(int(n), w.keep_ratio)
+                      for n in w.doc_lens) * w.n_heads_kv
+
+    def step():
+        for (q, k, v), o in zip(layers, outs):
+            binding.compress(p, q, k, v, w.keep_ratio, w.budget, o, stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    st = binding.tp_check_status(ws)
+    if st != 0:
+        raise RuntimeError(f"device status after warm-up: {binding.tp_status_string(st)}")
+
+    # ---- timed region (fused path)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = w.n_total * L * world / (ms / 1e3)
+    kernels_per_call = 5 if cap > 0 else 4
+    gpu_launches = kernels_per_call * L * args.steps
+
+    # ---- staged pass: per-kernel CUDA-event times of the same launches
+    rows = w.rows
+    lse = torch.empty((w.batch, w.n_heads_kv, rows), dtype=torch.float32, device=dev)
+    skey = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    gamma = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    scores = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    stage_names = ["vquant", "lse", "keyscore", "select+compact"]
+    stage_ms = {s: 0.0 for s in stage_names}
+    reps = max(1, args.steps)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+    nlayer_stage = min(L, 8)
+    for _ in range(reps):
+        for li in range(nlayer_stage):
+            (q, k, v), o = layers[li], outs[li]
+            evs[0].record(stream)
+            binding.tp_quantize_v(p, v, None, gamma, stream)
+            evs[1].record(stream)
+            binding.tp_guide_lse(p, q, k, lse, ws, stream)
+            evs[2].record(stream)
+            binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
+            evs[3].record(stream)
+            binding.tp_guide_scores(p, q, k, gamma, scores, ws, stream)  # scores for select; not timed
+            evs[4].record(stream)
+            binding.tp_select(p, scores, w.keep_ratio, w.budget, o.idx, ws, stream)
+            binding.tp_compact(p, k, v, gamma, o.idx, w.keep_ratio, w.budget, o.kc, o.vc, o.vqc,
+                               o.gammac, stream)
+            evs[5].record(stream)
+            torch.cuda.synchronize()
+            stage_ms["vquant"] += evs[0].elapsed_time(evs[1])
+            stage_ms["lse"] += evs[1].elapsed_time(evs[2])
+            stage_ms["keyscore"] += evs[2].elapsed_time(evs[3])
+            stage_ms["select+compact"] += evs[4].elapsed_time(evs[5])
+    nstage = reps * nlayer_stage
+    stage_ms = {s: v / nstage for s, v in stage_ms.items()}
+
+    read_b, write_b, flops1 = layer_algorithmic(w, kept_tokens)
+    dom = max(("lse", "keyscore"), key=lambda s: stage_ms[s])
+    dom_ms = stage_ms[dom]
+    achieved = flops1 / (dom_ms / 1e3) / 1e12
+    roofline = {"bound": "tensor", "kernel": f"{dom}_kernel", "achieved": achieved,
+                "peak": tf_sust, "unit": "TFLOP/s", "frac": achieved / tf_sust,
+                "peak_source": f"{peak_src} bf16 sustained",
+                "traffic": traffic_record(f"{dom}_kernel", w.name),
+                "per_launch_ms": dom_ms,
+                "flops_per_launch": flops1}
+    t_layer_s = ms / L / 1e3
+    hbm_fused = {"algorithmic_bytes": read_b + write_b, "achieved_gbs": (read_b + write_b) / t_layer_s / 1e9,
+                 "peak_gbs": hbm_peak, "frac": (read_b + write_b) / t_layer_s / 1e9 / hbm_peak,
+                 "frac_of_nominal_8tbs": (read_b + write_b) / t_layer_s / 8e12,
+                 "peak_source": peak_src}
+
+    # ---- e2e: host buffers through the public API, copies inside the timed region
+    Le = max(1, min(args.e2e_layers, L))
+    hq = [tuple(t.cpu().pin_memory() for t in layers[l]) for l in range(Le)]
+    dq = [tuple(torch.empty_like(t) for t in layers[l]) for l in range(Le)]
+    host_out = [(torch.empty(o.idx.shape, dtype=o.idx.dtype, pin_memory=True),
+                 torch.empty(o.kc.shape, dtype=o.kc.dtype, pin_memory=True),
+                 torch.empty(o.vc.shape, dtype=o.vc.dtype, pin_memory=True),
+                 torch.empty(o.vqc.shape, dtype=o.vqc.dtype, pin_memory=True),
+                 torch.empty(o.gammac.shape, dtype=o.gammac.dtype, pin_memory=True))
+                for o in outs[:Le]]
+    h2d = sum(t.numel() * t.element_size() for l in range(Le) for t in hq[l])
+    d2h = sum(t.numel() * t.element_size() for l in range(Le) for t in host_out[l])
+
+    def e2e_step():
+        for l in range(Le):
+            for dst, src in zip(dq[l], hq[l]):
+                dst.copy_(src, non_blocking=True)
+            o = outs[l]
+            binding.compress(p, *dq[l], w.keep_ratio, w.budget, o, stream)
+            for dst, src in zip(host_out[l], (o.idx, o.kc, o.vc, o.vqc, o.gammac)):
+                dst.copy_(src, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    esteps = max(1, args.steps)
+    for _ in range(esteps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ems = e0.elapsed_time(e1) / esteps
+    if world > 1:
+        t = torch.tensor([ems], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ems = float(t.item())
+    e2e = {"value": w.n_total * Le * world / (ems / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "layers_per_step": Le,
+           "ms_per_step": ems}
+
+    clk = clocks.summary()
+    st = binding.tp_check_status(ws)
+    if st != 0:
+        raise RuntimeError(f"device status after timing: {binding.tp_status_string(st)}")
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        nh = args.cpu_sample_heads or w.n_heads_kv
+        heads = list(range(min(nh, w.n_heads_kv)))
+        cv, detail, used = oracle_sample(w, oracle_inputs(w), heads, cores)
+        cpu = {"value": cv, "unit": UNIT, "cores": used, "kind": "oracle", "sample": detail}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": w.name, "layers": L, "n_ctx": w.n_total, "guide_len": w.guide_len,
+                       "heads_q": w.n_heads_q, "heads_kv": w.n_heads_kv, "head_dim": w.head_dim,
+                       "keep_ratio": w.keep_ratio if w.budget < 0 else None,
+                       "budget": w.budget if w.budget >= 0 else None,
+                       "l2": "inputs larger than L2 (each layer's K+V exceeds 129 MB; layers use distinct buffers)",
+                       "parallelism": f"replicas{world}"},
+            "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms,
+            "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    from paper_2608_03276_gb300 import synth
+    w = synth.WORKLOADS[args.config]
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,209 @@
+/*
+ * taskpress.h - C ABI of the TaskPress prefill-time KV-cache compression path
+ * for GB300 (sm_103a).
+ *
+ * TaskPress (Sec. 3) keeps, for every KV head of a layer, the context tokens
+ * that a short task guide attends to most (Eq. 1), weighted by each token's
+ * per-token V quantisation scale (Eq. 2, Eq. 3), and evicts the rest with a
+ * uniform per-head budget (Sec. 4, "Eviction").  This library runs that step
+ * on one GPU: score, select, and compact the kept K/V into a reusable cache.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - All tensor pointers are DEVICE pointers to contiguous row-major memory,
+ *    owned by the caller.  The library allocates nothing and keeps no state
+ *    between calls apart from a cache of TMA descriptors (guarded by a mutex).
+ *  - bf16 tensors are passed as `const void*` (IEEE bfloat16 bit patterns).
+ *  - Shapes (d = head_dim, N = total tokens = doc_offsets[batch]):
+ *        Q guide   [batch, H_q, L_t, d]   bf16, post-RoPE guide queries
+ *        K, V      [H_kv, N, d]           bf16, documents packed along N
+ *        gamma     [H_kv, N]              fp32 per-token V scale
+ *        Vq        [H_kv, N, d]           int8 codes
+ *        scores    [H_kv, N]              fp32 combined scores s_i
+ *        idx       [batch, H_kv, cap]     int32, doc-local kept indices
+ *        Kc, Vc    [batch, H_kv, cap, d]  bf16 compressed cache
+ *        Vqc       [batch, H_kv, cap, d]  int8
+ *        gammac    [batch, H_kv, cap]     fp32
+ *    where cap = tp_kept_capacity(...).  Document b keeps k_b <= cap tokens;
+ *    slots k_b..cap-1 of its rows are filled with idx = -1 and zero bytes.
+ *  - Query head h belongs to KV head h / (H_q / H_kv) (contiguous groups).
+ *  - Every call takes a cudaStream_t (passed as void*; NULL = legacy default
+ *    stream), enqueues its kernels and returns without synchronising.
+ *    Launch errors are reported through the return code; errors raised while
+ *    the kernels run surface at the next synchronisation of the stream.
+ *  - Return value: TP_OK (0) or a negative TP_ERR_* code; outputs are
+ *    undefined after an error.
+ *  - Inputs must be finite.  NaN scores are ranked as 0 (never preferred).
+ */
+#ifndef TASKPRESS_H_
+#define TASKPRESS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define TP_OK 0
+#define TP_ERR_INVALID_ARG (-1)       /* null pointer, bad count, bad ratio     */
+#define TP_ERR_WORKSPACE (-2)         /* workspace missing or too small          */
+#define TP_ERR_UNSUPPORTED_SHAPE (-3) /* d not in {64,128}, even pool kernel, .. */
+#define TP_ERR_CUDA (-4)              /* a CUDA runtime/driver call failed       */
+#define TP_ERR_TIMEOUT (-5)           /* a device-side wait gave up (see below)  */
+
+/* Flags (tp_problem.flags). */
+#define TP_SCORE_KEY_ONLY 0x1u /* s_i = pooled key score only (Sec. 4.3.1 ablation) */
+
+/* Limits. */
+#define TP_MAX_BATCH 256   /* documents per call                              */
+#define TP_MAX_ROWS 512    /* G * L_t stacked guide rows per KV head          */
+
+/*
+ * One layer's compression problem.
+ *   n_heads_q, n_heads_kv : H_q, H_kv (H_q a multiple of H_kv)
+ *   head_dim              : d, 64 or 128
+ *   guide_len             : L_t, the task guide's token count (Sec. 3.2)
+ *   batch                 : number of documents packed along the token axis
+ *   doc_offsets           : HOST pointer to batch+1 non-decreasing int64
+ *                           offsets, doc_offsets[0] = 0; document b owns
+ *                           tokens [doc_offsets[b], doc_offsets[b+1]).
+ *   pool_kernel           : K of Eq. 1's average pooling; odd, >= 1 (default 5)
+ *   quant_bits            : b of Eq. 2; only 8 is supported
+ *   softmax_scale         : logit scale; <= 0 means 1/sqrt(d)
+ *   flags                 : TP_SCORE_KEY_ONLY or 0
+ */
+typedef struct tp_problem {
+  int32_t n_heads_q;
+  int32_t n_heads_kv;
+  int32_t head_dim;
+  int32_t guide_len;
+  int32_t batch;
+  int32_t pool_kernel;
+  int32_t quant_bits;
+  float softmax_scale;
+  uint32_t flags;
+  const int64_t* doc_offsets;
+} tp_problem;
+
+/*
+ * Tokens kept per head for a keep ratio (Sec. 4: the eviction ratio is the
+ * pruned share, so keep = 1 - eviction).  Returns ceil(ratio*n - 1e-9*n)
+ * clamped to [0, n] (the small offset keeps exact decimal products such as
+ * 0.07*100 from rounding up), or -1 when n < 0 or the ratio is not in [0, 1].
+ */
+int64_t tp_budget(int64_t n, double keep_ratio);
+
+/*
+ * Capacity of the per-(document, head) output rows: max over documents of
+ * k_b, where k_b = min(budget, n_b) when budget >= 0, else
+ * tp_budget(n_b, keep_ratio).  Returns -1 on invalid arguments.
+ */
+int64_t tp_kept_capacity(const tp_problem* p, double keep_ratio, int64_t budget);
+
+/*
+ * Bytes of device workspace that tp_guide_scores, tp_select and
+ * tp_compress_layer need for this problem (0 on invalid arguments).  The
+ * workspace is caller-owned scratch, 256-byte aligned, with no required
+ * contents; it must not be shared by calls that may overlap on the GPU.
+ */
+size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget);
+
+/*
+ * Eq. 2 (Sec. 3.3) for every token of V: gamma_i = max_c |v_ic| / 127 (fp32,
+ * IEEE round-to-nearest division) and int8 codes q_ic = clamp(rint(v_ic /
+ * gamma_i), -127, 127) (IEEE fp32 quotient, round-half-even; gamma_i = 0
+ * gives q_i = 0).  v: [H_kv, N, d] bf16 in; vq: [H_kv, N, d] int8 out (may be
+ * NULL to compute gamma only); gamma: [H_kv, N] fp32 out.
+ */
+int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, void* stream);
+
+/*
+ * Combined importance s_i of every context token (Sec. 3.2-3.4):
+ *   A = softmax over the context of sigma * Q_guide K^T, per guide row
+ *       (the guide-to-context block of the prefill attention map, Sec. 3.2),
+ *   s_key_i = (1/K) sum_{k=-K/2..K/2} (1/G) sum_{rows r of the group} A[r, i+k]
+ *       (Eq. 1; rows are the G*L_t guide rows of the KV head's query heads,
+ *       terms outside the document are zero),
+ *   s_i = s_key_i * gamma_i (Eq. 3), or s_key_i with TP_SCORE_KEY_ONLY.
+ * q: [batch, H_q, L_t, d] bf16; k: [H_kv, N, d] bf16; gamma: [H_kv, N] fp32
+ * (may be NULL only with TP_SCORE_KEY_ONLY); scores: [H_kv, N] fp32 out.
+ * ws / ws_bytes: workspace of at least tp_workspace_bytes(p, 0, 0).
+ */
+int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const float* gamma,
+                    float* scores, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Stage 1 of the scores (Sec. 3.2): the softmax normaliser of every guide row,
+ *   lse[b, h, r] = log sum_{i in document b} exp(sigma * q_r . k_i)
+ * for the M = G*L_t stacked guide rows r of KV head h (rows ordered query
+ * head-major within the group, then guide token).  q, k as in tp_guide_scores;
+ * lse: [batch, H_kv, M] fp32 out (natural log).  Empty documents are skipped.
+ * ws / ws_bytes: workspace of at least tp_workspace_bytes(p, 0, 0).
+ */
+int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
+                 size_t ws_bytes, void* stream);
+
+/*
+ * Stage 2 of the scores (Sec. 3.2, Eq. 1's inner sums): given the row
+ * normalisers `lse` ([batch, H_kv, M] fp32, natural log, e.g. from
+ * tp_guide_lse or from the caller's own prefill attention), writes the
+ * unpooled key score of every context token,
+ *   key_scores[h, off_b + i] = (1/G) sum_r exp(sigma * q_r . k_i - lse[b, h, r]).
+ * Needs no workspace.  key_scores: [H_kv, N] fp32 out.
+ */
+int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
+                        float* key_scores, void* stream);
+
+/*
+ * Top-budget selection per (document, KV head) (Sec. 3.4; Sec. 4 uniform
+ * per-head budget): the k_b largest scores of each document's rows, equal
+ * scores resolved towards the lower token index, -0 treated as +0, NaN as 0.
+ * scores: [H_kv, N] fp32; idx: [batch, H_kv, cap] int32 out, doc-local,
+ * strictly ascending in each row, then -1 padding.  keep_ratio / budget as in
+ * tp_kept_capacity.  ws: tp_workspace_bytes(p, keep_ratio, budget) bytes.
+ */
+int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64_t budget,
+              int32_t* idx, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Order-preserving compaction of the kept tokens (Sec. 3.1: the compressed
+ * cache of the selected index subset).  For every (document b, head h, slot t)
+ * with j = idx[b,h,t] >= 0:  Kc = K[h, off_b + j], Vc = V[h, off_b + j],
+ * Vqc = Eq. 2 codes of that V row with scale gamma[h, off_b + j],
+ * gammac = gamma[h, off_b + j]; slots with idx = -1 are zero-filled.
+ * Any of kc, vc, vqc, gammac may be NULL to skip that output.
+ */
+int tp_compact(const tp_problem* p, const void* k, const void* v, const float* gamma,
+               const int32_t* idx, double keep_ratio, int64_t budget, void* kc, void* vc,
+               int8_t* vqc, float* gammac, void* stream);
+
+/*
+ * The fused per-layer path: Eq. 2 scales, Eq. 1 / Eq. 3 scores, per-head
+ * top-budget selection and compaction, all on `stream` with no host
+ * synchronisation.  Outputs as in tp_select and tp_compact; `scores` and
+ * `gamma` ([H_kv, N] fp32) are optional outputs (NULL to skip).
+ */
+int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
+                      double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
+                      int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
+                      size_t ws_bytes, void* stream);
+
+/*
+ * Synchronises `stream`, then reads the device status word that the kernels of
+ * the last call on this workspace left.  Every device-side wait in the
+ * kernels is bounded; one that gives up records TP_ERR_TIMEOUT there and the
+ * kernel returns early (its outputs are then undefined).  Returns TP_OK,
+ * TP_ERR_TIMEOUT, or TP_ERR_CUDA if the synchronisation itself failed.
+ */
+int tp_check_status(const void* ws, size_t ws_bytes, void* stream);
+
+/* Human-readable name of a status code (static storage). */
+const char* tp_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TASKPRESS_H_ */

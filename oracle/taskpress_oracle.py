@@ -113,6 +113,13 @@ def guide_attention(q_rows: np.ndarray, k_ctx: np.ndarray, sigma: float) -> np.n
     return e / z
 
 
+def guide_lse(q_rows: np.ndarray, k_ctx: np.ndarray, sigma: float) -> np.ndarray:
+    """lse[r] = log sum_i exp(sigma * q_r . k_i): each guide row's softmax normaliser."""
+    x = (q_rows @ k_ctx.T) * sigma
+    m = np.max(x, axis=1)
+    return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))
+
+
 def key_scores(q_group: np.ndarray, k_ctx: np.ndarray, sigma: float) -> np.ndarray:
     """Unpooled key importance of every context token for one KV head.
 
@@ -190,7 +197,8 @@ def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
         out["k"][b] = kb
         for h in heads:
             qg = q[b, h * g:(h + 1) * g]
-            s_key = key_scores(qg, k_all[h, lo:hi], sigma)
+            # an empty document has no context tokens: nothing to score or keep
+            s_key = key_scores(qg, k_all[h, lo:hi], sigma) if n > 0 else np.zeros(0)
             s = combine(pool(s_key, pool_kernel), gamma[h, lo:hi], key_only)
             out["key"][(b, h)] = s_key
             out["scores"][(b, h)] = s

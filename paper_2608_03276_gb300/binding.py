@@ -1,0 +1,292 @@
+"""ctypes binding of libtaskpress.so (include/taskpress.h), same names as the C ABI.
+
+Argument marshalling only: every wrapper checks the torch tensors it is given
+(device, dtype, contiguity, size), passes raw pointers and the current CUDA
+stream, and raises on a non-zero status.  All arithmetic runs in the library's
+kernels; there is no fallback when the library is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_float, c_int, c_int32, c_int64, c_size_t, c_uint32, c_void_p
+from typing import Optional, Sequence
+
+import numpy as np
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libtaskpress.so")
+
+TP_OK = 0
+TP_ERR_INVALID_ARG = -1
+TP_ERR_WORKSPACE = -2
+TP_ERR_UNSUPPORTED_SHAPE = -3
+TP_ERR_CUDA = -4
+TP_ERR_TIMEOUT = -5
+TP_SCORE_KEY_ONLY = 0x1
+TP_MAX_BATCH = 256
+TP_MAX_ROWS = 512
+
+#: every symbol include/taskpress.h declares
+EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
+           "tp_guide_scores", "tp_guide_lse", "tp_guide_key_scores", "tp_select", "tp_compact",
+           "tp_compress_layer", "tp_check_status", "tp_status_string")
+
+
+class TpProblem(ctypes.Structure):
+    _fields_ = [
+        ("n_heads_q", c_int32),
+        ("n_heads_kv", c_int32),
+        ("head_dim", c_int32),
+        ("guide_len", c_int32),
+        ("batch", c_int32),
+        ("pool_kernel", c_int32),
+        ("quant_bits", c_int32),
+        ("softmax_scale", c_float),
+        ("flags", c_uint32),
+        ("doc_offsets", POINTER(c_int64)),
+    ]
+
+
+class TaskPressError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {status} ({_status_string(status)})")
+
+
+_lib = None
+
+
+def load(path: Optional[str] = None):
+    """Loads libtaskpress.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libtaskpress.so not built ({p}); run __graft_entry__.build()")
+    lib = ctypes.CDLL(p)
+    lib.tp_budget.restype = c_int64
+    lib.tp_budget.argtypes = [c_int64, c_double]
+    lib.tp_kept_capacity.restype = c_int64
+    lib.tp_kept_capacity.argtypes = [POINTER(TpProblem), c_double, c_int64]
+    lib.tp_workspace_bytes.restype = c_size_t
+    lib.tp_workspace_bytes.argtypes = [POINTER(TpProblem), c_double, c_int64]
+    lib.tp_quantize_v.restype = c_int
+    lib.tp_quantize_v.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p]
+    lib.tp_guide_scores.restype = c_int
+    lib.tp_guide_scores.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
+                                    c_void_p, c_size_t, c_void_p]
+    lib.tp_guide_lse.restype = c_int
+    lib.tp_guide_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
+                                 c_size_t, c_void_p]
+    lib.tp_guide_key_scores.restype = c_int
+    lib.tp_guide_key_scores.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
+                                        c_void_p]
+    lib.tp_select.restype = c_int
+    lib.tp_select.argtypes = [POINTER(TpProblem), c_void_p, c_double, c_int64, c_void_p, c_void_p,
+                              c_size_t, c_void_p]
+    lib.tp_compact.restype = c_int
+    lib.tp_compact.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p, c_double,
+                               c_int64, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]
+    lib.tp_compress_layer.restype = c_int
+    lib.tp_compress_layer.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_double,
+                                      c_int64, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                      c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
+    lib.tp_check_status.restype = c_int
+    lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
+    lib.tp_status_string.restype = ctypes.c_char_p
+    lib.tp_status_string.argtypes = [c_int]
+    _lib = lib
+    return lib
+
+
+def _status_string(status: int) -> str:
+    try:
+        return load().tp_status_string(status).decode()
+    except Exception:
+        return "?"
+
+
+class Problem:
+    """A tp_problem plus the host offsets array it points to (kept alive here)."""
+
+    def __init__(self, n_heads_q: int, n_heads_kv: int, head_dim: int, guide_len: int,
+                 doc_offsets: Sequence[int], pool_kernel: int = 5, quant_bits: int = 8,
+                 softmax_scale: float = 0.0, flags: int = 0):
+        self.offsets = np.ascontiguousarray(np.asarray(doc_offsets, dtype=np.int64))
+        self.c = TpProblem(n_heads_q, n_heads_kv, head_dim, guide_len, len(self.offsets) - 1,
+                           pool_kernel, quant_bits, softmax_scale, flags,
+                           self.offsets.ctypes.data_as(POINTER(c_int64)))
+
+    @property
+    def n_total(self) -> int:
+        return int(self.offsets[-1])
+
+    @property
+    def batch(self) -> int:
+        return len(self.offsets) - 1
+
+    def ref(self):
+        return ctypes.byref(self.c)
+
+
+def _ptr(t, dtype=None, numel=None, name="tensor", nullable=False):
+    if t is None:
+        if nullable:
+            return None
+        raise ValueError(f"{name} is required")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name} must have {numel} elements, got {t.numel()}")
+    return c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return c_void_p(s.cuda_stream)
+
+
+def _check(fn: str, status: int):
+    if status != TP_OK:
+        raise TaskPressError(fn, status)
+
+
+def tp_budget(n: int, keep_ratio: float) -> int:
+    return int(load().tp_budget(n, keep_ratio))
+
+
+def tp_kept_capacity(p: Problem, keep_ratio: float, budget: int) -> int:
+    return int(load().tp_kept_capacity(p.ref(), keep_ratio, budget))
+
+
+def tp_workspace_bytes(p: Problem, keep_ratio: float = 0.0, budget: int = 0) -> int:
+    return int(load().tp_workspace_bytes(p.ref(), keep_ratio, budget))
+
+
+def tp_quantize_v(p: Problem, v, vq, gamma, stream=None):
+    import torch
+    hkv, d, n = p.c.n_heads_kv, p.c.head_dim, p.n_total
+    _check("tp_quantize_v", load().tp_quantize_v(
+        p.ref(), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
+        _ptr(vq, torch.int8, hkv * n * d, "vq", nullable=True),
+        _ptr(gamma, torch.float32, hkv * n, "gamma"), _stream(stream)))
+
+
+def tp_guide_scores(p: Problem, q, k, gamma, scores, ws, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    _check("tp_guide_scores", load().tp_guide_scores(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
+        _ptr(scores, torch.float32, hkv * n, "scores"),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_guide_lse(p: Problem, q, k, lse, ws, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    rows = (hq // hkv) * lt
+    _check("tp_guide_lse", load().tp_guide_lse(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_guide_key_scores(p: Problem, q, k, lse, key_scores, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    rows = (hq // hkv) * lt
+    _check("tp_guide_key_scores", load().tp_guide_key_scores(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
+        _ptr(key_scores, torch.float32, hkv * n, "key_scores"), _stream(stream)))
+
+
+def tp_select(p: Problem, scores, keep_ratio: float, budget: int, idx, ws, stream=None):
+    import torch
+    hkv, n = p.c.n_heads_kv, p.n_total
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    _check("tp_select", load().tp_select(
+        p.ref(), _ptr(scores, torch.float32, hkv * n, "scores"), keep_ratio, budget,
+        _ptr(idx, torch.int32, p.batch * hkv * cap, "idx", nullable=cap == 0),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_compact(p: Problem, k, v, gamma, idx, keep_ratio: float, budget: int, kc, vc, vqc, gammac,
+               stream=None):
+    import torch
+    hkv, d, n = p.c.n_heads_kv, p.c.head_dim, p.n_total
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+    _check("tp_compact", load().tp_compact(
+        p.ref(), _ptr(k, torch.bfloat16, hkv * n * d, "k"), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
+        _ptr(gamma, torch.float32, hkv * n, "gamma"), _ptr(idx, torch.int32, m, "idx"),
+        keep_ratio, budget,
+        _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
+        _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
+        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _ptr(gammac, torch.float32, m, "gammac", nullable=True), _stream(stream)))
+
+
+def tp_compress_layer(p: Problem, q, k, v, keep_ratio: float, budget: int, idx, kc, vc, vqc, gammac,
+                      scores, gamma, ws, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+    _check("tp_compress_layer", load().tp_compress_layer(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
+        keep_ratio, budget,
+        _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
+        _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
+        _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
+        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _ptr(gammac, torch.float32, m, "gammac", nullable=True),
+        _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_check_status(ws, stream=None) -> int:
+    return int(load().tp_check_status(c_void_p(ws.data_ptr()), ws.numel(), _stream(stream)))
+
+
+def tp_status_string(status: int) -> str:
+    return _status_string(status)
+
+
+class CompressOutputs:
+    """Device buffers for one tp_compress_layer call (plumbing: torch allocations)."""
+
+    def __init__(self, p: Problem, keep_ratio: float, budget: int, device, with_scores=True):
+        import torch
+        hkv, d, n = p.c.n_heads_kv, p.c.head_dim, p.n_total
+        self.cap = tp_kept_capacity(p, keep_ratio, budget)
+        if self.cap < 0:
+            raise ValueError("invalid keep ratio / budget")
+        shp = (p.batch, hkv, self.cap)
+        self.idx = torch.empty(shp, dtype=torch.int32, device=device)
+        self.kc = torch.empty(shp + (d,), dtype=torch.bfloat16, device=device)
+        self.vc = torch.empty(shp + (d,), dtype=torch.bfloat16, device=device)
+        self.vqc = torch.empty(shp + (d,), dtype=torch.int8, device=device)
+        self.gammac = torch.empty(shp, dtype=torch.float32, device=device)
+        self.scores = torch.empty((hkv, n), dtype=torch.float32, device=device) if with_scores else None
+        self.gamma = torch.empty((hkv, n), dtype=torch.float32, device=device) if with_scores else None
+        self.ws = torch.empty(max(256, tp_workspace_bytes(p, keep_ratio, budget)), dtype=torch.uint8,
+                              device=device)
+
+
+def compress(p: Problem, q, k, v, keep_ratio: float, budget: int, out: CompressOutputs, stream=None):
+    tp_compress_layer(p, q, k, v, keep_ratio, budget, out.idx, out.kc, out.vc, out.vqc, out.gammac,
+                      out.scores, out.gamma, out.ws, stream)
+    return out

@@ -1,0 +1,488 @@
+// C ABI of the TaskPress compression path (include/taskpress.h): argument
+// checks, launch planning, workspace carving, TMA descriptors and the kernel
+// sequence of each entry point.  Nothing here allocates device memory.
+#include <math.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "tp_internal.h"
+
+namespace tp {
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr int kMaxSmem = 232448;  // opt-in dynamic shared memory per block on sm_100-class GPUs
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+struct Plan {
+  int hq, hkv, d, lt, g, batch;
+  int64_t n_total;
+  int64_t off[kMaxBatch + 1];
+  int rows, nrb, rows_pad, rows_mma;
+  int tiles_per_cta, grid_x;
+  int32_t cta[kMaxBatch + 1];
+  int stages1, stages2;
+  size_t smem1, smem2;
+  float c2, inv_group;
+  int32_t kept[kMaxBatch];
+  int64_t cap;
+  // workspace offsets
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
+};
+
+int num_sms() {
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms > 0 ? sms : 148;
+}
+
+int64_t kept_for(int64_t n, double ratio, int64_t budget) {
+  if (budget >= 0) return budget < n ? budget : n;
+  return tp_budget(n, ratio);
+}
+
+// Validates the problem and fills the plan.  `need_select` adds the kept
+// counts (ratio/budget must then be valid).
+int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_select, Plan* P) {
+  if (!p || !P) return TP_ERR_INVALID_ARG;
+  if (p->n_heads_kv <= 0 || p->n_heads_q <= 0 || p->n_heads_q % p->n_heads_kv != 0)
+    return TP_ERR_INVALID_ARG;
+  if (p->guide_len <= 0 || p->batch <= 0 || p->batch > kMaxBatch || !p->doc_offsets)
+    return TP_ERR_INVALID_ARG;
+  if (p->head_dim != 64 && p->head_dim != 128) return TP_ERR_UNSUPPORTED_SHAPE;
+  if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0) return TP_ERR_UNSUPPORTED_SHAPE;
+  if (p->quant_bits != 8) return TP_ERR_UNSUPPORTED_SHAPE;
+  if (p->flags & ~TP_SCORE_KEY_ONLY) return TP_ERR_INVALID_ARG;
+  memset(P, 0, sizeof(*P));
+  P->hq = p->n_heads_q;
+  P->hkv = p->n_heads_kv;
+  P->d = p->head_dim;
+  P->lt = p->guide_len;
+  P->g = p->n_heads_q / p->n_heads_kv;
+  P->batch = p->batch;
+  if (p->doc_offsets[0] != 0) return TP_ERR_INVALID_ARG;
+  for (int b = 0; b <= p->batch; ++b) {
+    P->off[b] = p->doc_offsets[b];
+    if (b > 0 && (P->off[b] < P->off[b - 1] || P->off[b] - P->off[b - 1] > INT32_MAX / 2))
+      return TP_ERR_INVALID_ARG;
+  }
+  P->n_total = P->off[p->batch];
+  if (P->n_total > (int64_t(1) << 31) - 256) return TP_ERR_UNSUPPORTED_SHAPE;
+  const int64_t rows = int64_t(P->g) * P->lt;
+  if (rows > TP_MAX_ROWS) return TP_ERR_UNSUPPORTED_SHAPE;
+  P->rows = static_cast<int>(rows);
+  const int rb = (P->rows + 127) / 128;
+  P->nrb = rb <= 1 ? 1 : (rb <= 2 ? 2 : 4);
+  P->rows_pad = 128 * P->nrb;
+  P->rows_mma = (P->rows + 31) / 32 * 32;
+  const double sigma = p->softmax_scale > 0 ? double(p->softmax_scale) : 1.0 / sqrt(double(P->d));
+  P->c2 = static_cast<float>(sigma * 1.4426950408889634);
+  P->inv_group = 1.0f / static_cast<float>(P->g);
+
+  // Key tiles per CTA: the smallest T whose CTA count fits one wave.
+  const int sms = num_sms();
+  int64_t tiles_total = 0;
+  for (int b = 0; b < P->batch; ++b) tiles_total += (P->off[b + 1] - P->off[b] + 127) / 128;
+  tiles_total *= P->hkv;
+  int64_t T = tiles_total > 0 ? (tiles_total + sms - 1) / sms : 1;
+  if (T < 1) T = 1;
+  for (int iter = 0; iter < 64; ++iter) {
+    int64_t ctas = 0;
+    for (int b = 0; b < P->batch; ++b) ctas += ((P->off[b + 1] - P->off[b] + 127) / 128 + T - 1) / T;
+    if (ctas * P->hkv <= sms) break;
+    ++T;
+  }
+  P->tiles_per_cta = static_cast<int>(T);
+  P->cta[0] = 0;
+  for (int b = 0; b < P->batch; ++b) {
+    const int64_t tiles = (P->off[b + 1] - P->off[b] + 127) / 128;
+    P->cta[b + 1] = P->cta[b] + static_cast<int32_t>((tiles + T - 1) / T);
+  }
+  P->grid_x = P->cta[P->batch];
+
+  // Deepest K-tile ring that fits next to the resident guide block.
+  P->stages1 = 4;
+  while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
+  P->stages2 = 4;
+  while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
+  P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
+  P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
+  if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
+
+  P->cap = 0;
+  if (need_select) {
+    for (int b = 0; b < P->batch; ++b) {
+      const int64_t k = kept_for(P->off[b + 1] - P->off[b], ratio, budget);
+      if (k < 0) return TP_ERR_INVALID_ARG;
+      P->kept[b] = static_cast<int32_t>(k);
+      if (k > P->cap) P->cap = k;
+    }
+  }
+
+  size_t o = 0;
+  P->ws_status = o;
+  o = align_up(o + sizeof(int) * (1 + size_t(P->hkv) * P->batch));
+  P->ws_partials = o;
+  o = align_up(o + sizeof(float2) * size_t(P->hkv) * P->grid_x * P->rows_pad);
+  P->ws_lse = o;
+  o = align_up(o + sizeof(float) * size_t(P->batch) * P->hkv * P->rows);
+  P->ws_skey = o;
+  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
+  P->ws_gamma = o;
+  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
+  P->ws_keys = o;
+  o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
+  P->ws_total = o;
+  return TP_OK;
+}
+
+// --- TMA descriptors ---------------------------------------------------------
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  return fn;
+}
+
+// 3-D bf16 view {d, rows, planes} with a {64, box_rows, 1} box, 128-byte swizzle.
+bool encode_3d(CUtensorMap* map, const void* base, int d, int64_t rows, int64_t planes,
+               int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(rows), cuuint64_t(planes)};
+  cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(d) * 2 * cuuint64_t(rows)};
+  cuuint32_t box[3] = {64, cuuint32_t(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15) == 0; }
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? TP_OK : TP_ERR_CUDA; }
+
+bool encode_maps(const Plan& P, const void* q, const void* k, CUtensorMap* tmk, CUtensorMap* tmq) {
+  return encode_3d(tmk, k, P.d, P.n_total, P.hkv, 128) &&
+         encode_3d(tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv,
+                   P.rows_pad < 256 ? P.rows_pad : 256);
+}
+
+DocTable doc_table(const Plan& P) {
+  DocTable docs;
+  memset(&docs, 0, sizeof(docs));
+  docs.batch = P.batch;
+  for (int b = 0; b <= P.batch; ++b) {
+    docs.off[b] = P.off[b];
+    docs.cta[b] = P.cta[b];
+  }
+  return docs;
+}
+
+// Pass 1: row normalisers into `lse` ([batch, H_kv, rows]).  The counters and
+// the status word at the head of the workspace must be zero.
+int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, float* lse, char* ws,
+            cudaStream_t s) {
+  int* status = reinterpret_cast<int*>(ws + P.ws_status);
+  LseParams lp;
+  memset(&lp, 0, sizeof(lp));
+  lp.docs = doc_table(P);
+  lp.n_heads_kv = P.hkv;
+  lp.rows = P.rows;
+  lp.rows_pad = P.rows_pad;
+  lp.nrb = P.nrb;
+  lp.tiles_per_cta = P.tiles_per_cta;
+  lp.stages = P.stages1;
+  lp.c2 = P.c2;
+  lp.partials = reinterpret_cast<float2*>(ws + P.ws_partials);
+  lp.lse = lse;
+  lp.counters = status + 1;
+  lp.status = status;
+  return cuda_status(launch_lse(tmk, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
+}
+
+// Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
+int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const float* lse,
+                 float* skey, int* status, cudaStream_t s) {
+  KeyScoreParams kp;
+  memset(&kp, 0, sizeof(kp));
+  kp.docs = doc_table(P);
+  kp.n_heads_kv = P.hkv;
+  kp.rows = P.rows;
+  kp.rows_pad = P.rows_pad;
+  kp.rows_mma = P.rows_mma;
+  kp.tiles_per_cta = P.tiles_per_cta;
+  kp.stages = P.stages2;
+  kp.c2 = P.c2;
+  kp.inv_group = P.inv_group;
+  kp.n_total = P.n_total;
+  kp.lse = lse;
+  kp.skey = skey;
+  kp.status = status;
+  return cuda_status(launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, s));
+}
+
+// Both scoring passes; leaves the unpooled key scores in the workspace.
+int run_scoring(const Plan& P, const void* q, const void* k, char* ws, cudaStream_t s) {
+  if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  CUtensorMap tmk, tmq;
+  if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+  float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
+  int st = run_lse(P, tmk, tmq, lse, ws, s);
+  if (st != TP_OK) return st;
+  return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
+                      reinterpret_cast<int*>(ws + P.ws_status), s);
+}
+
+void fill_select(const Plan& P, SelectParams* sp) {
+  memset(sp, 0, sizeof(*sp));
+  for (int b = 0; b <= P.batch; ++b) sp->off[b] = P.off[b];
+  for (int b = 0; b < P.batch; ++b) sp->kept[b] = P.kept[b];
+  sp->batch = P.batch;
+  sp->n_heads_kv = P.hkv;
+  sp->n_total = P.n_total;
+  sp->cap = P.cap;
+  sp->pool_kernel = 1;
+}
+
+void fill_gather(const Plan& P, GatherParams* gp) {
+  memset(gp, 0, sizeof(*gp));
+  for (int b = 0; b <= P.batch; ++b) gp->off[b] = P.off[b];
+  gp->batch = P.batch;
+  gp->n_heads_kv = P.hkv;
+  gp->head_dim = P.d;
+  gp->n_total = P.n_total;
+  gp->cap = P.cap;
+  gp->qmax = 127.0f;
+}
+
+}  // namespace
+}  // namespace tp
+
+using namespace tp;
+
+extern "C" {
+
+int64_t tp_budget(int64_t n, double keep_ratio) {
+  if (n < 0 || !(keep_ratio >= 0.0 && keep_ratio <= 1.0)) return -1;
+  const double dn = static_cast<double>(n);
+  const double prod = keep_ratio * dn;
+  const double slack = 1e-9 * dn;
+  double k = ceil(prod - slack);
+  if (k < 0) k = 0;
+  if (k > dn) k = dn;
+  return static_cast<int64_t>(k);
+}
+
+int64_t tp_kept_capacity(const tp_problem* p, double keep_ratio, int64_t budget) {
+  Plan P;
+  if (make_plan(p, keep_ratio, budget, true, &P) != TP_OK) return -1;
+  return P.cap;
+}
+
+size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget) {
+  Plan P;
+  const bool sel = budget >= 0 || (keep_ratio >= 0.0 && keep_ratio <= 1.0);
+  if (make_plan(p, keep_ratio, budget, sel, &P) != TP_OK) return 0;
+  return P.ws_total;
+}
+
+int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  if (!v || !gamma || !aligned16(v) || (vq && (reinterpret_cast<uintptr_t>(vq) & 7)))
+    return TP_ERR_INVALID_ARG;
+  return cuda_status(launch_vquant(static_cast<const uint16_t*>(v), vq, gamma,
+                                   int64_t(P.hkv) * P.n_total, P.d, 127.0f, num_sms(),
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const float* gamma,
+                    float* scores, void* ws, size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  const bool key_only = (p->flags & TP_SCORE_KEY_ONLY) != 0;
+  if (!q || !k || !scores || (!gamma && !key_only) || !aligned16(q) || !aligned16(k))
+    return TP_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
+    return TP_ERR_CUDA;
+  st = run_scoring(P, q, k, w, s);
+  if (st != TP_OK) return st;
+  SelectParams sp;
+  fill_select(P, &sp);
+  sp.pool_kernel = p->pool_kernel;
+  sp.key_only = key_only ? 1 : 0;
+  sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
+  sp.gamma = gamma;
+  sp.scores_out = scores;
+  sp.keys = reinterpret_cast<uint32_t*>(w + P.ws_keys);
+  // k = 0 for every document: the select kernel only forms the scores.
+  for (int b = 0; b < P.batch; ++b) sp.kept[b] = 0;
+  sp.cap = 0;
+  sp.idx = nullptr;
+  return cuda_status(launch_select(sp, s));
+}
+
+int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
+                 size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k || !lse || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
+    return TP_ERR_CUDA;
+  if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  CUtensorMap tmk, tmq;
+  if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+  return run_lse(P, tmk, tmq, lse, w, s);
+}
+
+int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
+                        float* key_scores, void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k || !lse || !key_scores || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
+  if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  CUtensorMap tmk, tmq;
+  if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+  return run_keyscore(P, tmk, tmq, lse, key_scores, nullptr, static_cast<cudaStream_t>(stream));
+}
+
+int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64_t budget,
+              int32_t* idx, void* ws, size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (!scores || (!idx && P.cap > 0)) return TP_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  SelectParams sp;
+  fill_select(P, &sp);
+  sp.scores_in = scores;
+  sp.keys = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + P.ws_keys);
+  sp.idx = idx;
+  return cuda_status(launch_select(sp, static_cast<cudaStream_t>(stream)));
+}
+
+int tp_compact(const tp_problem* p, const void* k, const void* v, const float* gamma,
+               const int32_t* idx, double keep_ratio, int64_t budget, void* kc, void* vc,
+               int8_t* vqc, float* gammac, void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (P.cap == 0) return TP_OK;
+  if (!k || !v || !gamma || !idx || !aligned16(k) || !aligned16(v)) return TP_ERR_INVALID_ARG;
+  if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
+      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
+    return TP_ERR_INVALID_ARG;
+  GatherParams gp;
+  fill_gather(P, &gp);
+  gp.k = static_cast<const uint16_t*>(k);
+  gp.v = static_cast<const uint16_t*>(v);
+  gp.gamma = gamma;
+  gp.idx = idx;
+  gp.kc = static_cast<uint16_t*>(kc);
+  gp.vc = static_cast<uint16_t*>(vc);
+  gp.vqc = vqc;
+  gp.gammac = gammac;
+  return cuda_status(launch_gather(gp, static_cast<cudaStream_t>(stream)));
+}
+
+int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
+                      double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
+                      int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
+                      size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k || !v || (!idx && P.cap > 0) || !aligned16(q) || !aligned16(k) || !aligned16(v))
+    return TP_ERR_INVALID_ARG;
+  if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
+      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
+    return TP_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
+  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
+    return TP_ERR_CUDA;
+  cudaError_t e = launch_vquant(static_cast<const uint16_t*>(v), nullptr, g,
+                                int64_t(P.hkv) * P.n_total, P.d, 127.0f, num_sms(), s);
+  if (e != cudaSuccess) return TP_ERR_CUDA;
+  st = run_scoring(P, q, k, w, s);
+  if (st != TP_OK) return st;
+  SelectParams sp;
+  fill_select(P, &sp);
+  sp.pool_kernel = p->pool_kernel;
+  sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
+  sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
+  sp.gamma = g;
+  sp.scores_out = scores;
+  sp.keys = reinterpret_cast<uint32_t*>(w + P.ws_keys);
+  sp.idx = idx;
+  e = launch_select(sp, s);
+  if (e != cudaSuccess) return TP_ERR_CUDA;
+  if (P.cap == 0) return TP_OK;
+  GatherParams gp;
+  fill_gather(P, &gp);
+  gp.k = static_cast<const uint16_t*>(k);
+  gp.v = static_cast<const uint16_t*>(v);
+  gp.gamma = g;
+  gp.idx = idx;
+  gp.kc = static_cast<uint16_t*>(kc);
+  gp.vc = static_cast<uint16_t*>(vc);
+  gp.vqc = vqc;
+  gp.gammac = gammac;
+  return cuda_status(launch_gather(gp, s));
+}
+
+int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {
+  if (!ws || ws_bytes < sizeof(int)) return TP_ERR_WORKSPACE;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return TP_ERR_CUDA;
+  int status = 0;
+  if (cudaMemcpy(&status, ws, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return TP_ERR_CUDA;
+  return status == 0 ? TP_OK : status;
+}
+
+const char* tp_status_string(int status) {
+  switch (status) {
+    case TP_OK: return "ok";
+    case TP_ERR_INVALID_ARG: return "invalid argument";
+    case TP_ERR_WORKSPACE: return "workspace missing or too small";
+    case TP_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+    case TP_ERR_CUDA: return "CUDA error";
+    case TP_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

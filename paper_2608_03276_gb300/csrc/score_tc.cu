@@ -1,0 +1,506 @@
+// Guide-to-context scoring on tcgen05 tensor cores (Sec. 3.2, Eq. 1).
+//
+// The guide block of one KV head (M = G*L_t stacked query rows, at most 512)
+// against the document's keys is a dense M x n x d contraction.  Exact
+// per-row softmax normalisation needs every row's log-sum-exp before any
+// column (per-key) sum can be formed, so the scores take two passes:
+//
+//   pass 1 (lse_kernel)      D[row, key] = Q K^T in TMEM, one thread per guide
+//                            row keeps a running (max, sum of 2^x) over the
+//                            CTA's key tiles; the last CTA of a (document,
+//                            head) merges the partials into lse[row].
+//   pass 2 (keyscore_kernel) D[key, row] = K Q^T in TMEM (keys on lanes), one
+//                            thread per key sums exp(x*sigma - lse[row]) over all
+//                            rows of the group: s_key[key] (mean over G).
+//
+// Both passes stream 128-key tiles of K with TMA (128-byte swizzle) through a
+// ring of shared-memory stages; one thread issues the MMAs; four epilogue
+// warpgroups drain TMEM.  Warp roles per CTA (20 warps):
+//   warp 0  TMA producer      warp 1  MMA issuer
+//   warp 2  TMEM owner        warp 3  idle
+//   warps 4-19  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
+#include <math.h>
+
+#include "tp_device.cuh"
+
+namespace tp {
+
+namespace {
+
+constexpr int kThreads = 640;
+constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
+
+struct ScoreSmem {
+  uint32_t q, k, bars, misc, extra, total;
+};
+
+// Byte offsets inside the (1024-aligned) dynamic shared memory.
+__host__ __device__ inline ScoreSmem score_layout(int head_dim, int rows_pad, int stages,
+                                                  uint32_t extra_bytes) {
+  ScoreSmem L;
+  const int nkh = head_dim / 64;
+  L.q = 0;
+  L.k = static_cast<uint32_t>(nkh * rows_pad * 128);
+  L.bars = L.k + static_cast<uint32_t>(stages) * nkh * kHalfTileBytes;
+  L.misc = L.bars + static_cast<uint32_t>(2 * stages + 16) * 8;
+  L.extra = (L.misc + 16 + 15) & ~15u;
+  L.total = L.extra + extra_bytes;
+  return L;
+}
+
+__device__ __forceinline__ uint8_t* aligned_smem(uint8_t* raw) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) & ~uintptr_t(1023));
+}
+
+// Bounded wait that ignores the abort flag (used only while unwinding).
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+  }
+}
+
+__device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
+  const float m = fmaxf(a.x, b.x);
+  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
+  return make_float2(m, a.y * ex2(a.x - m) + b.y * ex2(b.x - m));
+}
+
+template <int N>
+__device__ __forceinline__ float tree_max(const float (&x)[N]) {
+  float t[N / 2];
+#pragma unroll
+  for (int i = 0; i < N / 2; ++i) t[i] = fmaxf(x[2 * i], x[2 * i + 1]);
+#pragma unroll
+  for (int w = N / 4; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) t[i] = fmaxf(t[2 * i], t[2 * i + 1]);
+  return t[0];
+}
+
+template <int N>
+__device__ __forceinline__ float tree_sum(float (&t)[N]) {
+#pragma unroll
+  for (int w = N / 2; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) t[i] = t[2 * i] + t[2 * i + 1];
+  return t[0];
+}
+
+// Issues the TMA loads of the guide block (all rows_pad rows, both K halves).
+template <int D>
+__device__ __forceinline__ void load_guide(uint8_t* sQ, const CUtensorMap* tmq, int rows_pad,
+                                           int group_index, uint64_t* bar) {
+  constexpr int NKH = D / 64;
+  const int qbox = rows_pad < 256 ? rows_pad : 256;
+  mbar_arrive_expect_tx(bar, static_cast<uint32_t>(NKH * rows_pad * 128));
+#pragma unroll
+  for (int kh = 0; kh < NKH; ++kh)
+    for (int r0 = 0; r0 < rows_pad; r0 += qbox)
+      tma_load_3d(sQ + (kh * rows_pad + r0) * 128, tmq, kh * 64, r0, group_index, bar);
+}
+
+// ---------------------------------------------------------------------------
+// Pass 1: per-row log-sum-exp of the scaled logits.
+// ---------------------------------------------------------------------------
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
+               const __grid_constant__ LseParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = aligned_smem(smem_raw);
+  constexpr int NKH = D / 64;
+  constexpr uint32_t KT = NKH * kHalfTileBytes;
+  const int stages = p.stages, rows_pad = p.rows_pad, nrb = p.nrb;
+  const ScoreSmem L = score_layout(D, rows_pad, stages, 4 * 128 * sizeof(float2));
+  uint8_t* sQ = smem + L.q;
+  uint8_t* sK = smem + L.k;
+  uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
+  uint64_t* empty_k = full_k + stages;
+  uint64_t* q_full = empty_k + stages;
+  uint64_t* tfull = q_full + 1;   // [4], one per epilogue warpgroup = TMEM buffer
+  uint64_t* tempty = tfull + 4;   // [4]
+  uint64_t* drain = tempty + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
+  int* last_flag = reinterpret_cast<int*>(smem + L.misc + 8);
+  float2* stats = reinterpret_cast<float2*>(smem + L.extra);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y;
+  const int b = find_doc(p.docs, blockIdx.x);
+  const int c = blockIdx.x - p.docs.cta[b];
+  const int ncta_doc = p.docs.cta[b + 1] - p.docs.cta[b];
+  const int64_t doc_lo = p.docs.off[b];
+  const int n = static_cast<int>(p.docs.off[b + 1] - doc_lo);
+  const int ntiles = (n + kKeyTile - 1) / kKeyTile;
+  const int t0 = c * p.tiles_per_cta;
+  const int nt = min(p.tiles_per_cta, ntiles - t0);
+  const int njobs = nt * nrb;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full_k[s], 1);
+      mbar_init(&empty_k[s], 1);
+    }
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    *last_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tensormap(&tmk);
+      prefetch_tensormap(&tmq);
+      load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
+      int issued = 0;
+      for (int lt = 0; lt < nt; ++lt) {
+        const int s = lt % stages, use = lt / stages;
+        if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
+        mbar_arrive_expect_tx(&full_k[s], KT);
+        const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
+#pragma unroll
+        for (int kh = 0; kh < NKH; ++kh)
+          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
+        issued = lt + 1;
+      }
+      if (*abort_flag) {  // let in-flight copies land before the CTA exits
+        mbar_drain(q_full, 0);
+        for (int lt = max(0, issued - stages); lt < issued; ++lt)
+          mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(128, kKeyTile);
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      for (int lt = 0; ok && lt < nt; ++lt) {
+        const int s = lt % stages;
+        if (!mbar_wait(&full_k[s], (lt / stages) & 1, abort_flag)) break;
+        tc_fence_after();
+        for (int rb = 0; rb < nrb; ++rb) {
+          const int j = lt * nrb + rb, buf = j & 3, use = j >> 2;
+          if (use > 0 && !mbar_wait(&tempty[buf], (use - 1) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dt = tmem + static_cast<uint32_t>(buf * 128);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const int kh = kk >> 2, k16 = kk & 3;
+            const uint64_t a = sdesc_k128(smem_u32(sQ + (kh * rows_pad + rb * 128) * 128 + k16 * 32));
+            const uint64_t bd = sdesc_k128(smem_u32(sK + s * KT + kh * kHalfTileBytes + k16 * 32));
+            mma_bf16_ss(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&tfull[buf]);
+        }
+        mma_commit(&empty_k[s]);
+      }
+      mma_commit(drain);  // completes once every MMA issued above has finished
+      mbar_drain(drain, 0);
+    }
+    __syncwarp();
+  } else if (warp >= 4) {
+    const int g = (warp - 4) >> 2, quad = warp & 3;
+    const float c2 = p.c2;
+    float m = -INFINITY, z = 0.f;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quad * 32) << 16) + g * 128;
+    for (int j = g, u = 0; j < njobs; j += 4, ++u) {
+      if (!mbar_wait(&tfull[g], u & 1, abort_flag)) break;
+      tc_fence_after();
+      const int lt = j / nrb;
+      const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
+#pragma unroll 1
+      for (int ch = 0; ch < 4; ++ch) {
+        uint32_t r[32];
+        tmem_ld32(trow + ch * 32, r);
+        float x[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
+        if (valid < kKeyTile) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (ch * 32 + i >= valid) x[i] = -INFINITY;
+        }
+        const float mn = fmaxf(m, tree_max<32>(x) * c2);
+        if (mn != -INFINITY) {
+          float e[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) e[i] = ex2(fmaf(x[i], c2, -mn));
+          z = z * ex2(m - mn) + tree_sum<32>(e);
+          m = mn;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[g]);
+    }
+    stats[g * 128 + quad * 32 + lane] = make_float2(m, z);
+  }
+  __syncthreads();
+
+  const bool aborted = *abort_flag != 0;
+  if (aborted) {
+    if (threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
+  } else {
+    if (threadIdx.x < rows_pad) {
+      const int r = threadIdx.x, rb = r >> 7, rr = r & 127;
+      float2 acc = make_float2(-INFINITY, 0.f);
+      for (int g = rb; g < 4; g += nrb) acc = lse_merge(acc, stats[g * 128 + rr]);
+      p.partials[(static_cast<size_t>(h) * gridDim.x + blockIdx.x) * rows_pad + r] = acc;
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      const int prev = atomicAdd(&p.counters[h * p.docs.batch + b], 1);
+      *last_flag = (prev == ncta_doc - 1) ? 1 : 0;
+    }
+    __syncthreads();
+    if (*last_flag) {
+      __threadfence();
+      const float2* part =
+          p.partials + (static_cast<size_t>(h) * gridDim.x + p.docs.cta[b]) * rows_pad;
+      for (int r = threadIdx.x; r < p.rows; r += blockDim.x) {
+        float2 acc = make_float2(-INFINITY, 0.f);
+        for (int cc = 0; cc < ncta_doc; ++cc) {
+          const float2 v = __ldcg(part + static_cast<size_t>(cc) * rows_pad + r);
+          acc = lse_merge(acc, v);
+        }
+        p.lse[(static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows + r] =
+            (acc.x + lg2(acc.y)) * 0.69314718055994531f;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Pass 2: s_key[key] = (1/G) sum over rows of 2^(x*c2 - lse[row]*log2(e)).
+// ---------------------------------------------------------------------------
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
+                    const __grid_constant__ KeyScoreParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = aligned_smem(smem_raw);
+  constexpr int NKH = D / 64;
+  constexpr uint32_t KT = NKH * kHalfTileBytes;
+  const int stages = p.stages, rows_pad = p.rows_pad, rows_mma = p.rows_mma;
+  const int nh = (rows_mma + 255) / 256;
+  const ScoreSmem L = score_layout(D, rows_pad, stages, rows_pad * sizeof(float));
+  uint8_t* sQ = smem + L.q;
+  uint8_t* sK = smem + L.k;
+  uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
+  uint64_t* empty_k = full_k + stages;
+  uint64_t* q_full = empty_k + stages;
+  uint64_t* tfull = q_full + 1;   // [4 warpgroups][2 row halves]
+  uint64_t* tempty = tfull + 8;   // [2 TMEM buffers]
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
+  float* l2s = reinterpret_cast<float*>(smem + L.extra);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y;
+  const int b = find_doc(p.docs, blockIdx.x);
+  const int c = blockIdx.x - p.docs.cta[b];
+  const int64_t doc_lo = p.docs.off[b];
+  const int n = static_cast<int>(p.docs.off[b + 1] - doc_lo);
+  const int ntiles = (n + kKeyTile - 1) / kKeyTile;
+  const int t0 = c * p.tiles_per_cta;
+  const int nt = min(p.tiles_per_cta, ntiles - t0);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full_k[s], 1);
+      mbar_init(&empty_k[s], 1);
+    }
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 8; ++i) mbar_init(&tfull[i], 1);
+    for (int i = 0; i < 2; ++i) mbar_init(&tempty[i], 4);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  {
+    const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
+    for (int r = threadIdx.x; r < rows_pad; r += blockDim.x)
+      l2s[r] = r < p.rows ? lse[r] * 1.4426950408889634f : INFINITY;
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tensormap(&tmk);
+      prefetch_tensormap(&tmq);
+      load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
+      int issued = 0;
+      for (int lt = 0; lt < nt; ++lt) {
+        const int s = lt % stages, use = lt / stages;
+        if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
+        mbar_arrive_expect_tx(&full_k[s], KT);
+        const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
+#pragma unroll
+        for (int kh = 0; kh < NKH; ++kh)
+          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
+        issued = lt + 1;
+      }
+      if (*abort_flag) {
+        mbar_drain(q_full, 0);
+        for (int lt = max(0, issued - stages); lt < issued; ++lt)
+          mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      for (int lt = 0; ok && lt < nt; ++lt) {
+        const int s = lt % stages;
+        if (!mbar_wait(&full_k[s], (lt / stages) & 1, abort_flag)) break;
+        tc_fence_after();
+        for (int hh = 0; hh < nh; ++hh) {
+          const int j = lt * nh + hh, buf = j & 1, use = j >> 1;
+          if (use > 0 && !mbar_wait(&tempty[buf], (use - 1) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int nrows = min(256, rows_mma - 256 * hh);
+          const uint32_t idesc = idesc_bf16_f32(128, nrows);
+          const uint32_t dt = tmem + static_cast<uint32_t>(buf * 256);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const int kh = kk >> 2, k16 = kk & 3;
+            const uint64_t a = sdesc_k128(smem_u32(sK + s * KT + kh * kHalfTileBytes + k16 * 32));
+            const uint64_t bd =
+                sdesc_k128(smem_u32(sQ + (kh * rows_pad + hh * 256) * 128 + k16 * 32));
+            mma_bf16_ss(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&tfull[(lt & 3) * 2 + hh]);
+        }
+        mma_commit(&empty_k[s]);
+      }
+      mma_commit(drain);
+      mbar_drain(drain, 0);
+    }
+    __syncwarp();
+  } else if (warp >= 4) {
+    const int g = (warp - 4) >> 2, quad = warp & 3;
+    const float c2 = p.c2;
+    const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    bool ok = true;
+    for (int lt = g, it = 0; ok && lt < nt; lt += 4, ++it) {
+      float acc = 0.f;
+      for (int hh = 0; hh < nh; ++hh) {
+        if (!mbar_wait(&tfull[g * 2 + hh], it & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int buf = (lt * nh + hh) & 1;
+        const int nrows = min(256, rows_mma - 256 * hh);
+#pragma unroll 1
+        for (int ch = 0; ch < nrows / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tlane + buf * 256 + ch * 32, r);
+          const float4* lp = reinterpret_cast<const float4*>(l2s + hh * 256 + ch * 32);
+          float e[32];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float4 l = lp[i];
+            e[4 * i + 0] = ex2(fmaf(__uint_as_float(r[4 * i + 0]), c2, -l.x));
+            e[4 * i + 1] = ex2(fmaf(__uint_as_float(r[4 * i + 1]), c2, -l.y));
+            e[4 * i + 2] = ex2(fmaf(__uint_as_float(r[4 * i + 2]), c2, -l.z));
+            e[4 * i + 3] = ex2(fmaf(__uint_as_float(r[4 * i + 3]), c2, -l.w));
+          }
+          acc += tree_sum<32>(e);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[buf]);
+      }
+      if (!ok) break;
+      const int key = (t0 + lt) * kKeyTile + quad * 32 + lane;
+      if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = acc * p.inv_group;
+    }
+  }
+  __syncthreads();
+  if (*abort_flag != 0 && threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace
+
+size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
+  return score_layout(head_dim, rows_pad, stages, 4 * 128 * sizeof(float2)).total + 1024;
+}
+
+size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
+  return score_layout(head_dim, rows_pad, stages, rows_pad * sizeof(float)).total + 1024;
+}
+
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmq, const LseParams& p,
+                       int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
+  if (head_dim == 128) {
+    cudaError_t e = cudaFuncSetAttribute(lse_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    lse_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(lse_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    lse_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
+                            const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
+                            cudaStream_t s) {
+  if (head_dim == 128) {
+    cudaError_t e = cudaFuncSetAttribute(
+        keyscore_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    keyscore_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(
+        keyscore_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    keyscore_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace tp

@@ -1,0 +1,116 @@
+// Internal interface between the C-ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/taskpress.h"
+
+namespace tp {
+
+constexpr int kKeyTile = 128;      // context keys per MMA tile
+constexpr int kMaxBatch = TP_MAX_BATCH;
+
+// Where each document's CTAs start inside a head's row of the grid, and where
+// each document's tokens start.  Passed by value (kernel parameter space).
+struct DocTable {
+  int64_t off[kMaxBatch + 1];      // token offsets, off[batch] = N
+  int32_t cta[kMaxBatch + 1];      // CTA prefix per document (grid.x = cta[batch])
+  int32_t batch;
+};
+
+__host__ __device__ inline int find_doc(const DocTable& t, int cta) {
+  int lo = 0, hi = t.batch - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (t.cta[mid] <= cta) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Pass 1: per-row log-sum-exp partials over a CTA's key tiles, then the
+// per-(document, head) merge by the last CTA to finish.
+struct LseParams {
+  DocTable docs;
+  int n_heads_kv;
+  int rows;          // M = G * L_t
+  int rows_pad;      // 128 * nrb
+  int nrb;           // 128-row blocks of the guide (1, 2 or 4)
+  int tiles_per_cta;
+  int stages;        // K-tile ring depth
+  float c2;          // softmax scale * log2(e)
+  float2* partials;  // [H_kv, grid.x, rows_pad] (max2, sum)
+  float* lse;        // [batch, H_kv, rows] natural-log sum-exp of scaled logits
+  int* counters;     // [H_kv * batch], zero at launch
+  int* status;
+};
+
+// Pass 2: per-key sum over all guide rows of exp(logit - lse).
+struct KeyScoreParams {
+  DocTable docs;
+  int n_heads_kv;
+  int rows;
+  int rows_pad;
+  int rows_mma;      // rows rounded up to 32 (the MMA N extent, split in 256s)
+  int tiles_per_cta;
+  int stages;
+  float c2;
+  float inv_group;
+  int64_t n_total;
+  const float* lse;  // [batch, H_kv, rows] natural log
+  float* skey;       // [H_kv, N]
+  int* status;
+};
+
+struct SelectParams {
+  int64_t off[kMaxBatch + 1];
+  int32_t kept[kMaxBatch];   // k_b per document
+  int batch;
+  int n_heads_kv;
+  int64_t n_total;
+  int64_t cap;
+  int pool_kernel;           // >= 1, odd; 1 with mode_scores
+  int key_only;
+  const float* scores_in;    // combined scores (tp_select) or null
+  const float* skey;         // unpooled key scores (fused path) or null
+  const float* gamma;        // per-token scale (fused path) or null
+  float* scores_out;         // optional combined scores out (fused path)
+  uint32_t* keys;            // [H_kv, N] scratch
+  int32_t* idx;              // [batch, H_kv, cap]
+};
+
+struct GatherParams {
+  int64_t off[kMaxBatch + 1];
+  int batch;
+  int n_heads_kv;
+  int head_dim;
+  int64_t n_total;
+  int64_t cap;
+  float qmax;
+  const uint16_t* k;
+  const uint16_t* v;
+  const float* gamma;
+  const int32_t* idx;
+  uint16_t* kc;
+  uint16_t* vc;
+  int8_t* vqc;
+  float* gammac;
+};
+
+// Launchers (return cudaError_t of the launch).
+cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
+                          float qmax, int num_sms, cudaStream_t s);
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmq, const LseParams& p,
+                       int head_dim, dim3 grid, size_t smem, cudaStream_t s);
+cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
+                            const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
+                            cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
+cudaError_t launch_gather(const GatherParams& p, cudaStream_t s);
+
+// Shared-memory layout sizes of the scoring kernels (host side).
+size_t lse_smem_bytes(int head_dim, int rows_pad, int stages);
+size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages);
+
+}  // namespace tp

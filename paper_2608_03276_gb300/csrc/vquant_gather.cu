@@ -1,0 +1,164 @@
+// Eq. 2 (Sec. 3.3) per-token V scale and int8 codes, and the order-preserving
+// compaction of kept rows into the compressed cache (Sec. 3.1).
+//
+// Both kernels move 16-byte vectors: a row of d bf16 is d/8 lanes wide, so a
+// warp covers 32/(d/8) rows per instruction.  The quantisation rule is the
+// IEEE one shared with the oracle: gamma = fp32 round-to-nearest(absmax/qmax),
+// code = round-half-even of the fp32 quotient v/gamma, clamped; gamma = 0
+// gives code 0.  Divisions use __fdiv_rn so that no reciprocal shortcut or
+// fused rounding changes a code.
+#include <cuda_bf16.h>
+
+#include "tp_device.cuh"
+
+namespace tp {
+
+namespace {
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&f)[8]) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__device__ __forceinline__ int8_t quant_code(float v, float gamma, float qmax) {
+  if (!(gamma > 0.f)) return 0;
+  float q = rintf(__fdiv_rn(v, gamma));
+  q = fminf(fmaxf(q, -qmax), qmax);
+  return static_cast<int8_t>(static_cast<int>(q));
+}
+
+__device__ __forceinline__ uint2 quant8(const float (&f)[8], float gamma, float qmax) {
+  uint32_t lo = 0, hi = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[i], gamma, qmax))) << (8 * i);
+    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[4 + i], gamma, qmax))) << (8 * i);
+  }
+  return make_uint2(lo, hi);
+}
+
+// One row = LPR lanes x 8 bf16.  Rows are processed UNROLL at a time per
+// lane group so that several 16-byte loads are in flight per thread.
+template <int LPR, int UNROLL>
+__global__ void __launch_bounds__(256) vquant_kernel(const uint4* __restrict__ v,
+                                                      uint2* __restrict__ vq,
+                                                      float* __restrict__ gamma, int64_t rows,
+                                                      float qmax) {
+  constexpr int RPW = 32 / LPR;  // rows per warp instruction
+  const int lane = threadIdx.x & 31;
+  const int sub = lane / LPR, part = lane % LPR;
+  const int64_t warps_total = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  const int64_t gw = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  for (int64_t base = gw * RPW * UNROLL; base < rows; base += warps_total * RPW * UNROLL) {
+    uint4 u[UNROLL];
+#pragma unroll
+    for (int k = 0; k < UNROLL; ++k) {
+      const int64_t row = base + k * RPW + sub;
+      u[k] = row < rows ? __ldcs(v + row * LPR + part) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int k = 0; k < UNROLL; ++k) {
+      const int64_t row = base + k * RPW + sub;
+      float f[8];
+      bf16x8_to_f32(u[k], f);
+      float a = 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) a = fmaxf(a, fabsf(f[i]));
+#pragma unroll
+      for (int o = LPR / 2; o >= 1; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+      const float g = __fdiv_rn(a, qmax);
+      if (row < rows) {
+        if (vq) vq[row * LPR + part] = quant8(f, g, qmax);
+        if (part == 0) gamma[row] = g;
+      }
+    }
+  }
+}
+
+// Compaction: one (document, head, slot) per LPR-lane group for K and one for
+// V; idx < 0 marks an unused slot (zero-filled).
+template <int LPR>
+__global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherParams p) {
+  constexpr int SPW = 32 / (2 * LPR);  // slots per warp
+  const int lane = threadIdx.x & 31;
+  const int grp = lane / (2 * LPR);            // slot within the warp
+  const bool is_v = (lane % (2 * LPR)) >= LPR;  // K lanes then V lanes
+  const int part = lane % LPR;
+  const int b = blockIdx.z, h = blockIdx.y;
+  const int64_t unit = static_cast<int64_t>(b) * p.n_heads_kv + h;
+  const int64_t warp_global = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int64_t t = warp_global * SPW + grp;
+  if (t >= p.cap) return;
+  const int64_t slot = unit * p.cap + t;
+  const int32_t j = p.idx[slot];
+  const int64_t dst = slot * LPR + part;
+  if (j < 0) {
+    const uint4 z = make_uint4(0, 0, 0, 0);
+    if (!is_v) {
+      if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = z;
+    } else {
+      if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = z;
+      if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = make_uint2(0, 0);
+      if (p.gammac && part == 0) p.gammac[slot] = 0.f;
+    }
+    return;
+  }
+  const int64_t tok = static_cast<int64_t>(h) * p.n_total + p.off[b] + j;
+  if (!is_v) {
+    if (p.kc) {
+      const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.k) + tok * LPR + part);
+      reinterpret_cast<uint4*>(p.kc)[dst] = u;
+    }
+  } else {
+    const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.v) + tok * LPR + part);
+    if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = u;
+    const float g = p.gamma[tok];
+    if (p.vqc) {
+      float f[8];
+      bf16x8_to_f32(u, f);
+      reinterpret_cast<uint2*>(p.vqc)[dst] = quant8(f, g, p.qmax);
+    }
+    if (p.gammac && part == 0) p.gammac[slot] = g;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
+                          float qmax, int num_sms, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  constexpr int kUnroll = 4;
+  const int threads = 256;
+  const int lpr = head_dim / 8;
+  const int64_t rows_per_block = static_cast<int64_t>(threads / 32) * (32 / lpr) * kUnroll;
+  int64_t blocks = (rows + rows_per_block - 1) / rows_per_block;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  if (blocks > cap) blocks = cap;
+  const uint4* vv = reinterpret_cast<const uint4*>(v);
+  uint2* qq = reinterpret_cast<uint2*>(vq);
+  if (head_dim == 128)
+    vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+  else
+    vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
+  if (p.cap <= 0) return cudaSuccess;
+  const int threads = 256;
+  const int lpr = p.head_dim / 8;
+  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr));
+  dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
+            p.batch);
+  if (p.head_dim == 128)
+    gather_kernel<16><<<grid, threads, 0, s>>>(p);
+  else
+    gather_kernel<8><<<grid, threads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace tp

@@ -94,6 +94,23 @@ def pin_default_scale_in_layer(O):
         assert abs(out["key"][(0, 0)][0] - p0) <= 1e-14, (d, a, scale, out["key"][(0, 0)], p0)
 
 
+def pin_row_normaliser(O):
+    """lse = log n for Q = 0; two keys +-e1 and q = a*e1: lse = |t| + log1p(exp(-2|t|)), t = a*sigma."""
+    for n, d in [(1, 4), (7, 8), (1000, 16)]:
+        got = O.guide_lse(np.zeros((3, d)), _rand(n, (n, d)), 0.25)
+        assert np.allclose(got, math.log(n), rtol=0, atol=1e-13), (got, math.log(n))
+    d = 16
+    k = np.zeros((2, d))
+    k[0, 0], k[1, 0] = 1.0, -1.0
+    for a in (0.0, 0.75, -3.0, 50.0, 9000.0):
+        q = np.zeros((1, d))
+        q[0, 0] = a
+        t = abs(a) * 0.25
+        want = t + math.log1p(math.exp(-2 * t))
+        got = O.guide_lse(q, k, 0.25)[0]
+        assert abs(got - want) <= 1e-12 * max(1.0, t), (a, got, want)
+
+
 # -- Eq. 1: sum over guide tokens, mean over the GQA group --------------------
 
 def pin_key_scores_total_mass(O):

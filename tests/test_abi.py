@@ -1,0 +1,87 @@
+"""C ABI checks that need no GPU: the library loads, exports every declared
+symbol, and its host-side logic (budget rule, capacity, workspace sizing,
+argument validation) behaves as include/taskpress.h states."""
+import math
+import os
+import re
+from fractions import Fraction
+
+import pytest
+
+from oracle import taskpress_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_03276_gb300 import build as b
+    from paper_2608_03276_gb300 import binding
+    b.build()
+    return binding
+
+
+def declared_symbols():
+    with open(os.path.join(ROOT, "include", "taskpress.h")) as f:
+        src = f.read()
+    return sorted(set(re.findall(r"^\s*(?:[\w\*]+\s+)+\**(tp_\w+)\s*\(", src, re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_symbols()
+    assert len(names) == 12, names
+    assert sorted(lib.EXPORTS) == names
+    cdll = lib.load()
+    for n in names:
+        assert hasattr(cdll, n), n
+
+
+def test_budget_matches_oracle_and_exact_decimals(lib):
+    for r in ["0", "0.05", "0.07", "0.1", "0.2", "0.25", "0.33", "0.5", "0.9", "1"]:
+        for n in [0, 1, 2, 7, 100, 129, 2048, 32768, 65536, 131072, 294912]:
+            got = lib.tp_budget(n, float(r))
+            assert got == O.budget(n, float(r)) == math.ceil(Fraction(r) * n), (r, n, got)
+    assert lib.tp_budget(10, -0.5) == -1 and lib.tp_budget(10, 1.01) == -1
+    assert lib.tp_budget(10, float("nan")) == -1 and lib.tp_budget(-1, 0.5) == -1
+
+
+def _prob(lib, offs, **kw):
+    args = dict(n_heads_q=8, n_heads_kv=2, head_dim=64, guide_len=16, doc_offsets=offs)
+    args.update(kw)
+    return lib.Problem(**args)
+
+
+def test_capacity_and_workspace(lib):
+    p = _prob(lib, [0, 1000, 1001, 3000])
+    assert lib.tp_kept_capacity(p, 0.25, -1) == 500
+    assert lib.tp_kept_capacity(p, 0.0, 300) == 300
+    assert lib.tp_kept_capacity(p, 0.0, 5000) == 1999
+    assert lib.tp_kept_capacity(p, 1.5, -1) == -1
+    assert lib.tp_workspace_bytes(p, 0.25, -1) > 3000 * 2 * 12
+    assert lib.tp_workspace_bytes(p, 0.25, -1) % 256 == 0
+
+
+@pytest.mark.parametrize("kw", [
+    dict(head_dim=96), dict(head_dim=256), dict(pool_kernel=4), dict(pool_kernel=0),
+    dict(quant_bits=4), dict(n_heads_q=7), dict(guide_len=0), dict(guide_len=65, n_heads_q=16),
+])
+def test_rejects_unsupported(lib, kw):
+    p = _prob(lib, [0, 100], **kw)
+    assert lib.tp_kept_capacity(p, 0.5, -1) == -1
+    assert lib.tp_workspace_bytes(p, 0.5, -1) == 0
+
+
+def test_rejects_bad_offsets(lib):
+    assert lib.tp_kept_capacity(_prob(lib, [1, 100]), 0.5, -1) == -1
+    assert lib.tp_kept_capacity(_prob(lib, [0, 100, 50]), 0.5, -1) == -1
+    assert lib.tp_kept_capacity(_prob(lib, list(range(0, 258))), 0.5, -1) == -1
+
+
+def test_null_pointers_rejected_before_any_launch(lib):
+    cdll = lib.load()
+    p = _prob(lib, [0, 100])
+    assert cdll.tp_quantize_v(p.ref(), None, None, None, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_compress_layer(p.ref(), None, None, None, 0.5, -1, None, None, None, None, None,
+                                  None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_select(p.ref(), None, 0.5, -1, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_status_string(-5) == b"device-side wait timed out"

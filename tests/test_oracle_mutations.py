@@ -18,6 +18,8 @@ MUTATIONS = {
     "softmax over the wrong axis": ("z = np.sum(e, axis=1, keepdims=True)", "z = np.sum(e, axis=0, keepdims=True)"),
     "scale 1/d instead of 1/sqrt(d)": ("1.0 / math.sqrt(d)\n    gamma", "1.0 / d\n    gamma"),
     "no max subtraction": ("e = np.exp(x - m)", "e = np.exp(x)"),
+    "row normaliser drops the max": ("return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))", "return np.log(np.sum(np.exp(x), axis=1))"),
+    "row normaliser log2": ("return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))", "return m + np.log2(np.sum(np.exp(x - m[:, None]), axis=1))"),
     "sum over the GQA group": ("return a.sum(axis=0) / g", "return a.sum(axis=0)"),
     "mean over guide tokens": ("return a.sum(axis=0) / g", "return a.mean(axis=0)"),
     "interleaved GQA heads": ("qg = q[b, h * g:(h + 1) * g]", "qg = q[b, h::n_heads_kv]"),
@@ -34,7 +36,7 @@ MUTATIONS = {
     "kept indices not ascending": ("return np.sort(order[:k]).astype(np.int64)", "return order[:k].astype(np.int64)"),
     "naive ceil budget": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.ceil(keep_ratio * float(n))"),
     "budget rounds down": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.floor(keep_ratio * float(n))"),
-    "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma)", "s_key = key_scores(qg, k_all[h, 0:n], sigma)"),
+    "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma) if", "s_key = key_scores(qg, k_all[h, 0:n], sigma) if"),
 }
 
 
