@@ -52,6 +52,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--config", type=int, default=3, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layers", type=int, default=0, help="override the workload's layer count")
     ap.add_argument("--e2e-layers", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-heads", type=int, default=0, help="0: every KV head of one layer")
@@ -300,7 +301,7 @@ def run_ours(args, w):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     value = w.n_total * L * world / (ms / 1e3)
-    kernels_per_call = 5 if cap > 0 else 4
+    kernels_per_call = binding.KERNELS_PER_COMPRESS
     gpu_launches = kernels_per_call * L * args.steps
 
     # ---- staged pass: per-kernel CUDA-event times of the same launches
@@ -434,6 +435,8 @@ def main():
     args = parse()
     from paper_2608_03276_gb300 import synth
     w = synth.WORKLOADS[args.config]
+    if args.layers > 0:
+        w = w.with_(layers=args.layers)
     if args.impl == "reference":
         run_reference(args, w)
     else:

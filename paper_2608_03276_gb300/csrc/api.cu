@@ -4,6 +4,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "tp_internal.h"
@@ -29,7 +30,9 @@ struct Plan {
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
-  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
+  int max_chunks;
+  size_t ws_status, ws_hist, ws_partials, ws_counts, ws_thresh, ws_lse, ws_skey, ws_gamma, ws_keys,
+      ws_total;
 };
 
 int num_sms() {
@@ -122,11 +125,23 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
     }
   }
 
+  int64_t max_n = 0;
+  for (int b = 0; b < P->batch; ++b) max_n = std::max<int64_t>(max_n, P->off[b + 1] - P->off[b]);
+  P->max_chunks = static_cast<int>((max_n + kChunk - 1) / kChunk);
+  const size_t units = size_t(P->hkv) * P->batch;
+
+  // [status | counters | radix histograms] are zeroed at the start of a call.
   size_t o = 0;
   P->ws_status = o;
-  o = align_up(o + sizeof(int) * (1 + size_t(P->hkv) * P->batch));
+  o = align_up(o + sizeof(int) * (1 + units));
+  P->ws_hist = o;
+  o = align_up(o + sizeof(int) * units * kHistInts);
   P->ws_partials = o;
   o = align_up(o + sizeof(float2) * size_t(P->hkv) * P->grid_x * P->rows_pad);
+  P->ws_counts = o;
+  o = align_up(o + sizeof(int2) * units * (P->max_chunks > 0 ? P->max_chunks : 1));
+  P->ws_thresh = o;
+  o = align_up(o + sizeof(int2) * units);
   P->ws_lse = o;
   o = align_up(o + sizeof(float) * size_t(P->batch) * P->hkv * P->rows);
   P->ws_skey = o;
@@ -250,15 +265,28 @@ int run_scoring(const Plan& P, const void* q, const void* k, char* ws, cudaStrea
                       reinterpret_cast<int*>(ws + P.ws_status), s);
 }
 
-void fill_select(const Plan& P, SelectParams* sp) {
+void fill_select(const Plan& P, char* ws, SelectParams* sp) {
   memset(sp, 0, sizeof(*sp));
   for (int b = 0; b <= P.batch; ++b) sp->off[b] = P.off[b];
   for (int b = 0; b < P.batch; ++b) sp->kept[b] = P.kept[b];
   sp->batch = P.batch;
   sp->n_heads_kv = P.hkv;
+  sp->head_dim = P.d;
   sp->n_total = P.n_total;
   sp->cap = P.cap;
+  sp->max_chunks = P.max_chunks;
   sp->pool_kernel = 1;
+  sp->qmax = 127.0f;
+  sp->keys = reinterpret_cast<uint32_t*>(ws + P.ws_keys);
+  sp->hist = reinterpret_cast<int*>(ws + P.ws_hist);
+  sp->counts = reinterpret_cast<int2*>(ws + P.ws_counts);
+  sp->thresh = reinterpret_cast<int2*>(ws + P.ws_thresh);
+}
+
+int zero_head(const Plan& P, char* ws, cudaStream_t s) {
+  return cudaMemsetAsync(ws + P.ws_status, 0, P.ws_partials - P.ws_status, s) == cudaSuccess
+             ? TP_OK
+             : TP_ERR_CUDA;
 }
 
 void fill_gather(const Plan& P, GatherParams* gp) {
@@ -326,23 +354,17 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
     return TP_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
-    return TP_ERR_CUDA;
-  st = run_scoring(P, q, k, w, s);
-  if (st != TP_OK) return st;
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
+  if ((st = run_scoring(P, q, k, w, s)) != TP_OK) return st;
   SelectParams sp;
-  fill_select(P, &sp);
+  fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;
   sp.key_only = key_only ? 1 : 0;
   sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
   sp.gamma = gamma;
   sp.scores_out = scores;
-  sp.keys = reinterpret_cast<uint32_t*>(w + P.ws_keys);
-  // k = 0 for every document: the select kernel only forms the scores.
-  for (int b = 0; b < P.batch; ++b) sp.kept[b] = 0;
-  sp.cap = 0;
-  sp.idx = nullptr;
-  return cuda_status(launch_select(sp, s));
+  sp.hist = nullptr;  // scores only
+  return cuda_status(launch_select(sp, true, s));
 }
 
 int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
@@ -355,8 +377,7 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, 
     return TP_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
-    return TP_ERR_CUDA;
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
@@ -383,12 +404,14 @@ int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64
   if (!scores || (!idx && P.cap > 0)) return TP_ERR_INVALID_ARG;
   if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
     return TP_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
   SelectParams sp;
-  fill_select(P, &sp);
+  fill_select(P, w, &sp);
   sp.scores_in = scores;
-  sp.keys = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + P.ws_keys);
   sp.idx = idx;
-  return cuda_status(launch_select(sp, static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_select(sp, false, s));
 }
 
 int tp_compact(const tp_problem* p, const void* k, const void* v, const float* gamma,
@@ -432,36 +455,27 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
-  if (cudaMemsetAsync(w + P.ws_status, 0, P.ws_partials - P.ws_status, s) != cudaSuccess)
-    return TP_ERR_CUDA;
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
   cudaError_t e = launch_vquant(static_cast<const uint16_t*>(v), nullptr, g,
                                 int64_t(P.hkv) * P.n_total, P.d, 127.0f, num_sms(), s);
   if (e != cudaSuccess) return TP_ERR_CUDA;
-  st = run_scoring(P, q, k, w, s);
-  if (st != TP_OK) return st;
+  if ((st = run_scoring(P, q, k, w, s)) != TP_OK) return st;
   SelectParams sp;
-  fill_select(P, &sp);
+  fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;
   sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
   sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
   sp.gamma = g;
   sp.scores_out = scores;
-  sp.keys = reinterpret_cast<uint32_t*>(w + P.ws_keys);
   sp.idx = idx;
-  e = launch_select(sp, s);
-  if (e != cudaSuccess) return TP_ERR_CUDA;
-  if (P.cap == 0) return TP_OK;
-  GatherParams gp;
-  fill_gather(P, &gp);
-  gp.k = static_cast<const uint16_t*>(k);
-  gp.v = static_cast<const uint16_t*>(v);
-  gp.gamma = g;
-  gp.idx = idx;
-  gp.kc = static_cast<uint16_t*>(kc);
-  gp.vc = static_cast<uint16_t*>(vc);
-  gp.vqc = vqc;
-  gp.gammac = gammac;
-  return cuda_status(launch_gather(gp, s));
+  sp.gather = 1;
+  sp.k = static_cast<const uint16_t*>(k);
+  sp.v = static_cast<const uint16_t*>(v);
+  sp.kc = static_cast<uint16_t*>(kc);
+  sp.vc = static_cast<uint16_t*>(vc);
+  sp.vqc = vqc;
+  sp.gammac = gammac;
+  return cuda_status(launch_select(sp, false, s));
 }
 
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {

@@ -236,4 +236,47 @@ __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int* total)
   return res;
 }
 
+// Sum over the block; `warp_tot` is the same 33-int scratch as block_excl_scan.
+__device__ __forceinline__ int block_sum(int v, int* warp_tot) {
+  int total;
+  block_excl_scan(v, warp_tot, &total);
+  return total;
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 2 codes: round-half-even of the IEEE fp32 quotient v / gamma, clamped to
+// +-qmax; gamma = 0 gives 0.  __fdiv_rn keeps the quotient correctly rounded.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int8_t quant_code(float v, float gamma, float qmax) {
+  if (!(gamma > 0.f)) return 0;
+  float q = rintf(__fdiv_rn(v, gamma));
+  q = fminf(fmaxf(q, -qmax), qmax);
+  return static_cast<int8_t>(static_cast<int>(q));
+}
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&f)[8]) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__device__ __forceinline__ uint2 quant8(const float (&f)[8], float gamma, float qmax) {
+  uint32_t lo = 0, hi = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[i], gamma, qmax))) << (8 * i);
+    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[4 + i], gamma, qmax))) << (8 * i);
+  }
+  return make_uint2(lo, hi);
+}
+
+__device__ __forceinline__ uint2 quant8_bf16(const uint4& u, float gamma, float qmax) {
+  float f[8];
+  bf16x8_to_f32(u, f);
+  return quant8(f, gamma, qmax);
+}
+
 }  // namespace tp

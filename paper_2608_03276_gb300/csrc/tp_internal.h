@@ -63,21 +63,37 @@ struct KeyScoreParams {
   int* status;
 };
 
+constexpr int kChunk = 4096;      // tokens per CTA in the selection kernels
+constexpr int kHistInts = 2048 + 2048 + 1024;  // radix histograms per unit
+
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
   int32_t kept[kMaxBatch];   // k_b per document
   int batch;
   int n_heads_kv;
+  int head_dim;
   int64_t n_total;
   int64_t cap;
-  int pool_kernel;           // >= 1, odd; 1 with mode_scores
+  int max_chunks;            // chunks of the longest document
+  int pool_kernel;           // >= 1, odd
   int key_only;
+  int gather;                // fused path: also write the compressed rows
+  float qmax;
   const float* scores_in;    // combined scores (tp_select) or null
   const float* skey;         // unpooled key scores (fused path) or null
   const float* gamma;        // per-token scale (fused path) or null
   float* scores_out;         // optional combined scores out (fused path)
   uint32_t* keys;            // [H_kv, N] scratch
+  int* hist;                 // [units, kHistInts] scratch, zero at launch
+  int2* counts;              // [units, max_chunks] scratch
+  int2* thresh;              // [units] scratch
   int32_t* idx;              // [batch, H_kv, cap]
+  const uint16_t* k;         // rows gathered when `gather`
+  const uint16_t* v;
+  uint16_t* kc;
+  uint16_t* vc;
+  int8_t* vqc;
+  float* gammac;
 };
 
 struct GatherParams {
@@ -106,7 +122,7 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmq, const Lse
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             cudaStream_t s);
-cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, bool form_scores_only, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s);
 
 // Shared-memory layout sizes of the scoring kernels (host side).

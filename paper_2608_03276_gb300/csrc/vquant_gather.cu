@@ -15,32 +15,6 @@ namespace tp {
 
 namespace {
 
-__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&f)[8]) {
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    f[2 * i] = __uint_as_float(w[i] << 16);
-    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-  }
-}
-
-__device__ __forceinline__ int8_t quant_code(float v, float gamma, float qmax) {
-  if (!(gamma > 0.f)) return 0;
-  float q = rintf(__fdiv_rn(v, gamma));
-  q = fminf(fmaxf(q, -qmax), qmax);
-  return static_cast<int8_t>(static_cast<int>(q));
-}
-
-__device__ __forceinline__ uint2 quant8(const float (&f)[8], float gamma, float qmax) {
-  uint32_t lo = 0, hi = 0;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[i], gamma, qmax))) << (8 * i);
-    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[4 + i], gamma, qmax))) << (8 * i);
-  }
-  return make_uint2(lo, hi);
-}
-
 // One row = LPR lanes x 8 bf16.  Rows are processed UNROLL at a time per
 // lane group so that several 16-byte loads are in flight per thread.
 template <int LPR, int UNROLL>

@@ -196,19 +196,23 @@ def test_pool_kernels(cuda_lib, pool_kernel):
 # ---------------------------------------------------------------------------
 # Selection and compaction as separate entry points (bit-exact)
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("budget", [0, 1, 2, 299, 300, 301, 5000])
+@pytest.mark.parametrize("budget", [0, 1, 2, 299, 300, 301, 5000, 9000, 13000])
 def test_select_bit_exact(cuda_lib, budget):
+    """Documents of 1 to 12,000 tokens (several 4096-token chunks), with tie groups
+    that span chunks, zeros and negative zeros."""
     import torch
     from paper_2608_03276_gb300 import binding
     rng = np.random.Generator(np.random.PCG64(budget))
-    offs = np.array([0, 300, 301, 1500, 1500, 4000])
+    offs = np.array([0, 300, 301, 1500, 1500, 4000, 16000, 25000])
     hkv = 3
     n = int(offs[-1])
     sc = rng.random((hkv, n)).astype(np.float32)
     sc[0, :300] = 0.5                        # all ties
     sc[1, 1500:1600] = 0.0                   # zeros
     sc[1, 1600:1610] = -0.0
-    sc[2, 2000:] = np.round(sc[2, 2000:] * 8) / 8   # heavy ties
+    sc[2, 2000:] = np.round(sc[2, 2000:] * 8) / 8   # heavy ties across chunks
+    sc[0, 4000:16000] = np.round(sc[0, 4000:16000] * 3) / 3
+    sc[1, 16000:25000] = 0.25
     p = binding.Problem(hkv * 2, hkv, 64, 8, offs)
     cap = binding.tp_kept_capacity(p, 0.0, budget)
     idx = torch.empty((len(offs) - 1, hkv, cap), dtype=torch.int32, device="cuda")
