@@ -15,10 +15,9 @@
 //
 // Both passes stream 128-key tiles of K with TMA (128-byte swizzle) through a
 // ring of shared-memory stages; one thread issues the MMAs; four epilogue
-// warpgroups drain TMEM.  Warp roles per CTA (20 warps):
-//   warp 0  TMA producer      warp 1  MMA issuer
-//   warp 2  TMEM owner        warp 3  idle
-//   warps 4-19  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
+// warpgroups drain TMEM.  Warp roles per CTA (18 warps):
+//   warp 0  TMEM owner + TMA producer      warp 1  MMA issuer
+//   warps 2-17  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
 #include <math.h>
 
 #include "tp_device.cuh"
@@ -27,7 +26,8 @@ namespace tp {
 
 namespace {
 
-constexpr int kThreads = 640;
+constexpr int kThreads = 576;
+constexpr int kEpiWarp0 = 2;  // first epilogue warp
 constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
 
 struct ScoreSmem {
@@ -66,25 +66,85 @@ __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
   return make_float2(m, a.y * ex2(a.x - m) + b.y * ex2(b.x - m));
 }
 
-template <int N>
-__device__ __forceinline__ float tree_max(const float (&x)[N]) {
-  float t[N / 2];
+// Max of 32 values (three-input max, 16 instructions).
+__device__ __forceinline__ float max32(const float (&x)[32]) {
+  float t[11];
 #pragma unroll
-  for (int i = 0; i < N / 2; ++i) t[i] = fmaxf(x[2 * i], x[2 * i + 1]);
-#pragma unroll
-  for (int w = N / 4; w >= 1; w >>= 1)
-#pragma unroll
-    for (int i = 0; i < w; ++i) t[i] = fmaxf(t[2 * i], t[2 * i + 1]);
-  return t[0];
+  for (int i = 0; i < 10; ++i) t[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
+  t[10] = fmaxf(x[30], x[31]);
+  const float a = fmax3(t[0], t[1], t[2]), b = fmax3(t[3], t[4], t[5]);
+  const float c = fmax3(t[6], t[7], t[8]), d = fmaxf(t[9], t[10]);
+  return fmaxf(fmax3(a, b, c), d);
 }
 
-template <int N>
-__device__ __forceinline__ float tree_sum(float (&t)[N]) {
+// sum_i 2^(x_i * c2 + off) for 32 values with packed fma/add into four
+// partial sums (keeps few registers live while the next chunk is in flight).
+__device__ __forceinline__ float sum_exp2(const float (&x)[32], float c2, float off) {
+  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
+  const float2 cc = make_float2(c2, c2), oo = make_float2(off, off);
 #pragma unroll
-  for (int w = N / 2; w >= 1; w >>= 1)
+  for (int i = 0; i < 16; ++i) {
+    const float2 y = ffma2(make_float2(x[2 * i], x[2 * i + 1]), cc, oo);
+    a[i & 3] = fadd2(a[i & 3], make_float2(ex2(y.x), ex2(y.y)));
+  }
+  const float2 t = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
+  return t.x + t.y;
+}
+
+// One 32-column chunk of a guide row's logits into the running (offset m,
+// sum z) of pass 1, both in log2 units: z = sum 2^(x*c2 - m).  The offset is
+// refreshed from the exact chunk maximum only when it is unset or the chunk
+// sum would leave the safe range (2^64); otherwise no max is computed.
+__device__ __forceinline__ void lse_chunk(const uint32_t (&r)[32], int col0, int valid, float c2,
+                                          float& m, float& z) {
+  float x[32];
 #pragma unroll
-    for (int i = 0; i < w; ++i) t[i] = t[2 * i] + t[2 * i + 1];
-  return t[0];
+  for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
+  if (valid < col0 + 32) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (col0 + i >= valid) x[i] = -INFINITY;
+  }
+  float s = 0.f;
+  bool exact = (m == -INFINITY);
+  if (!exact) {
+    s = sum_exp2(x, c2, -m);
+    exact = !(s <= 0x1p64f);
+  }
+  if (exact) {
+    const float mn = fmaxf(m, max32(x) * c2);
+    if (mn == -INFINITY) return;
+    s = sum_exp2(x, c2, -mn);
+    z *= ex2(m - mn);
+    m = mn;
+  }
+  z += s;
+  if (z > 0x1p64f) {
+    z *= 0x1p-64f;
+    m += 64.f;
+  }
+}
+
+// One 32-column chunk of a key's logits in pass 2: sum_r 2^(x_r*c2 - l_r),
+// with the negated row normalisers -l_r read from shared memory.
+__device__ __forceinline__ float key_chunk(const uint32_t (&r)[32], const float* nl, float c2) {
+  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
+  const float2 cc = make_float2(c2, c2);
+  const float4* nl4 = reinterpret_cast<const float4*>(nl);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 l = nl4[i];
+    const float2 y0 = ffma2(make_float2(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1])),
+                            cc, make_float2(l.x, l.y));
+    const float2 y1 = ffma2(make_float2(__uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3])),
+                            cc, make_float2(l.z, l.w));
+    a[(2 * i) & 3] = fadd2(a[(2 * i) & 3], make_float2(ex2(y0.x), ex2(y0.y)));
+    a[(2 * i + 1) & 3] = fadd2(a[(2 * i + 1) & 3], make_float2(ex2(y1.x), ex2(y1.y)));
+  }
+  const float2 t = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
+  return t.x + t.y;
 }
 
 // Issues the TMA loads of the guide block (all rows_pad rows, both K halves).
@@ -153,7 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *last_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 2) {
+  if (warp == 0) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
@@ -216,8 +276,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0);
     }
     __syncwarp();
-  } else if (warp >= 4) {
-    const int g = (warp - 4) >> 2, quad = warp & 3;
+  } else if (warp >= kEpiWarp0) {
+    const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     const float c2 = p.c2;
     float m = -INFINITY, z = 0.f;
     const uint32_t trow = tmem + (static_cast<uint32_t>(quad * 32) << 16) + g * 128;
@@ -226,30 +286,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const int lt = j / nrb;
       const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
-#pragma unroll 1
-      for (int ch = 0; ch < 4; ++ch) {
-        uint32_t r[32];
-        tmem_ld32(trow + ch * 32, r);
-        float x[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
-        if (valid < kKeyTile) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (ch * 32 + i >= valid) x[i] = -INFINITY;
-        }
-        const float mn = fmaxf(m, tree_max<32>(x) * c2);
-        if (mn != -INFINITY) {
-          float e[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) e[i] = ex2(fmaf(x[i], c2, -mn));
-          z = z * ex2(m - mn) + tree_sum<32>(e);
-          m = mn;
-        }
-      }
-      tc_fence_before();
+      // four 32-column chunks; the next chunk's TMEM load overlaps this chunk's math
+      uint32_t ra[32], rb[32];
+      tmem_ld32_async(trow, ra);
+      tmem_wait(ra);
+      tmem_ld32_async(trow + 32, rb);
+      lse_chunk(ra, 0, valid, c2, m, z);
+      tmem_wait(rb);
+      tmem_ld32_async(trow + 64, ra);
+      lse_chunk(rb, 32, valid, c2, m, z);
+      tmem_wait(ra);
+      tmem_ld32_async(trow + 96, rb);
+      lse_chunk(ra, 64, valid, c2, m, z);
+      tmem_wait(rb);
+      tc_fence_before();  // TMEM buffer free before the last chunk's math
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[g]);
+      lse_chunk(rb, 96, valid, c2, m, z);
     }
     stats[g * 128 + quad * 32 + lane] = make_float2(m, z);
   }
@@ -288,7 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __syncthreads();
-  if (warp == 2) {
+  if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
@@ -345,9 +398,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
     for (int r = threadIdx.x; r < rows_pad; r += blockDim.x)
-      l2s[r] = r < p.rows ? lse[r] * 1.4426950408889634f : INFINITY;
+      l2s[r] = r < p.rows ? -(lse[r] * 1.4426950408889634f) : -INFINITY;
   }
-  if (warp == 2) {
+  if (warp == 0) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
@@ -412,8 +465,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0);
     }
     __syncwarp();
-  } else if (warp >= 4) {
-    const int g = (warp - 4) >> 2, quad = warp & 3;
+  } else if (warp >= kEpiWarp0) {
+    const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     const float c2 = p.c2;
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
@@ -426,26 +479,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const int buf = (lt * nh + hh) & 1;
-        const int nrows = min(256, rows_mma - 256 * hh);
-#pragma unroll 1
-        for (int ch = 0; ch < nrows / 32; ++ch) {
-          uint32_t r[32];
-          tmem_ld32(tlane + buf * 256 + ch * 32, r);
-          const float4* lp = reinterpret_cast<const float4*>(l2s + hh * 256 + ch * 32);
-          float e[32];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const float4 l = lp[i];
-            e[4 * i + 0] = ex2(fmaf(__uint_as_float(r[4 * i + 0]), c2, -l.x));
-            e[4 * i + 1] = ex2(fmaf(__uint_as_float(r[4 * i + 1]), c2, -l.y));
-            e[4 * i + 2] = ex2(fmaf(__uint_as_float(r[4 * i + 2]), c2, -l.z));
-            e[4 * i + 3] = ex2(fmaf(__uint_as_float(r[4 * i + 3]), c2, -l.w));
+        const int nch = min(256, rows_mma - 256 * hh) / 32;
+        const uint32_t tb = tlane + buf * 256;
+        const float* nl = l2s + hh * 256;
+        // chunk pipeline: load chunk c+1 while chunk c is reduced; the buffer is
+        // released as soon as its last chunk has landed in registers
+        uint32_t ra[32], rb[32];
+        tmem_ld32_async(tb, ra);
+        tmem_wait(ra);
+        for (int ch = 0;; ch += 2) {
+          const bool more_a = ch + 1 < nch;
+          if (more_a) {
+            tmem_ld32_async(tb + (ch + 1) * 32, rb);
+          } else {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
           }
-          acc += tree_sum<32>(e);
+          acc += key_chunk(ra, nl + ch * 32, c2);
+          if (!more_a) break;
+          tmem_wait(rb);
+          const bool more_b = ch + 2 < nch;
+          if (more_b) {
+            tmem_ld32_async(tb + (ch + 2) * 32, ra);
+          } else {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[buf]);
+          }
+          acc += key_chunk(rb, nl + (ch + 1) * 32, c2);
+          if (!more_b) break;
+          tmem_wait(ra);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[buf]);
       }
       if (!ok) break;
       const int key = (t0 + lt) * kKeyTile + quad * 32 + lane;
@@ -454,7 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   if (*abort_flag != 0 && threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
-  if (warp == 2) {
+  if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
