@@ -69,7 +69,7 @@ extern "C" {
  *   doc_offsets           : HOST pointer to batch+1 non-decreasing int64
  *                           offsets, doc_offsets[0] = 0; document b owns
  *                           tokens [doc_offsets[b], doc_offsets[b+1]).
- *   pool_kernel           : K of Eq. 1's average pooling; odd, >= 1 (default 5)
+ *   pool_kernel           : K of Eq. 1's average pooling; odd, 1..33 (default 5)
  *   quant_bits            : b of Eq. 2; only 8 is supported
  *   softmax_scale         : logit scale; <= 0 means 1/sqrt(d)
  *   flags                 : TP_SCORE_KEY_ONLY or 0

@@ -26,8 +26,8 @@ TP_SCORE_KEY_ONLY = 0x1
 TP_MAX_BATCH = 256
 TP_MAX_ROWS = 512
 #: kernels one tp_compress_layer call launches (V scales, two scoring passes,
-#: score formation, two radix passes, threshold/counts, compaction)
-KERNELS_PER_COMPRESS = 8
+#: selection, compaction)
+KERNELS_PER_COMPRESS = 5
 
 #: every symbol include/taskpress.h declares
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",

@@ -30,9 +30,7 @@ struct Plan {
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
-  int max_chunks;
-  size_t ws_status, ws_hist, ws_partials, ws_counts, ws_thresh, ws_lse, ws_skey, ws_gamma, ws_keys,
-      ws_total;
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
 };
 
 int num_sms() {
@@ -56,7 +54,8 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   if (p->guide_len <= 0 || p->batch <= 0 || p->batch > kMaxBatch || !p->doc_offsets)
     return TP_ERR_INVALID_ARG;
   if (p->head_dim != 64 && p->head_dim != 128) return TP_ERR_UNSUPPORTED_SHAPE;
-  if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0) return TP_ERR_UNSUPPORTED_SHAPE;
+  if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0 || p->pool_kernel > 33)
+    return TP_ERR_UNSUPPORTED_SHAPE;
   if (p->quant_bits != 8) return TP_ERR_UNSUPPORTED_SHAPE;
   if (p->flags & ~TP_SCORE_KEY_ONLY) return TP_ERR_INVALID_ARG;
   memset(P, 0, sizeof(*P));
@@ -107,7 +106,7 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->grid_x = P->cta[P->batch];
 
   // Deepest K-tile ring that fits next to the resident guide block.
-  P->stages1 = 4;
+  P->stages1 = 6;
   while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
   P->stages2 = 4;
   while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
@@ -125,23 +124,14 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
     }
   }
 
-  int64_t max_n = 0;
-  for (int b = 0; b < P->batch; ++b) max_n = std::max<int64_t>(max_n, P->off[b + 1] - P->off[b]);
-  P->max_chunks = static_cast<int>((max_n + kChunk - 1) / kChunk);
   const size_t units = size_t(P->hkv) * P->batch;
 
-  // [status | counters | radix histograms] are zeroed at the start of a call.
+  // [status | counters] are zeroed at the start of a call.
   size_t o = 0;
   P->ws_status = o;
   o = align_up(o + sizeof(int) * (1 + units));
-  P->ws_hist = o;
-  o = align_up(o + sizeof(int) * units * kHistInts);
   P->ws_partials = o;
   o = align_up(o + sizeof(float2) * size_t(P->hkv) * P->grid_x * P->rows_pad);
-  P->ws_counts = o;
-  o = align_up(o + sizeof(int2) * units * (P->max_chunks > 0 ? P->max_chunks : 1));
-  P->ws_thresh = o;
-  o = align_up(o + sizeof(int2) * units);
   P->ws_lse = o;
   o = align_up(o + sizeof(float) * size_t(P->batch) * P->hkv * P->rows);
   P->ws_skey = o;
@@ -212,12 +202,13 @@ DocTable doc_table(const Plan& P) {
 
 // Pass 1: row normalisers into `lse` ([batch, H_kv, rows]).  The counters and
 // the status word at the head of the workspace must be zero.
-int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, float* lse, char* ws,
+int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, float* lse, char* ws,
             cudaStream_t s) {
   int* status = reinterpret_cast<int*>(ws + P.ws_status);
   LseParams lp;
   memset(&lp, 0, sizeof(lp));
   lp.docs = doc_table(P);
+  lp.q = static_cast<const uint16_t*>(q);
   lp.n_heads_kv = P.hkv;
   lp.rows = P.rows;
   lp.rows_pad = P.rows_pad;
@@ -229,7 +220,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, float
   lp.lse = lse;
   lp.counters = status + 1;
   lp.status = status;
-  return cuda_status(launch_lse(tmk, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
+  return cuda_status(launch_lse(tmk, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
 }
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
@@ -259,7 +250,7 @@ int run_scoring(const Plan& P, const void* q, const void* k, char* ws, cudaStrea
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
-  int st = run_lse(P, tmk, tmq, lse, ws, s);
+  int st = run_lse(P, tmk, q, lse, ws, s);
   if (st != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), s);
@@ -274,13 +265,8 @@ void fill_select(const Plan& P, char* ws, SelectParams* sp) {
   sp->head_dim = P.d;
   sp->n_total = P.n_total;
   sp->cap = P.cap;
-  sp->max_chunks = P.max_chunks;
   sp->pool_kernel = 1;
-  sp->qmax = 127.0f;
   sp->keys = reinterpret_cast<uint32_t*>(ws + P.ws_keys);
-  sp->hist = reinterpret_cast<int*>(ws + P.ws_hist);
-  sp->counts = reinterpret_cast<int2*>(ws + P.ws_counts);
-  sp->thresh = reinterpret_cast<int2*>(ws + P.ws_thresh);
 }
 
 int zero_head(const Plan& P, char* ws, cudaStream_t s) {
@@ -363,8 +349,8 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
   sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
   sp.gamma = gamma;
   sp.scores_out = scores;
-  sp.hist = nullptr;  // scores only
-  return cuda_status(launch_select(sp, true, s));
+  sp.scores_only = 1;
+  return cuda_status(launch_select(sp, s));
 }
 
 int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
@@ -381,7 +367,7 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, 
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_lse(P, tmk, tmq, lse, w, s);
+  return run_lse(P, tmk, q, lse, w, s);
 }
 
 int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
@@ -411,7 +397,7 @@ int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64
   fill_select(P, w, &sp);
   sp.scores_in = scores;
   sp.idx = idx;
-  return cuda_status(launch_select(sp, false, s));
+  return cuda_status(launch_select(sp, s));
 }
 
 int tp_compact(const tp_problem* p, const void* k, const void* v, const float* gamma,
@@ -468,14 +454,20 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
   sp.gamma = g;
   sp.scores_out = scores;
   sp.idx = idx;
-  sp.gather = 1;
-  sp.k = static_cast<const uint16_t*>(k);
-  sp.v = static_cast<const uint16_t*>(v);
-  sp.kc = static_cast<uint16_t*>(kc);
-  sp.vc = static_cast<uint16_t*>(vc);
-  sp.vqc = vqc;
-  sp.gammac = gammac;
-  return cuda_status(launch_select(sp, false, s));
+  cudaError_t e2 = launch_select(sp, s);
+  if (e2 != cudaSuccess) return TP_ERR_CUDA;
+  if (P.cap == 0) return TP_OK;
+  GatherParams gp;
+  fill_gather(P, &gp);
+  gp.k = static_cast<const uint16_t*>(k);
+  gp.v = static_cast<const uint16_t*>(v);
+  gp.gamma = g;
+  gp.idx = idx;
+  gp.kc = static_cast<uint16_t*>(kc);
+  gp.vc = static_cast<uint16_t*>(vc);
+  gp.vqc = vqc;
+  gp.gammac = gammac;
+  return cuda_status(launch_gather(gp, s));
 }
 
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {

@@ -28,6 +28,7 @@ namespace {
 
 constexpr int kThreads = 576;
 constexpr int kEpiWarp0 = 2;  // first epilogue warp
+constexpr int kEpiWarps = 16;  // four warpgroups
 constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
 
 struct ScoreSmem {
@@ -162,29 +163,35 @@ __device__ __forceinline__ void load_guide(uint8_t* sQ, const CUtensorMap* tmq, 
 
 // ---------------------------------------------------------------------------
 // Pass 1: per-row log-sum-exp of the scaled logits.
+//
+// The group's guide rows stay in tensor memory for the whole CTA (the MMA's A
+// operand, NRB row blocks of 128 rows), so each MMA reads only the K tile from
+// shared memory.  Job (tile, row block) accumulates D[row, key] for 128 keys
+// into one of NB rotating TMEM buffers; all four epilogue warpgroups share
+// every job (warpgroup g owns columns 32g..32g+31), each thread keeping a
+// running (offset, sum) per row block for its row.
 // ---------------------------------------------------------------------------
-template <int D>
+template <int D, int NRB>
 __global__ void __launch_bounds__(kThreads, 1)
-    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
-               const __grid_constant__ LseParams p) {
+    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ LseParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
   constexpr int NKH = D / 64;
   constexpr uint32_t KT = NKH * kHalfTileBytes;
-  const int stages = p.stages, rows_pad = p.rows_pad, nrb = p.nrb;
-  const ScoreSmem L = score_layout(D, rows_pad, stages, 4 * 128 * sizeof(float2));
-  uint8_t* sQ = smem + L.q;
+  constexpr int ACOLS = NRB * D / 2;                       // TMEM columns of the guide rows
+  constexpr int NB = (512 - ACOLS) / 128 < 3 ? (512 - ACOLS) / 128 : 3;  // accumulator buffers
+  const int stages = p.stages, rows_pad = NRB * 128;
+  const ScoreSmem L = score_layout(D, 0, stages, 4 * 512 * sizeof(float2));
   uint8_t* sK = smem + L.k;
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty_k = full_k + stages;
-  uint64_t* q_full = empty_k + stages;
-  uint64_t* tfull = q_full + 1;   // [4], one per epilogue warpgroup = TMEM buffer
-  uint64_t* tempty = tfull + 4;   // [4]
-  uint64_t* drain = tempty + 4;
+  uint64_t* tfull = empty_k + stages;  // [NB]
+  uint64_t* tempty = tfull + 3;        // [NB], one arrival per epilogue warp
+  uint64_t* drain = tempty + 3;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   int* last_flag = reinterpret_cast<int*>(smem + L.misc + 8);
-  float2* stats = reinterpret_cast<float2*>(smem + L.extra);
+  float2* stats = reinterpret_cast<float2*>(smem + L.extra);  // [4 warpgroups][rows_pad]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -196,17 +203,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ntiles = (n + kKeyTile - 1) / kKeyTile;
   const int t0 = c * p.tiles_per_cta;
   const int nt = min(p.tiles_per_cta, ntiles - t0);
-  const int njobs = nt * nrb;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
       mbar_init(&full_k[s], 1);
       mbar_init(&empty_k[s], 1);
     }
-    mbar_init(q_full, 1);
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < NB; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], 4);
+      mbar_init(&tempty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -222,11 +227,37 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  // Guide rows -> TMEM columns [0, ACOLS): warpgroup g writes row block g,
+  // warp quadrant q its 32 rows, one row per thread (rows >= M are zero).
+  if (warp >= kEpiWarp0) {
+    const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
+    if (g < NRB) {
+      const int row = g * 128 + quad * 32 + lane;
+      const uint4* src = reinterpret_cast<const uint4*>(
+          p.q + ((static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows + row) * D);
+      const bool live = row < p.rows;
+#pragma unroll
+      for (int part = 0; part < D / 64; ++part) {
+        uint32_t r[32];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const uint4 v = live ? __ldg(src + part * 8 + i) : make_uint4(0, 0, 0, 0);
+          r[4 * i] = v.x;
+          r[4 * i + 1] = v.y;
+          r[4 * i + 2] = v.z;
+          r[4 * i + 3] = v.w;
+        }
+        tmem_st32(tmem + (static_cast<uint32_t>(quad * 32) << 16) + g * (D / 2) + part * 32, r);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmk);
-      prefetch_tensormap(&tmq);
-      load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
       int issued = 0;
       for (int lt = 0; lt < nt; ++lt) {
         const int s = lt % stages, use = lt / stages;
@@ -239,7 +270,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         issued = lt + 1;
       }
       if (*abort_flag) {  // let in-flight copies land before the CTA exits
-        mbar_drain(q_full, 0);
         for (int lt = max(0, issued - stages); lt < issued; ++lt)
           mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
       }
@@ -248,25 +278,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, kKeyTile);
-      bool ok = mbar_wait(q_full, 0, abort_flag);
+      bool ok = true;
       for (int lt = 0; ok && lt < nt; ++lt) {
         const int s = lt % stages;
         if (!mbar_wait(&full_k[s], (lt / stages) & 1, abort_flag)) break;
         tc_fence_after();
-        for (int rb = 0; rb < nrb; ++rb) {
-          const int j = lt * nrb + rb, buf = j & 3, use = j >> 2;
+#pragma unroll
+        for (int rb = 0; rb < NRB; ++rb) {
+          const int j = lt * NRB + rb, buf = j % NB, use = j / NB;
           if (use > 0 && !mbar_wait(&tempty[buf], (use - 1) & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t dt = tmem + static_cast<uint32_t>(buf * 128);
+          const uint32_t dt = tmem + static_cast<uint32_t>(ACOLS + buf * 128);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const int kh = kk >> 2, k16 = kk & 3;
-            const uint64_t a = sdesc_k128(smem_u32(sQ + (kh * rows_pad + rb * 128) * 128 + k16 * 32));
             const uint64_t bd = sdesc_k128(smem_u32(sK + s * KT + kh * kHalfTileBytes + k16 * 32));
-            mma_bf16_ss(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
+            mma_bf16_ts(dt, tmem + rb * (D / 2) + kk * 8, bd, idesc, kk > 0 ? 1u : 0u);
           }
           mma_commit(&tfull[buf]);
         }
@@ -276,35 +306,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0);
     }
     __syncwarp();
-  } else if (warp >= kEpiWarp0) {
+  } else {
     const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     const float c2 = p.c2;
-    float m = -INFINITY, z = 0.f;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(quad * 32) << 16) + g * 128;
-    for (int j = g, u = 0; j < njobs; j += 4, ++u) {
-      if (!mbar_wait(&tfull[g], u & 1, abort_flag)) break;
-      tc_fence_after();
-      const int lt = j / nrb;
-      const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
-      // four 32-column chunks; the next chunk's TMEM load overlaps this chunk's math
-      uint32_t ra[32], rb[32];
-      tmem_ld32_async(trow, ra);
-      tmem_wait(ra);
-      tmem_ld32_async(trow + 32, rb);
-      lse_chunk(ra, 0, valid, c2, m, z);
-      tmem_wait(rb);
-      tmem_ld32_async(trow + 64, ra);
-      lse_chunk(rb, 32, valid, c2, m, z);
-      tmem_wait(ra);
-      tmem_ld32_async(trow + 96, rb);
-      lse_chunk(ra, 64, valid, c2, m, z);
-      tmem_wait(rb);
-      tc_fence_before();  // TMEM buffer free before the last chunk's math
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[g]);
-      lse_chunk(rb, 96, valid, c2, m, z);
+    float m[NRB], z[NRB];
+#pragma unroll
+    for (int rb = 0; rb < NRB; ++rb) {
+      m[rb] = -INFINITY;
+      z[rb] = 0.f;
     }
-    stats[g * 128 + quad * 32 + lane] = make_float2(m, z);
+    const uint32_t tcol = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ACOLS + g * 32;
+    bool ok = true;
+    for (int lt = 0; ok && lt < nt; ++lt) {
+      const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
+#pragma unroll
+      for (int rb = 0; rb < NRB; ++rb) {
+        const int j = lt * NRB + rb, buf = j % NB;
+        if (ok && !mbar_wait(&tfull[buf], (j / NB) & 1, abort_flag)) ok = false;
+        if (!ok) break;
+        tc_fence_after();
+        uint32_t r[32];
+        tmem_ld32_async(tcol + buf * 128, r);
+        tmem_wait(r);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[buf]);
+        lse_chunk(r, g * 32, valid, c2, m[rb], z[rb]);
+      }
+    }
+#pragma unroll
+    for (int rb = 0; rb < NRB; ++rb) stats[g * rows_pad + rb * 128 + quad * 32 + lane] = make_float2(m[rb], z[rb]);
   }
   __syncthreads();
 
@@ -312,10 +343,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (aborted) {
     if (threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
   } else {
-    if (threadIdx.x < rows_pad) {
-      const int r = threadIdx.x, rb = r >> 7, rr = r & 127;
+    for (int r = threadIdx.x; r < rows_pad; r += blockDim.x) {
       float2 acc = make_float2(-INFINITY, 0.f);
-      for (int g = rb; g < 4; g += nrb) acc = lse_merge(acc, stats[g * 128 + rr]);
+#pragma unroll
+      for (int g = 0; g < 4; ++g) acc = lse_merge(acc, stats[g * rows_pad + r]);
       p.partials[(static_cast<size_t>(h) * gridDim.x + blockIdx.x) * rows_pad + r] = acc;
     }
     __threadfence();
@@ -349,6 +380,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------------------
 // Pass 2: s_key[key] = (1/G) sum over rows of 2^(x*c2 - lse[row]*log2(e)).
+//
+// Keys sit on TMEM lanes (D[key, row] = K Q^T); each MMA job covers one
+// 128-key tile and up to 256 guide rows (N).  All four epilogue warpgroups
+// share every job: warpgroup g reduces the 32-column chunks c = g, g+4 of it,
+// so sixteen warps drain each TMEM buffer.  A thread's partial sum for its key
+// (over its chunks of all row halves of the tile) goes to shared memory, and
+// after a named barrier warpgroup 0 adds the four partials in a fixed order.
 // ---------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -360,18 +398,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr uint32_t KT = NKH * kHalfTileBytes;
   const int stages = p.stages, rows_pad = p.rows_pad, rows_mma = p.rows_mma;
   const int nh = (rows_mma + 255) / 256;
-  const ScoreSmem L = score_layout(D, rows_pad, stages, rows_pad * sizeof(float));
+  const ScoreSmem L = score_layout(D, rows_pad, stages, rows_pad * sizeof(float) + 2 * 4 * 128 * sizeof(float));
   uint8_t* sQ = smem + L.q;
   uint8_t* sK = smem + L.k;
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty_k = full_k + stages;
   uint64_t* q_full = empty_k + stages;
-  uint64_t* tfull = q_full + 1;   // [4 warpgroups][2 row halves]
-  uint64_t* tempty = tfull + 8;   // [2 TMEM buffers]
+  uint64_t* tfull = q_full + 1;   // [2 TMEM buffers]
+  uint64_t* tempty = tfull + 2;   // [2 TMEM buffers], one arrival per epilogue warp
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
-  float* l2s = reinterpret_cast<float*>(smem + L.extra);
+  float* l2s = reinterpret_cast<float*>(smem + L.extra);              // -lse*log2(e) per row
+  float* part = reinterpret_cast<float*>(smem + L.extra + rows_pad * sizeof(float));  // [2][4][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -389,8 +428,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&empty_k[s], 1);
     }
     mbar_init(q_full, 1);
-    for (int i = 0; i < 8; ++i) mbar_init(&tfull[i], 1);
-    for (int i = 0; i < 2; ++i) mbar_init(&tempty[i], 4);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], kEpiWarps);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -457,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 sdesc_k128(smem_u32(sQ + (kh * rows_pad + hh * 256) * 128 + k16 * 32));
             mma_bf16_ss(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
           }
-          mma_commit(&tfull[(lt & 3) * 2 + hh]);
+          mma_commit(&tfull[buf]);
         }
         mma_commit(&empty_k[s]);
       }
@@ -465,56 +506,47 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0);
     }
     __syncwarp();
-  } else if (warp >= kEpiWarp0) {
+  } else {
     const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     const float c2 = p.c2;
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
-    for (int lt = g, it = 0; ok && lt < nt; lt += 4, ++it) {
+    for (int lt = 0; lt < nt; ++lt) {
       float acc = 0.f;
       for (int hh = 0; hh < nh; ++hh) {
-        if (!mbar_wait(&tfull[g * 2 + hh], it & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
+        const int j = lt * nh + hh, buf = j & 1;
+        if (ok && !mbar_wait(&tfull[buf], (j >> 1) & 1, abort_flag)) ok = false;
+        if (!ok) break;
         tc_fence_after();
-        const int buf = (lt * nh + hh) & 1;
         const int nch = min(256, rows_mma - 256 * hh) / 32;
         const uint32_t tb = tlane + buf * 256;
         const float* nl = l2s + hh * 256;
-        // chunk pipeline: load chunk c+1 while chunk c is reduced; the buffer is
-        // released as soon as its last chunk has landed in registers
+        const int c0 = g, c1 = g + 4;
         uint32_t ra[32], rb[32];
-        tmem_ld32_async(tb, ra);
-        tmem_wait(ra);
-        for (int ch = 0;; ch += 2) {
-          const bool more_a = ch + 1 < nch;
-          if (more_a) {
-            tmem_ld32_async(tb + (ch + 1) * 32, rb);
-          } else {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[buf]);
-          }
-          acc += key_chunk(ra, nl + ch * 32, c2);
-          if (!more_a) break;
-          tmem_wait(rb);
-          const bool more_b = ch + 2 < nch;
-          if (more_b) {
-            tmem_ld32_async(tb + (ch + 2) * 32, ra);
-          } else {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[buf]);
-          }
-          acc += key_chunk(rb, nl + (ch + 1) * 32, c2);
-          if (!more_b) break;
-          tmem_wait(ra);
-        }
+        if (c0 < nch) tmem_ld32_async(tb + c0 * 32, ra);
+        if (c1 < nch) tmem_ld32_async(tb + c1 * 32, rb);
+        if (c0 < nch) tmem_wait(ra);
+        if (c1 < nch) tmem_wait(rb);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[buf]);
+        if (c0 < nch) acc += key_chunk(ra, nl + c0 * 32, c2);
+        if (c1 < nch) acc += key_chunk(rb, nl + c1 * 32, c2);
       }
-      if (!ok) break;
-      const int key = (t0 + lt) * kKeyTile + quad * 32 + lane;
-      if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = acc * p.inv_group;
+      // fixed-order sum of the four warpgroups' partials for this tile's keys
+      float* slot = part + (lt & 1) * 4 * 128;
+      if (ok) slot[g * 128 + quad * 32 + lane] = acc;
+      asm volatile("bar.sync 1, %0;" ::"r"(kEpiWarps * 32) : "memory");
+      if (!ok || *abort_flag) {
+        ok = false;
+        continue;
+      }
+      if (g == 0) {
+        const int kl = quad * 32 + lane;
+        const float s4 = ((slot[kl] + slot[128 + kl]) + slot[256 + kl]) + slot[384 + kl];
+        const int key = (t0 + lt) * kKeyTile + kl;
+        if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = s4 * p.inv_group;
+      }
     }
   }
   __syncthreads();
@@ -528,27 +560,36 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
-  return score_layout(head_dim, rows_pad, stages, 4 * 128 * sizeof(float2)).total + 1024;
+  (void)rows_pad;  // the guide rows live in tensor memory
+  return score_layout(head_dim, 0, stages, 4 * 512 * sizeof(float2)).total + 1024;
 }
 
 size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
-  return score_layout(head_dim, rows_pad, stages, rows_pad * sizeof(float)).total + 1024;
+  return score_layout(head_dim, rows_pad, stages,
+                      rows_pad * sizeof(float) + 2 * 4 * 128 * sizeof(float)).total + 1024;
 }
 
-cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmq, const LseParams& p,
-                       int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
-  if (head_dim == 128) {
-    cudaError_t e = cudaFuncSetAttribute(lse_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    lse_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
-  } else {
-    cudaError_t e = cudaFuncSetAttribute(lse_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
-    lse_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
-  }
+template <int D, int NRB>
+cudaError_t launch_lse_t(const CUtensorMap& tmk, const LseParams& p, dim3 grid, size_t smem,
+                         cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(lse_kernel<D, NRB>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  lse_kernel<D, NRB><<<grid, kThreads, smem, s>>>(tmk, p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_lse(const CUtensorMap& tmk, const LseParams& p, int head_dim, dim3 grid,
+                       size_t smem, cudaStream_t s) {
+  if (head_dim == 128) {
+    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, p, grid, smem, s);
+    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, p, grid, smem, s);
+    return launch_lse_t<128, 4>(tmk, p, grid, smem, s);
+  }
+  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, p, grid, smem, s);
+  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, p, grid, smem, s);
+  return launch_lse_t<64, 4>(tmk, p, grid, smem, s);
 }
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,

@@ -8,325 +8,278 @@
 // kept set is every key > T plus the first (k - above) keys equal to T in
 // token order (the lowest-index tie-break), written in ascending order.
 //
-// Every kernel covers one 4096-token chunk of one (document, head) per CTA, so
-// the whole GPU works on each stage:
-//   score_hist  form keys (Eq. 1 pooling x gamma in the fused path) + digit-1 histogram
-//   radix<2,3>  digit-2 / digit-3 histograms of the keys under the chosen prefix
-//   count       threshold T per unit (chunk 0 records it) and (>T, ==T) counts per chunk
-//   compact     ordered compaction into idx, then (fused path) the row gather:
-//               K, V, Eq. 2 int8 codes of V, gamma
-// Histograms are global (atomics on the few non-empty bins) and zeroed by the
-// caller before score_hist.
+// One thread-block cluster of kClusterCtas CTAs handles one (document, head):
+// CTA r owns a contiguous slice of the tokens.  Histograms and per-slice
+// counts live in each CTA's shared memory and are summed across the cluster
+// through distributed shared memory, separated by hardware cluster barriers,
+// so the whole selection is one launch:
+//   A  form keys (Eq. 1 pooling x gamma in the fused path), digit-1 histogram
+//   B  digit-2 histogram under the chosen prefix        C  digit-3 histogram
+//   D  (> T, == T) counts per slice, then the ordered compaction into idx.
+// The kept rows are then copied by the grid-wide gather kernel.
+#include <cooperative_groups.h>
+
 #include "tp_device.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace tp {
 
 namespace {
 
 constexpr int kThreads = 512;
-constexpr int kPer = kChunk / kThreads;  // tokens per thread
+constexpr int kPer = kChunk / kThreads;  // tokens per thread in one compaction round
 constexpr int kBins1 = 2048;             // bits 31..21
 constexpr int kBins2 = 2048;             // bits 20..10
 constexpr int kBins3 = 1024;             // bits 9..0
-constexpr int kMaxHalf = 16;             // pooling half-window supported by the staging strip
 
 __device__ __forceinline__ uint32_t score_key(float s) {
   return (s > 0.f) ? __float_as_uint(s) : 0u;  // -0, +0, NaN and negatives -> 0
 }
 
-struct Unit {
-  int b, h, n, k;
-  int64_t lo;
-  size_t row;  // offset of the unit's first token in [H_kv, N] arrays
-};
-
-__device__ __forceinline__ Unit unit_of(const SelectParams& p) {
-  Unit u;
-  const int unit = blockIdx.y;
-  u.b = unit / p.n_heads_kv;
-  u.h = unit % p.n_heads_kv;
-  u.lo = p.off[u.b];
-  u.n = static_cast<int>(p.off[u.b + 1] - u.lo);
-  u.k = p.kept[u.b];
-  u.row = static_cast<size_t>(u.h) * p.n_total + u.lo;
-  return u;
+// Adds one to hist[bin] for every active lane, one shared atomic per distinct
+// bin in the warp (keys concentrate in few bins).  All 32 lanes must call it.
+__device__ __forceinline__ void hist_add(int* hist, uint32_t bin, bool active) {
+  const unsigned mask = __ballot_sync(0xffffffffu, active);
+  if (!active) return;
+  const unsigned peers = __match_any_sync(mask, bin);
+  if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
 }
 
-// Bin holding the `need`-th largest key (1-based) of a global histogram;
+constexpr int kSliceKeys = 16384;  // keys of a CTA's slice kept in shared memory
+constexpr int kMaxHalf = 16;       // largest pooling half-window of the staging strip
+
+struct SelectSmem {
+  uint32_t keys[kSliceKeys];
+  float strip[kSliceKeys + 2 * kMaxHalf];  // unpooled key scores of a sub-slice + halo
+  int hist1[kBins1];
+  int hist2[kBins2];
+  int hist3[kBins3];
+  int counts[2];  // (> T, == T) in this CTA's slice
+  int scratch[33];
+  int result[2];
+};
+
+// Bin holding the `need`-th largest key (1-based) of the cluster-wide
+// histogram (the sum of every CTA's shared histogram at byte offset `off`);
 // *above = keys in higher bins.  Called by the whole block.
-__device__ int find_digit(const int* ghist, int nbins, int need, int* above, int* scratch,
-                          int* result) {
+__device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const int* local_hist,
+                             int nbins, int need, int* above) {
   const int per = nbins / kThreads;  // 2 or 4 bins per thread, highest bins first
-  int cnt[4];
+  int cnt[4] = {0, 0, 0, 0};
+  for (int r = 0; r < kClusterCtas; ++r) {
+    const int* h = cluster.map_shared_rank(local_hist, r);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < per) cnt[i] += h[nbins - 1 - (threadIdx.x * per + i)];
+  }
   int local = 0;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    cnt[i] = i < per ? __ldcg(ghist + (nbins - 1 - (threadIdx.x * per + i))) : 0;
-    local += cnt[i];
-  }
+  for (int i = 0; i < 4; ++i) local += cnt[i];
   int total;
-  int before = block_excl_scan(local, scratch, &total);
+  int before = block_excl_scan(local, sm.scratch, &total);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     if (i < per && before < need && before + cnt[i] >= need) {
-      result[0] = nbins - 1 - (threadIdx.x * per + i);
-      result[1] = before;
+      sm.result[0] = nbins - 1 - (threadIdx.x * per + i);
+      sm.result[1] = before;
     }
     before += cnt[i];
   }
   __syncthreads();
-  *above = result[1];
-  const int d = result[0];
+  *above = sm.result[1];
+  const int d = sm.result[0];
   __syncthreads();
   return d;
 }
 
-// Adds the non-zero bins of a shared histogram into a global one.
-__device__ __forceinline__ void flush_hist(const int* sh, int* gh, int nbins) {
-  __syncthreads();
-  for (int i = threadIdx.x; i < nbins; i += kThreads) {
-    const int v = sh[i];
-    if (v) atomicAdd(gh + i, v);
-  }
-}
+__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads, 1)
+    select_kernel(const __grid_constant__ SelectParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int unit = blockIdx.y;
+  const int b = unit / p.n_heads_kv, h = unit % p.n_heads_kv;
+  const int64_t lo = p.off[b];
+  const int n = static_cast<int>(p.off[b + 1] - lo);
+  const int k = p.kept[b];
+  const size_t row = static_cast<size_t>(h) * p.n_total + lo;
+  // this CTA's slice [s0, s1) of the document's tokens
+  const int per_cta = (((n + kClusterCtas - 1) / kClusterCtas) + 3) & ~3;
+  const int s0 = min(rank * per_cta, n), s1 = min(s0 + per_cta, n);
+  // the slice's keys: in shared memory when they fit, else in the global scratch
+  const bool in_smem = (s1 - s0 <= kSliceKeys);
+  uint32_t* const keys_base = in_smem ? sm.keys : p.keys + row;
+  const int kofs = in_smem ? s0 : 0;  // keys of token i live at keys_base[i - kofs]
 
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) score_hist_kernel(const __grid_constant__ SelectParams p) {
-  __shared__ int hist[kBins1];
-  __shared__ float strip[kChunk + 2 * kMaxHalf];
-  const Unit u = unit_of(p);
-  const int i0 = blockIdx.x * kChunk;
-  if (i0 >= u.n) return;
-  const int len = min(kChunk, u.n - i0);
-  for (int i = threadIdx.x; i < kBins1; i += kThreads) hist[i] = 0;
+  for (int i = threadIdx.x; i < kBins1; i += kThreads) {
+    sm.hist1[i] = 0;
+    sm.hist2[i] = 0;
+  }
+  for (int i = threadIdx.x; i < kBins3; i += kThreads) sm.hist3[i] = 0;
+  __syncthreads();
+
+  // A: keys of the slice (scores formed here in the fused path) + digit-1 histogram,
+  // in sub-slices of kSliceKeys tokens whose key scores are staged with their halo
   const int half = p.pool_kernel / 2;
-  if (!p.scores_in) {
-    const float* sk = p.skey + u.row;
-    for (int j = threadIdx.x; j < len + 2 * half; j += kThreads) {
-      const int i = i0 - half + j;
-      strip[j] = (i >= 0 && i < u.n) ? sk[i] : 0.f;
-    }
-  }
-  __syncthreads();
   const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
-  for (int j = threadIdx.x; j < len; j += kThreads) {
-    const size_t t = u.row + i0 + j;
-    float s;
-    if (p.scores_in) {
-      s = p.scores_in[t];
-    } else {
-      float acc = 0.f;
-      for (int o = 0; o <= 2 * half; ++o) acc += strip[j + o];
-      s = acc * inv_k;
-      if (!p.key_only) s *= p.gamma[t];
-      if (p.scores_out) p.scores_out[t] = s;
+  for (int c0 = s0; c0 < s1; c0 += kSliceKeys) {
+    const int c1 = min(c0 + kSliceKeys, s1);
+    if (!p.scores_in) {
+      const float* sk = p.skey + row;
+      for (int j = threadIdx.x; j < c1 - c0 + 2 * half; j += kThreads) {
+        const int i = c0 - half + j;
+        sm.strip[j] = (i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
+      }
+      __syncthreads();
     }
-    const uint32_t key = score_key(s);
-    p.keys[t] = key;
-    atomicAdd(&hist[key >> 21], 1);
-  }
-  if (p.hist) flush_hist(hist, p.hist + static_cast<size_t>(blockIdx.y) * kHistInts, kBins1);
-}
-
-template <int PASS>
-__global__ void __launch_bounds__(kThreads) radix_kernel(const __grid_constant__ SelectParams p) {
-  __shared__ int hist[kBins2];
-  __shared__ int scratch[33];
-  __shared__ int result[2];
-  const Unit u = unit_of(p);
-  const int i0 = blockIdx.x * kChunk;
-  if (i0 >= u.n || u.k <= 0 || u.k >= u.n) return;
-  const int len = min(kChunk, u.n - i0);
-  const int* gh = p.hist + static_cast<size_t>(blockIdx.y) * kHistInts;
-  int above;
-  const int d1 = find_digit(gh, kBins1, u.k, &above, scratch, result);
-  uint32_t pre = static_cast<uint32_t>(d1);
-  if (PASS == 3) {
-    const int d2 = find_digit(gh + kBins1, kBins2, u.k - above, &above, scratch, result);
-    pre = (pre << 11) | static_cast<uint32_t>(d2);
-  }
-  const int nb = PASS == 2 ? kBins2 : kBins3;
-  for (int i = threadIdx.x; i < nb; i += kThreads) hist[i] = 0;
-  __syncthreads();
-  const uint32_t* keys = p.keys + u.row + i0;
-  for (int j = threadIdx.x; j < len; j += kThreads) {
-    const uint32_t key = keys[j];
-    if (PASS == 2) {
-      if ((key >> 21) == pre) atomicAdd(&hist[(key >> 10) & 0x7FF], 1);
-    } else {
-      if ((key >> 10) == pre) atomicAdd(&hist[key & 0x3FF], 1);
-    }
-  }
-  flush_hist(hist, const_cast<int*>(gh) + (PASS == 2 ? kBins1 : kBins1 + kBins2), nb);
-}
-
-__global__ void __launch_bounds__(kThreads) count_kernel(const __grid_constant__ SelectParams p) {
-  __shared__ int scratch[33];
-  __shared__ int result[2];
-  const Unit u = unit_of(p);
-  const int i0 = blockIdx.x * kChunk;
-  if (i0 >= u.n || u.k <= 0) return;
-  const int len = min(kChunk, u.n - i0);
-  int2* counts = p.counts + static_cast<size_t>(blockIdx.y) * p.max_chunks;
-  if (u.k >= u.n) {  // everything kept
-    if (threadIdx.x == 0) {
-      counts[blockIdx.x] = make_int2(len, 0);
-      if (blockIdx.x == 0) p.thresh[blockIdx.y] = make_int2(0, -1);
-    }
-    return;
-  }
-  const int* gh = p.hist + static_cast<size_t>(blockIdx.y) * kHistInts;
-  int a1, a2, a3;
-  const int d1 = find_digit(gh, kBins1, u.k, &a1, scratch, result);
-  const int d2 = find_digit(gh + kBins1, kBins2, u.k - a1, &a2, scratch, result);
-  const int d3 = find_digit(gh + kBins1 + kBins2, kBins3, u.k - a1 - a2, &a3, scratch, result);
-  const uint32_t thr = (static_cast<uint32_t>(d1) << 21) | (static_cast<uint32_t>(d2) << 10) |
-                       static_cast<uint32_t>(d3);
-  const int need_eq = u.k - a1 - a2 - a3;
-  const uint32_t* keys = p.keys + u.row + i0;
-  int gt = 0, eq = 0;
-  for (int j = threadIdx.x; j < len; j += kThreads) {
-    const uint32_t key = keys[j];
-    gt += key > thr;
-    eq += key == thr;
-  }
-  int tg, te;
-  block_excl_scan(gt, scratch, &tg);
-  block_excl_scan(eq, scratch, &te);
-  if (threadIdx.x == 0) {
-    counts[blockIdx.x] = make_int2(tg, te);
-    if (blockIdx.x == 0) p.thresh[blockIdx.y] = make_int2(static_cast<int>(thr), need_eq);
-  }
-}
-
-// Copies one kept row: K lanes then V lanes (LPR lanes each), int8 codes of V.
-template <int LPR>
-__device__ __forceinline__ void copy_row(const SelectParams& p, const Unit& u, int64_t slot_index,
-                                         int token, int lane_in_pair) {
-  const bool is_v = lane_in_pair >= LPR;
-  const int part = lane_in_pair % LPR;
-  const int64_t tok = static_cast<int64_t>(u.h) * p.n_total + u.lo + token;
-  const int64_t dst = slot_index * LPR + part;
-  if (!is_v) {
-    if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] =
-        __ldcs(reinterpret_cast<const uint4*>(p.k) + tok * LPR + part);
-  } else {
-    const uint4 v = __ldcs(reinterpret_cast<const uint4*>(p.v) + tok * LPR + part);
-    if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = v;
-    const float g = p.gamma[tok];
-    if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = quant8_bf16(v, g, p.qmax);
-    if (p.gammac && part == 0) p.gammac[slot_index] = g;
-  }
-}
-
-template <int LPR>
-__global__ void __launch_bounds__(kThreads) compact_kernel(const __grid_constant__ SelectParams p) {
-  __shared__ int scratch[33];
-  __shared__ int2 list[kChunk];  // (slot, token) of the rows this CTA keeps
-  __shared__ int nlist;
-  const Unit u = unit_of(p);
-  const int i0 = blockIdx.x * kChunk;
-  const int64_t unit_slot0 = static_cast<int64_t>(blockIdx.y) * p.cap;
-  // padding slots [k, cap): chunk 0 of the unit (also for empty documents)
-  if (blockIdx.x == 0) {
-    const int k0 = max(0, min(u.k, u.n));
-    for (int64_t t = k0 + threadIdx.x; t < p.cap; t += kThreads) p.idx[unit_slot0 + t] = -1;
-    if (p.gather) {
-      constexpr int SPW = 32 / (2 * LPR);
-      const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-      for (int64_t t = k0 + warp * SPW + lane / (2 * LPR); t < p.cap; t += (kThreads / 32) * SPW) {
-        const int lp = lane % (2 * LPR);
-        const int part = lp % LPR;
-        const int64_t dst = (unit_slot0 + t) * LPR + part;
-        if (lp < LPR) {
-          if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = make_uint4(0, 0, 0, 0);
-        } else {
-          if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = make_uint4(0, 0, 0, 0);
-          if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = make_uint2(0, 0);
-          if (p.gammac && part == 0) p.gammac[unit_slot0 + t] = 0.f;
+    for (int base = c0; base < c1; base += 4 * kThreads) {
+      float sv[4];
+      bool live[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = base + u * kThreads + threadIdx.x;
+        live[u] = i < c1;
+        sv[u] = 0.f;
+        if (live[u]) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
+                                         : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = base + u * kThreads + threadIdx.x;
+        uint32_t key = 0;
+        if (live[u]) {
+          float s = sv[u];
+          if (!p.scores_in) {
+            float acc = 0.f;
+            const float* w = sm.strip + (i - c0);
+            for (int o = 0; o <= 2 * half; ++o) acc += w[o];
+            s = p.key_only ? acc * inv_k : (acc * inv_k) * sv[u];
+            if (p.scores_out) p.scores_out[row + i] = s;
+          }
+          key = score_key(s);
+          keys_base[i - kofs] = key;
         }
+        if (!p.scores_only) hist_add(sm.hist1, key >> 21, live[u]);
       }
     }
+    __syncthreads();
   }
-  if (i0 >= u.n || u.k <= 0) return;
-  const int len = min(kChunk, u.n - i0);
-  const int2 th = p.thresh[blockIdx.y];
-  const uint32_t thr = static_cast<uint32_t>(th.x);
-  const int need_eq = th.y;  // -1: keep everything
-  // tokens > T and == T in the chunks before this one
-  const int2* counts = p.counts + static_cast<size_t>(blockIdx.y) * p.max_chunks;
+  if (p.scores_only) return;  // no cluster-wide exchange follows
+
+  const int64_t unit_slot0 = static_cast<int64_t>(unit) * p.cap;
+  const int kk = max(0, min(k, n));
+  if (rank == 0)
+    for (int64_t t = kk + threadIdx.x; t < p.cap; t += kThreads) p.idx[unit_slot0 + t] = -1;
+  cluster.sync();  // histograms of phase A complete everywhere
+
+  uint32_t thr = 0;
+  int need_eq = -1;  // -1: keep every token of the document
+  if (kk > 0 && kk < n) {
+    int above;
+    const int d1 = cluster_digit(cluster, sm, sm.hist1, kBins1, kk, &above);
+    int need = kk - above;
+    for (int base = s0; base < s1; base += kThreads) {
+      const int i = base + threadIdx.x;
+      const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
+      hist_add(sm.hist2, (key >> 10) & 0x7FF, i < s1 && (key >> 21) == static_cast<uint32_t>(d1));
+    }
+    cluster.sync();
+    const int d2 = cluster_digit(cluster, sm, sm.hist2, kBins2, need, &above);
+    need -= above;
+    const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
+    for (int base = s0; base < s1; base += kThreads) {
+      const int i = base + threadIdx.x;
+      const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
+      hist_add(sm.hist3, key & 0x3FF, i < s1 && (key >> 10) == pre);
+    }
+    cluster.sync();
+    const int d3 = cluster_digit(cluster, sm, sm.hist3, kBins3, need, &above);
+    need_eq = need - above;
+    thr = (pre << 10) | static_cast<uint32_t>(d3);
+  } else {
+    // the cluster-wide barriers must match on every CTA
+    cluster.sync();
+    cluster.sync();
+  }
+
+  // D: counts of this slice, then prefix over the slices before it
+  {
+    int gt = 0, eq = 0;
+    if (kk > 0) {
+      for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
+        const uint32_t key = keys_base[i - kofs];
+        if (need_eq < 0 || key > thr) ++gt;
+        else if (key == thr) ++eq;
+      }
+    }
+    gt = block_sum(gt, sm.scratch);
+    eq = block_sum(eq, sm.scratch);
+    if (threadIdx.x == 0) {
+      sm.counts[0] = gt;
+      sm.counts[1] = eq;
+    }
+  }
+  cluster.sync();
   int gt_before = 0, eq_before = 0;
-  for (int c = threadIdx.x; c < blockIdx.x; c += kThreads) {
-    const int2 v = __ldcg(counts + c);
-    gt_before += v.x;
-    eq_before += v.y;
+  for (int r = 0; r < rank; ++r) {
+    const int* c = cluster.map_shared_rank(sm.counts, r);
+    gt_before += c[0];
+    eq_before += c[1];
   }
-  gt_before = block_sum(gt_before, scratch);
-  eq_before = block_sum(eq_before, scratch);
-  // ordered compaction: kPer consecutive tokens per thread.  A token's slot is
-  // (tokens > T before it) + min(tokens == T before it, need_eq).
-  const uint32_t* keys = p.keys + u.row + i0;
-  const int j0 = threadIdx.x * kPer;
-  int ngt = 0, neq = 0;
-  uint32_t kk[kPer];
+  cluster.sync();  // no CTA leaves while another may still read its counts
+
+  if (kk <= 0) return;
+  // ordered compaction in rounds of kChunk tokens: a token's slot is
+  // (tokens > T before it) + min(tokens == T before it, need_eq)
+  for (int base = s0; base < s1; base += kChunk) {
+    const int j0 = base + threadIdx.x * kPer;
+    int ngt = 0, neq = 0;
+    uint32_t kv[kPer];
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) {
-    const int j = j0 + e;
-    kk[e] = j < len ? keys[j] : 0u;
-    if (j < len) {
-      if (need_eq < 0 || kk[e] > thr) ++ngt;
-      else if (kk[e] == thr) ++neq;
-    }
-  }
-  int tot;
-  int gt_rank = gt_before + block_excl_scan(ngt, scratch, &tot);
-  int eq_rank = eq_before + block_excl_scan(neq, scratch, &tot);
-  if (threadIdx.x == 0) nlist = 0;
-  __syncthreads();
-#pragma unroll
-  for (int e = 0; e < kPer; ++e) {
-    const int j = j0 + e;
-    if (j >= len) break;
-    const bool is_gt = need_eq < 0 || kk[e] > thr;
-    const bool is_eq = !is_gt && kk[e] == thr;
-    if (is_gt || (is_eq && eq_rank < need_eq)) {
-      const int slot = gt_rank + (need_eq < 0 ? 0 : min(eq_rank, need_eq));
-      p.idx[unit_slot0 + slot] = i0 + j;
-      if (p.gather) {
-        const int at = atomicAdd(&nlist, 1);
-        list[at] = make_int2(slot, i0 + j);
+    for (int e = 0; e < kPer; ++e) {
+      const int j = j0 + e;
+      kv[e] = j < s1 ? keys_base[j - kofs] : 0u;
+      if (j < s1) {
+        if (need_eq < 0 || kv[e] > thr) ++ngt;
+        else if (kv[e] == thr) ++neq;
       }
     }
-    gt_rank += is_gt;
-    eq_rank += is_eq;
-  }
-  if (!p.gather) return;
-  __syncthreads();
-  constexpr int SPW = 32 / (2 * LPR);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m = nlist;
-  for (int e = warp * SPW + lane / (2 * LPR); e < m; e += (kThreads / 32) * SPW) {
-    const int2 st = list[e];
-    copy_row<LPR>(p, u, unit_slot0 + st.x, st.y, lane % (2 * LPR));
+    int tot_gt, tot_eq;
+    int gt_rank = gt_before + block_excl_scan(ngt, sm.scratch, &tot_gt);
+    int eq_rank = eq_before + block_excl_scan(neq, sm.scratch, &tot_eq);
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      const int j = j0 + e;
+      if (j >= s1) break;
+      const bool is_gt = need_eq < 0 || kv[e] > thr;
+      const bool is_eq = !is_gt && kv[e] == thr;
+      if (is_gt || (is_eq && eq_rank < need_eq)) {
+        const int slot = gt_rank + (need_eq < 0 ? 0 : min(eq_rank, need_eq));
+        p.idx[unit_slot0 + slot] = j;
+      }
+      gt_rank += is_gt;
+      eq_rank += is_eq;
+    }
+    gt_before += tot_gt;
+    eq_before += tot_eq;
   }
 }
 
 }  // namespace
 
-cudaError_t launch_select(const SelectParams& p, bool form_scores_only, cudaStream_t s) {
+size_t select_smem_bytes() { return sizeof(SelectSmem); }
+
+cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
   const int units = p.batch * p.n_heads_kv;
-  if (units <= 0 || p.max_chunks <= 0) return cudaSuccess;
+  if (units <= 0) return cudaSuccess;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
-  const dim3 grid(p.max_chunks, units);
-  score_hist_kernel<<<grid, kThreads, 0, s>>>(p);
-  if (form_scores_only) return cudaGetLastError();
-  radix_kernel<2><<<grid, kThreads, 0, s>>>(p);
-  radix_kernel<3><<<grid, kThreads, 0, s>>>(p);
-  count_kernel<<<grid, kThreads, 0, s>>>(p);
-  if (p.head_dim == 64)
-    compact_kernel<8><<<grid, kThreads, 0, s>>>(p);
-  else
-    compact_kernel<16><<<grid, kThreads, 0, s>>>(p);
+  const size_t smem = sizeof(SelectSmem);
+  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  select_kernel<<<dim3(kClusterCtas, units), kThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 

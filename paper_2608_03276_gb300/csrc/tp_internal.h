@@ -33,6 +33,7 @@ __host__ __device__ inline int find_doc(const DocTable& t, int cta) {
 // per-(document, head) merge by the last CTA to finish.
 struct LseParams {
   DocTable docs;
+  const uint16_t* q;  // guide rows [batch * H_kv, rows, d] bf16
   int n_heads_kv;
   int rows;          // M = G * L_t
   int rows_pad;      // 128 * nrb
@@ -63,8 +64,8 @@ struct KeyScoreParams {
   int* status;
 };
 
-constexpr int kChunk = 4096;      // tokens per CTA in the selection kernels
-constexpr int kHistInts = 2048 + 2048 + 1024;  // radix histograms per unit
+constexpr int kChunk = 4096;       // tokens per compaction round in the selection kernel
+constexpr int kClusterCtas = 8;    // CTAs (one cluster) per (document, head) in the selection
 
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
@@ -74,26 +75,15 @@ struct SelectParams {
   int head_dim;
   int64_t n_total;
   int64_t cap;
-  int max_chunks;            // chunks of the longest document
   int pool_kernel;           // >= 1, odd
   int key_only;
-  int gather;                // fused path: also write the compressed rows
-  float qmax;
+  int scores_only;           // form the scores (and keys) and stop
   const float* scores_in;    // combined scores (tp_select) or null
   const float* skey;         // unpooled key scores (fused path) or null
   const float* gamma;        // per-token scale (fused path) or null
   float* scores_out;         // optional combined scores out (fused path)
   uint32_t* keys;            // [H_kv, N] scratch
-  int* hist;                 // [units, kHistInts] scratch, zero at launch
-  int2* counts;              // [units, max_chunks] scratch
-  int2* thresh;              // [units] scratch
   int32_t* idx;              // [batch, H_kv, cap]
-  const uint16_t* k;         // rows gathered when `gather`
-  const uint16_t* v;
-  uint16_t* kc;
-  uint16_t* vc;
-  int8_t* vqc;
-  float* gammac;
 };
 
 struct GatherParams {
@@ -117,12 +107,12 @@ struct GatherParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int num_sms, cudaStream_t s);
-cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmq, const LseParams& p,
-                       int head_dim, dim3 grid, size_t smem, cudaStream_t s);
+cudaError_t launch_lse(const CUtensorMap& tmk, const LseParams& p, int head_dim, dim3 grid,
+                       size_t smem, cudaStream_t s);
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             cudaStream_t s);
-cudaError_t launch_select(const SelectParams& p, bool form_scores_only, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s);
 
 // Shared-memory layout sizes of the scoring kernels (host side).

@@ -54,49 +54,48 @@ __global__ void __launch_bounds__(256) vquant_kernel(const uint4* __restrict__ v
 }
 
 // Compaction: one (document, head, slot) per LPR-lane group for K and one for
-// V; idx < 0 marks an unused slot (zero-filled).
+// V, kUnroll slot groups per warp with their loads in flight together; idx < 0
+// marks an unused slot (zero-filled).
 template <int LPR>
 __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherParams p) {
-  constexpr int SPW = 32 / (2 * LPR);  // slots per warp
+  constexpr int SPW = 32 / (2 * LPR);  // slots per warp instruction
+  constexpr int UNR = 8;
   const int lane = threadIdx.x & 31;
-  const int grp = lane / (2 * LPR);            // slot within the warp
-  const bool is_v = (lane % (2 * LPR)) >= LPR;  // K lanes then V lanes
-  const int part = lane % LPR;
+  const int lp = lane % (2 * LPR), part = lp % LPR;
+  const bool is_v = lp >= LPR;  // K lanes then V lanes
   const int b = blockIdx.z, h = blockIdx.y;
   const int64_t unit = static_cast<int64_t>(b) * p.n_heads_kv + h;
   const int64_t warp_global = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int64_t t = warp_global * SPW + grp;
-  if (t >= p.cap) return;
-  const int64_t slot = unit * p.cap + t;
-  const int32_t j = p.idx[slot];
-  const int64_t dst = slot * LPR + part;
-  if (j < 0) {
-    const uint4 z = make_uint4(0, 0, 0, 0);
-    if (!is_v) {
-      if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = z;
-    } else {
-      if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = z;
-      if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = make_uint2(0, 0);
-      if (p.gammac && part == 0) p.gammac[slot] = 0.f;
-    }
-    return;
+  const int64_t t0 = warp_global * SPW * UNR + lane / (2 * LPR);
+  const uint4* src = reinterpret_cast<const uint4*>(is_v ? p.v : p.k);
+  int32_t j[UNR];
+  uint4 val[UNR];
+#pragma unroll
+  for (int u = 0; u < UNR; ++u) {
+    const int64_t t = t0 + u * SPW;
+    j[u] = t < p.cap ? p.idx[unit * p.cap + t] : -2;
   }
-  const int64_t tok = static_cast<int64_t>(h) * p.n_total + p.off[b] + j;
-  if (!is_v) {
-    if (p.kc) {
-      const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.k) + tok * LPR + part);
-      reinterpret_cast<uint4*>(p.kc)[dst] = u;
+#pragma unroll
+  for (int u = 0; u < UNR; ++u) {
+    val[u] = make_uint4(0, 0, 0, 0);
+    if (j[u] >= 0) {
+      const int64_t tok = static_cast<int64_t>(h) * p.n_total + p.off[b] + j[u];
+      val[u] = __ldcs(src + tok * LPR + part);
     }
-  } else {
-    const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p.v) + tok * LPR + part);
-    if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = u;
-    const float g = p.gamma[tok];
-    if (p.vqc) {
-      float f[8];
-      bf16x8_to_f32(u, f);
-      reinterpret_cast<uint2*>(p.vqc)[dst] = quant8(f, g, p.qmax);
+  }
+#pragma unroll
+  for (int u = 0; u < UNR; ++u) {
+    if (j[u] == -2) continue;
+    const int64_t slot = unit * p.cap + t0 + u * SPW;
+    const int64_t dst = slot * LPR + part;
+    if (!is_v) {
+      if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = val[u];
+    } else {
+      const float g = j[u] >= 0 ? p.gamma[static_cast<int64_t>(h) * p.n_total + p.off[b] + j[u]] : 0.f;
+      if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = val[u];
+      if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_bf16(val[u], g, p.qmax) : make_uint2(0, 0);
+      if (p.gammac && part == 0) p.gammac[slot] = g;
     }
-    if (p.gammac && part == 0) p.gammac[slot] = g;
   }
 }
 
@@ -125,7 +124,7 @@ cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
   if (p.cap <= 0) return cudaSuccess;
   const int threads = 256;
   const int lpr = p.head_dim / 8;
-  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr));
+  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr)) * 8;
   dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
             p.batch);
   if (p.head_dim == 128)

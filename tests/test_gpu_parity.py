@@ -228,6 +228,22 @@ def test_select_bit_exact(cuda_lib, budget):
             assert np.all(got[b, h, k:] == -1)
 
 
+@pytest.mark.parametrize("budget", [1, 14000, 139999])
+def test_select_long_document(cuda_lib, budget):
+    """A document longer than the shared-memory key slices (8 x 16384 tokens)."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    n = 140000
+    rng = np.random.Generator(np.random.PCG64(budget + 7))
+    sc = np.round(rng.random((1, n)) * 64).astype(np.float32) / 64  # many ties
+    p = binding.Problem(2, 1, 128, 4, [0, n])
+    idx = torch.empty((1, 1, budget), dtype=torch.int32, device="cuda")
+    ws = torch.empty(binding.tp_workspace_bytes(p, 0.0, budget), dtype=torch.uint8, device="cuda")
+    binding.tp_select(p, torch.tensor(sc, device="cuda"), 0.0, budget, idx, ws)
+    want = O.select_topk(sc[0].astype(np.float64), budget)
+    assert np.array_equal(idx.cpu().numpy()[0, 0], want)
+
+
 @pytest.mark.parametrize("ratio", [0.0, 0.07, 0.5, 1.0])
 def test_select_ratio(cuda_lib, ratio):
     import torch
