@@ -310,7 +310,7 @@ def run_ours(args, w):
     skey = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
     gamma = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
     scores = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
-    stage_names = ["vquant", "lse", "keyscore", "select+compact"]
+    stage_names = ["lse+vscale", "keyscore", "select", "gather"]
     stage_ms = {s: 0.0 for s in stage_names}
     reps = max(1, args.steps)
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
@@ -318,35 +318,32 @@ def run_ours(args, w):
     for _ in range(reps):
         for li in range(nlayer_stage):
             (q, k, v), o = layers[li], outs[li]
-            evs[0].record(stream)
-            binding.tp_quantize_v(p, v, None, gamma, stream)
-            evs[1].record(stream)
-            binding.tp_guide_lse(p, q, k, lse, ws, stream)
-            evs[2].record(stream)
-            binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
-            evs[3].record(stream)
             binding.tp_guide_scores(p, q, k, gamma, scores, ws, stream)  # scores for select; not timed
-            evs[4].record(stream)
+            evs[0].record(stream)
+            binding.tp_guide_lse(p, q, k, lse, ws, stream, v=v, gamma=gamma)
+            evs[1].record(stream)
+            binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
+            evs[2].record(stream)
             binding.tp_select(p, scores, w.keep_ratio, w.budget, o.idx, ws, stream)
+            evs[3].record(stream)
             binding.tp_compact(p, k, v, gamma, o.idx, w.keep_ratio, w.budget, o.kc, o.vc, o.vqc,
                                o.gammac, stream)
-            evs[5].record(stream)
+            evs[4].record(stream)
             torch.cuda.synchronize()
-            stage_ms["vquant"] += evs[0].elapsed_time(evs[1])
-            stage_ms["lse"] += evs[1].elapsed_time(evs[2])
-            stage_ms["keyscore"] += evs[2].elapsed_time(evs[3])
-            stage_ms["select+compact"] += evs[4].elapsed_time(evs[5])
+            for i, name in enumerate(stage_names):
+                stage_ms[name] += evs[i].elapsed_time(evs[i + 1])
     nstage = reps * nlayer_stage
     stage_ms = {s: v / nstage for s, v in stage_ms.items()}
 
     read_b, write_b, flops1 = layer_algorithmic(w, kept_tokens)
-    dom = max(("lse", "keyscore"), key=lambda s: stage_ms[s])
+    dom = max(("lse+vscale", "keyscore"), key=lambda s: stage_ms[s])
     dom_ms = stage_ms[dom]
     achieved = flops1 / (dom_ms / 1e3) / 1e12
-    roofline = {"bound": "tensor", "kernel": f"{dom}_kernel", "achieved": achieved,
+    kname = {"lse+vscale": "lse_kernel", "keyscore": "keyscore_kernel"}[dom]
+    roofline = {"bound": "tensor", "kernel": kname, "achieved": achieved,
                 "peak": tf_sust, "unit": "TFLOP/s", "frac": achieved / tf_sust,
                 "peak_source": f"{peak_src} bf16 sustained",
-                "traffic": traffic_record(f"{dom}_kernel", w.name),
+                "traffic": traffic_record(kname, w.name),
                 "per_launch_ms": dom_ms,
                 "flops_per_launch": flops1}
     t_layer_s = ms / L / 1e3

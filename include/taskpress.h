@@ -140,10 +140,13 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
  * for the M = G*L_t stacked guide rows r of KV head h (rows ordered query
  * head-major within the group, then guide token).  q, k as in tp_guide_scores;
  * lse: [batch, H_kv, M] fp32 out (natural log).  Empty documents are skipped.
+ * With v ([H_kv, N, d] bf16) and gamma ([H_kv, N] fp32 out) both non-NULL, the
+ * same pass also writes the Eq. 2 scales of every token (as tp_quantize_v),
+ * reading V alongside K; both NULL skips that.
  * ws / ws_bytes: workspace of at least tp_workspace_bytes(p, 0, 0).
  */
-int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
-                 size_t ws_bytes, void* stream);
+int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* v, float* lse,
+                 float* gamma, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * Stage 2 of the scores (Sec. 3.2, Eq. 1's inner sums): given the row

@@ -25,9 +25,9 @@ TP_ERR_TIMEOUT = -5
 TP_SCORE_KEY_ONLY = 0x1
 TP_MAX_BATCH = 256
 TP_MAX_ROWS = 512
-#: kernels one tp_compress_layer call launches (V scales, two scoring passes,
-#: selection, compaction)
-KERNELS_PER_COMPRESS = 5
+#: kernels one tp_compress_layer call launches (scoring pass 1 with the V
+#: scales, scoring pass 2, selection, compaction)
+KERNELS_PER_COMPRESS = 4
 
 #: every symbol include/taskpress.h declares
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
@@ -81,7 +81,7 @@ def load(path: Optional[str] = None):
                                     c_void_p, c_size_t, c_void_p]
     lib.tp_guide_lse.restype = c_int
     lib.tp_guide_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
-                                 c_size_t, c_void_p]
+                                 c_void_p, c_void_p, c_size_t, c_void_p]
     lib.tp_guide_key_scores.restype = c_int
     lib.tp_guide_key_scores.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
                                         c_void_p]
@@ -192,14 +192,16 @@ def tp_guide_scores(p: Problem, q, k, gamma, scores, ws, stream=None):
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 
-def tp_guide_lse(p: Problem, q, k, lse, ws, stream=None):
+def tp_guide_lse(p: Problem, q, k, lse, ws, stream=None, v=None, gamma=None):
     import torch
     hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
     rows = (hq // hkv) * lt
     _check("tp_guide_lse", load().tp_guide_lse(
         p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
         _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(v, torch.bfloat16, hkv * n * d, "v", nullable=True),
         _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 

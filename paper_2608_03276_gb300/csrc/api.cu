@@ -106,7 +106,7 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->grid_x = P->cta[P->batch];
 
   // Deepest K-tile ring that fits next to the resident guide block.
-  P->stages1 = 6;
+  P->stages1 = 6;  // K ring of pass 1 (next to its 2-stage V ring)
   while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
   P->stages2 = 4;
   while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
@@ -200,15 +200,21 @@ DocTable doc_table(const Plan& P) {
   return docs;
 }
 
-// Pass 1: row normalisers into `lse` ([batch, H_kv, rows]).  The counters and
+// Pass 1: row normalisers into `lse` ([batch, H_kv, rows]), and the Eq. 2
+// scales of every token into `gamma` when v/gamma are given.  The counters and
 // the status word at the head of the workspace must be zero.
-int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, float* lse, char* ws,
-            cudaStream_t s) {
+int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, const void* v, float* gamma,
+            float* lse, char* ws, cudaStream_t s) {
+  CUtensorMap tmv = tmk;
+  if (gamma && !encode_3d(&tmv, v, P.d, P.n_total, P.hkv, 128)) return TP_ERR_CUDA;
   int* status = reinterpret_cast<int*>(ws + P.ws_status);
   LseParams lp;
   memset(&lp, 0, sizeof(lp));
   lp.docs = doc_table(P);
   lp.q = static_cast<const uint16_t*>(q);
+  lp.gamma = gamma;
+  lp.qmax = 127.0f;
+  lp.n_total = P.n_total;
   lp.n_heads_kv = P.hkv;
   lp.rows = P.rows;
   lp.rows_pad = P.rows_pad;
@@ -220,7 +226,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, float* lse, ch
   lp.lse = lse;
   lp.counters = status + 1;
   lp.status = status;
-  return cuda_status(launch_lse(tmk, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
+  return cuda_status(launch_lse(tmk, tmv, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
 }
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
@@ -244,13 +250,15 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
   return cuda_status(launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, s));
 }
 
-// Both scoring passes; leaves the unpooled key scores in the workspace.
-int run_scoring(const Plan& P, const void* q, const void* k, char* ws, cudaStream_t s) {
+// Both scoring passes (with the Eq. 2 scales fused into the first when gamma
+// is given); leaves the unpooled key scores in the workspace.
+int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
+                cudaStream_t s) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
-  int st = run_lse(P, tmk, q, lse, ws, s);
+  int st = run_lse(P, tmk, q, v, gamma, lse, ws, s);
   if (st != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), s);
@@ -341,7 +349,7 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  if ((st = run_scoring(P, q, k, w, s)) != TP_OK) return st;
+  if ((st = run_scoring(P, q, k, nullptr, nullptr, w, s)) != TP_OK) return st;
   SelectParams sp;
   fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;
@@ -353,12 +361,13 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
   return cuda_status(launch_select(sp, s));
 }
 
-int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, void* ws,
-                 size_t ws_bytes, void* stream) {
+int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* v, float* lse,
+                 float* gamma, void* ws, size_t ws_bytes, void* stream) {
   Plan P;
   int st = make_plan(p, 0.0, 0, false, &P);
   if (st != TP_OK) return st;
   if (!q || !k || !lse || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
+  if ((v == nullptr) != (gamma == nullptr) || (v && !aligned16(v))) return TP_ERR_INVALID_ARG;
   if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
     return TP_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -367,7 +376,7 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, float* lse, 
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_lse(P, tmk, q, lse, w, s);
+  return run_lse(P, tmk, q, v, gamma, lse, w, s);
 }
 
 int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
@@ -442,10 +451,7 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
   char* w = static_cast<char*>(ws);
   float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  cudaError_t e = launch_vquant(static_cast<const uint16_t*>(v), nullptr, g,
-                                int64_t(P.hkv) * P.n_total, P.d, 127.0f, num_sms(), s);
-  if (e != cudaSuccess) return TP_ERR_CUDA;
-  if ((st = run_scoring(P, q, k, w, s)) != TP_OK) return st;
+  if ((st = run_scoring(P, q, k, v, g, w, s)) != TP_OK) return st;
   SelectParams sp;
   fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;

@@ -26,7 +26,10 @@ namespace tp {
 
 namespace {
 
-constexpr int kThreads = 576;
+constexpr int kThreads = 576;      // pass 2: TMA, MMA, 16 epilogue warps
+constexpr int kLseThreads = 640;   // pass 1: the same plus 2 V-scale warps
+constexpr int kVWarp0 = 18;        // first V-scale warp of pass 1
+constexpr int kVStages = 2;        // V-tile ring depth of pass 1
 constexpr int kEpiWarp0 = 2;  // first epilogue warp
 constexpr int kEpiWarps = 16;  // four warpgroups
 constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
@@ -170,10 +173,15 @@ __device__ __forceinline__ void load_guide(uint8_t* sQ, const CUtensorMap* tmq, 
 // into one of NB rotating TMEM buffers; all four epilogue warpgroups share
 // every job (warpgroup g owns columns 32g..32g+31), each thread keeping a
 // running (offset, sum) per row block for its row.
+//
+// With p.gamma set, the same CTA also produces the Eq. 2 scale of every token
+// of its key range: the producer streams the V tiles into a second ring and
+// two warps reduce each row's absmax (the V stream hides under the scoring).
 // ---------------------------------------------------------------------------
 template <int D, int NRB>
-__global__ void __launch_bounds__(kThreads, 1)
-    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ LseParams p) {
+__global__ void __launch_bounds__(kLseThreads, 1)
+    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+               const __grid_constant__ LseParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
   constexpr int NKH = D / 64;
@@ -181,13 +189,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int ACOLS = NRB * D / 2;                       // TMEM columns of the guide rows
   constexpr int NB = (512 - ACOLS) / 128 < 3 ? (512 - ACOLS) / 128 : 3;  // accumulator buffers
   const int stages = p.stages, rows_pad = NRB * 128;
-  const ScoreSmem L = score_layout(D, 0, stages, 4 * 512 * sizeof(float2));
+  const bool with_v = p.gamma != nullptr;
+  const ScoreSmem L = score_layout(D, 0, stages + kVStages, 4 * 512 * sizeof(float2));
   uint8_t* sK = smem + L.k;
+  uint8_t* sV = sK + stages * KT;
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty_k = full_k + stages;
   uint64_t* tfull = empty_k + stages;  // [NB]
   uint64_t* tempty = tfull + 3;        // [NB], one arrival per epilogue warp
   uint64_t* drain = tempty + 3;
+  uint64_t* full_v = drain + 1;        // [kVStages]
+  uint64_t* empty_v = full_v + kVStages;  // [kVStages], one arrival per V warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   int* last_flag = reinterpret_cast<int*>(smem + L.misc + 8);
@@ -214,6 +226,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&tempty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
+    for (int i = 0; i < kVStages; ++i) {
+      mbar_init(&full_v[i], 1);
+      mbar_init(&empty_v[i], 2);
+    }
     *abort_flag = 0;
     *last_flag = 0;
     fence_barrier_init();
@@ -229,7 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // Guide rows -> TMEM columns [0, ACOLS): warpgroup g writes row block g,
   // warp quadrant q its 32 rows, one row per thread (rows >= M are zero).
-  if (warp >= kEpiWarp0) {
+  if (warp >= kEpiWarp0 && warp < kVWarp0) {
     const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     if (g < NRB) {
       const int row = g * 128 + quad * 32 + lane;
@@ -258,7 +274,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmk);
-      int issued = 0;
+      if (with_v) prefetch_tensormap(&tmv);
+      int issued = 0, issued_v = 0;
       for (int lt = 0; lt < nt; ++lt) {
         const int s = lt % stages, use = lt / stages;
         if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
@@ -268,13 +285,58 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kh = 0; kh < NKH; ++kh)
           tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
         issued = lt + 1;
+        if (with_v) {
+          const int vs = lt % kVStages, vuse = lt / kVStages;
+          if (vuse > 0 && !mbar_wait(&empty_v[vs], (vuse - 1) & 1, abort_flag)) break;
+          mbar_arrive_expect_tx(&full_v[vs], KT);
+#pragma unroll
+          for (int kh = 0; kh < NKH; ++kh)
+            tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+          issued_v = lt + 1;
+        }
       }
       if (*abort_flag) {  // let in-flight copies land before the CTA exits
         for (int lt = max(0, issued - stages); lt < issued; ++lt)
           mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
+        for (int lt = max(0, issued_v - kVStages); lt < issued_v; ++lt)
+          mbar_drain(&full_v[lt % kVStages], (lt / kVStages) & 1);
       }
     }
     __syncwarp();
+  } else if (warp >= kVWarp0) {
+    // Eq. 2 scales: each thread reduces 2 of the tile's 128 V rows.  The 128-byte
+    // swizzle only permutes 16-byte chunks within a row, so a row's absmax reads
+    // its own 8 chunks of each K half in any order.
+    if (with_v) {
+      const int vw = warp - kVWarp0;
+      for (int lt = 0; lt < nt; ++lt) {
+        const int vs = lt % kVStages;
+        if (!mbar_wait(&full_v[vs], (lt / kVStages) & 1, abort_flag)) break;
+        const uint8_t* tile = sV + vs * KT;
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+          const int r = vw * 64 + rr * 32 + lane;
+          uint32_t mx = 0;
+#pragma unroll
+          for (int kh = 0; kh < NKH; ++kh)
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              const uint4 u = *reinterpret_cast<const uint4*>(tile + kh * kHalfTileBytes + r * 128 + c * 16);
+              mx = __vmaxu2(mx, u.x & 0x7FFF7FFFu);
+              mx = __vmaxu2(mx, u.y & 0x7FFF7FFFu);
+              mx = __vmaxu2(mx, u.z & 0x7FFF7FFFu);
+              mx = __vmaxu2(mx, u.w & 0x7FFF7FFFu);
+            }
+          const uint32_t a16 = max(mx & 0xFFFFu, mx >> 16);
+          const int tok = (t0 + lt) * kKeyTile + r;
+          if (tok < n)
+            p.gamma[static_cast<size_t>(h) * p.n_total + doc_lo + tok] =
+                __fdiv_rn(__uint_as_float(a16 << 16), p.qmax);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty_v[vs]);
+      }
+    }
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(128, kKeyTile);
@@ -560,8 +622,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
-  (void)rows_pad;  // the guide rows live in tensor memory
-  return score_layout(head_dim, 0, stages, 4 * 512 * sizeof(float2)).total + 1024;
+  (void)rows_pad;  // the guide rows live in tensor memory; V has its own 2-stage ring
+  return score_layout(head_dim, 0, stages + kVStages, 4 * 512 * sizeof(float2)).total + 1024;
 }
 
 size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
@@ -570,26 +632,26 @@ size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
 }
 
 template <int D, int NRB>
-cudaError_t launch_lse_t(const CUtensorMap& tmk, const LseParams& p, dim3 grid, size_t smem,
-                         cudaStream_t s) {
+cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
+                         dim3 grid, size_t smem, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(lse_kernel<D, NRB>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  lse_kernel<D, NRB><<<grid, kThreads, smem, s>>>(tmk, p);
+  lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse(const CUtensorMap& tmk, const LseParams& p, int head_dim, dim3 grid,
-                       size_t smem, cudaStream_t s) {
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
+                       int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
   if (head_dim == 128) {
-    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, p, grid, smem, s);
-    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, p, grid, smem, s);
-    return launch_lse_t<128, 4>(tmk, p, grid, smem, s);
+    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, tmv, p, grid, smem, s);
+    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, tmv, p, grid, smem, s);
+    return launch_lse_t<128, 4>(tmk, tmv, p, grid, smem, s);
   }
-  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, p, grid, smem, s);
-  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, p, grid, smem, s);
-  return launch_lse_t<64, 4>(tmk, p, grid, smem, s);
+  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, tmv, p, grid, smem, s);
+  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, tmv, p, grid, smem, s);
+  return launch_lse_t<64, 4>(tmk, tmv, p, grid, smem, s);
 }
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,

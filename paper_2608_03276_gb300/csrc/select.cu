@@ -128,17 +128,25 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
     const int c1 = min(c0 + kSliceKeys, s1);
     if (!p.scores_in) {
       const float* sk = p.skey + row;
-      for (int j = threadIdx.x; j < c1 - c0 + 2 * half; j += kThreads) {
-        const int i = c0 - half + j;
-        sm.strip[j] = (i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
+      const int len = c1 - c0 + 2 * half;
+      for (int j0 = threadIdx.x; j0 < len; j0 += 8 * kThreads) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {  // eight independent loads in flight
+          const int j = j0 + u * kThreads, i = c0 - half + j;
+          v[u] = (j < len && i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (j0 + u * kThreads < len) sm.strip[j0 + u * kThreads] = v[u];
       }
       __syncthreads();
     }
-    for (int base = c0; base < c1; base += 4 * kThreads) {
-      float sv[4];
-      bool live[4];
+    for (int base = c0; base < c1; base += 8 * kThreads) {
+      float sv[8];
+      bool live[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 8; ++u) {
         const int i = base + u * kThreads + threadIdx.x;
         live[u] = i < c1;
         sv[u] = 0.f;
@@ -146,7 +154,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
                                          : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 8; ++u) {
         const int i = base + u * kThreads + threadIdx.x;
         uint32_t key = 0;
         if (live[u]) {

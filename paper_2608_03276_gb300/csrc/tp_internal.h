@@ -34,6 +34,9 @@ __host__ __device__ inline int find_doc(const DocTable& t, int cta) {
 struct LseParams {
   DocTable docs;
   const uint16_t* q;  // guide rows [batch * H_kv, rows, d] bf16
+  float* gamma;       // Eq. 2 scales [H_kv, N] written alongside, or null
+  float qmax;
+  int64_t n_total;
   int n_heads_kv;
   int rows;          // M = G * L_t
   int rows_pad;      // 128 * nrb
@@ -107,8 +110,8 @@ struct GatherParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int num_sms, cudaStream_t s);
-cudaError_t launch_lse(const CUtensorMap& tmk, const LseParams& p, int head_dim, dim3 grid,
-                       size_t smem, cudaStream_t s);
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
+                       int head_dim, dim3 grid, size_t smem, cudaStream_t s);
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             cudaStream_t s);

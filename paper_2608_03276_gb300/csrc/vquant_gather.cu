@@ -59,7 +59,7 @@ __global__ void __launch_bounds__(256) vquant_kernel(const uint4* __restrict__ v
 template <int LPR>
 __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherParams p) {
   constexpr int SPW = 32 / (2 * LPR);  // slots per warp instruction
-  constexpr int UNR = 8;
+  constexpr int UNR = 4;
   const int lane = threadIdx.x & 31;
   const int lp = lane % (2 * LPR), part = lp % LPR;
   const bool is_v = lp >= LPR;  // K lanes then V lanes
@@ -124,7 +124,7 @@ cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
   if (p.cap <= 0) return cudaSuccess;
   const int threads = 256;
   const int lpr = p.head_dim / 8;
-  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr)) * 8;
+  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr)) * 4;
   dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
             p.batch);
   if (p.head_dim == 128)

@@ -155,7 +155,13 @@ def test_stage_entry_points(cuda_lib, name):
     rows = w.group * w.guide_len
     lse = torch.empty((w.batch, w.n_heads_kv, rows), dtype=torch.float32, device="cuda")
     ws = torch.empty(binding.tp_workspace_bytes(p), dtype=torch.uint8, device="cuda")
-    binding.tp_guide_lse(p, q, k, lse, ws)
+    gam = torch.empty((w.n_heads_kv, p.n_total), dtype=torch.float32, device="cuda")
+    binding.tp_guide_lse(p, q, k, lse, ws, v=parity.to_device_bf16(x.v), gamma=gam)
+    rg, _ = O.quantize_v(x.v)
+    assert np.array_equal(gam.cpu().numpy().view(np.uint32), rg.view(np.uint32)), "fused gamma"
+    lse2 = torch.empty_like(lse)
+    binding.tp_guide_lse(p, q, k, lse2, ws)
+    assert torch.equal(lse, lse2), "lse differs with and without the fused V scales"
     got = lse.cpu().numpy()
     qf, kf = O.decode_bf16(x.q), O.decode_bf16(x.k)
     sigma = 1.0 / math.sqrt(w.head_dim)
