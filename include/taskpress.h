@@ -149,6 +149,28 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
                  float* gamma, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * tp_guide_lse without a caller workspace.  The paper has no counterpart; this
+ * entry point exists for callers that cannot allocate device memory: code
+ * that runs inside a CUDA stream capture or a host framework's launch hook
+ * where calling the allocator is not allowed, or plugins that are handed
+ * only a stream and the tensors they must read and write.  Arguments and
+ * results are those of tp_guide_lse; the scratch it needs (status word,
+ * counters, partial sums) lives in a fixed 2 MiB device array inside the
+ * library, which every GPU that loads the library keeps until exit.
+ *  - Problems whose pass-1 scratch exceeds 2 MiB are rejected with
+ *    TP_ERR_WORKSPACE (typical shapes need well under 1 MiB: about
+ *    8 bytes x number of SMs x guide rows, plus 4 bytes per document and head).
+ *  - The first call on each device looks up that array's device address
+ *    (cudaGetSymbolAddress) with the device current; make that first call
+ *    before any stream capture.
+ *  - All calls share the one array: calls that may overlap on the GPU (other
+ *    streams, other threads) race and must be serialised by the caller.
+ *  - Nothing is allocated: no cudaMalloc, cudaFree or allocating library call.
+ */
+int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const void* v,
+                        float* lse, float* gamma, void* stream);
+
+/*
  * Stage 2 of the scores (Sec. 3.2, Eq. 1's inner sums): given the row
  * normalisers `lse` ([batch, H_kv, M] fp32, natural log, e.g. from
  * tp_guide_lse or from the caller's own prefill attention), writes the

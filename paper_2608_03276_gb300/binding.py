@@ -31,7 +31,8 @@ KERNELS_PER_COMPRESS = 4
 
 #: every symbol include/taskpress.h declares
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
-           "tp_guide_scores", "tp_guide_lse", "tp_guide_key_scores", "tp_select", "tp_compact",
+           "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
+           "tp_select", "tp_compact",
            "tp_compress_layer", "tp_check_status", "tp_status_string")
 
 
@@ -82,6 +83,9 @@ def load(path: Optional[str] = None):
     lib.tp_guide_lse.restype = c_int
     lib.tp_guide_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
                                  c_void_p, c_void_p, c_size_t, c_void_p]
+    lib.tp_guide_lse_static.restype = c_int
+    lib.tp_guide_lse_static.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
+                                        c_void_p, c_void_p]
     lib.tp_guide_key_scores.restype = c_int
     lib.tp_guide_key_scores.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
                                         c_void_p]
@@ -203,6 +207,19 @@ def tp_guide_lse(p: Problem, q, k, lse, ws, stream=None, v=None, gamma=None):
         _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_guide_lse_static(p: Problem, q, k, lse, stream=None, v=None, gamma=None):
+    """tp_guide_lse with the library's fixed device scratch (no workspace argument)."""
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    rows = (hq // hkv) * lt
+    _check("tp_guide_lse_static", load().tp_guide_lse_static(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(v, torch.bfloat16, hkv * n * d, "v", nullable=True),
+        _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True), _stream(stream)))
 
 
 def tp_guide_key_scores(p: Problem, q, k, lse, key_scores, stream=None):

@@ -295,6 +295,37 @@ void fill_gather(const Plan& P, GatherParams* gp) {
 }
 
 }  // namespace
+
+// ---------------------------------------------------------------------------
+// Fixed device scratch for tp_guide_lse_static: the status word, the per-
+// (document, head) counters and the per-CTA partial sums of pass 1.  Every
+// GPU that loads the library holds it until the process exits.
+// ---------------------------------------------------------------------------
+constexpr size_t kStaticScratchBytes = size_t(2) << 20;  // 2 MiB
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+void* g_static_ptr[kMaxDevices];
+
+// Device address of g_static_scratch on the current device (host code cannot
+// use the symbol itself as an address), looked up once per device.
+int static_scratch(char** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TP_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) return TP_ERR_CUDA;
+    g_static_ptr[dev] = ptr;
+  }
+  *out = static_cast<char*>(g_static_ptr[dev]);
+  return TP_OK;
+}
+
+}  // namespace
 }  // namespace tp
 
 using namespace tp;
@@ -373,6 +404,25 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
+  if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  CUtensorMap tmk, tmq;
+  if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+  return run_lse(P, tmk, q, v, gamma, lse, w, s);
+}
+
+int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const void* v,
+                        float* lse, float* gamma, void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k || !lse || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
+  if ((v == nullptr) != (gamma == nullptr) || (v && !aligned16(v))) return TP_ERR_INVALID_ARG;
+  // pass 1 touches the workspace only up to the end of its partial sums
+  if (P.ws_lse > kStaticScratchBytes) return TP_ERR_WORKSPACE;
+  char* w = nullptr;
+  if ((st = static_scratch(&w)) != TP_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;  // counters must start at zero
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
