@@ -339,7 +339,7 @@ def run_ours(args, w):
     dom = max(("lse+vscale", "keyscore"), key=lambda s: stage_ms[s])
     dom_ms = stage_ms[dom]
     achieved = flops1 / (dom_ms / 1e3) / 1e12
-    kname = {"lse+vscale": "lse_kernel", "keyscore": "keyscore_kernel"}[dom]
+    kname = {"lse+vscale": "tp_lse_kernel", "keyscore": "tp_keyscore_kernel"}[dom]
     roofline = {"bound": "tensor", "kernel": kname, "achieved": achieved,
                 "peak": tf_sust, "unit": "TFLOP/s", "frac": achieved / tf_sust,
                 "peak_source": f"{peak_src} bf16 sustained",

@@ -5,11 +5,11 @@
 // per-row softmax normalisation needs every row's log-sum-exp before any
 // column (per-key) sum can be formed, so the scores take two passes:
 //
-//   pass 1 (lse_kernel)      D[row, key] = Q K^T in TMEM, one thread per guide
+//   pass 1 (tp_lse_kernel)      D[row, key] = Q K^T in TMEM, one thread per guide
 //                            row keeps a running (max, sum of 2^x) over the
 //                            CTA's key tiles; the last CTA of a (document,
 //                            head) merges the partials into lse[row].
-//   pass 2 (keyscore_kernel) D[key, row] = K Q^T in TMEM (keys on lanes), one
+//   pass 2 (tp_keyscore_kernel) D[key, row] = K Q^T in TMEM (keys on lanes), one
 //                            thread per key sums exp(x*sigma - lse[row]) over all
 //                            rows of the group: s_key[key] (mean over G).
 //
@@ -180,7 +180,7 @@ __device__ __forceinline__ void load_guide(uint8_t* sQ, const CUtensorMap* tmq, 
 // ---------------------------------------------------------------------------
 template <int D, int NRB>
 __global__ void __launch_bounds__(kLseThreads, 1)
-    lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+    tp_lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                const __grid_constant__ LseParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
@@ -452,7 +452,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
 // ---------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
-    keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
+    tp_keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
                     const __grid_constant__ KeyScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
@@ -634,11 +634,11 @@ size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
 template <int D, int NRB>
 cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
                          dim3 grid, size_t smem, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(lse_kernel<D, NRB>,
+  cudaError_t e = cudaFuncSetAttribute(tp_lse_kernel<D, NRB>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, p);
+  tp_lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, p);
   return cudaGetLastError();
 }
 
@@ -659,14 +659,14 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             cudaStream_t s) {
   if (head_dim == 128) {
     cudaError_t e = cudaFuncSetAttribute(
-        keyscore_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        tp_keyscore_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    keyscore_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+    tp_keyscore_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
   } else {
     cudaError_t e = cudaFuncSetAttribute(
-        keyscore_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        tp_keyscore_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    keyscore_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
+    tp_keyscore_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
   }
   return cudaGetLastError();
 }

@@ -94,7 +94,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
 }
 
 __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads, 1)
-    select_kernel(const __grid_constant__ SelectParams p) {
+    tp_select_kernel(const __grid_constant__ SelectParams p) {
   extern __shared__ uint8_t smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
@@ -284,10 +284,10 @@ cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
   if (units <= 0) return cudaSuccess;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
   const size_t smem = sizeof(SelectSmem);
-  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(tp_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  select_kernel<<<dim3(kClusterCtas, units), kThreads, smem, s>>>(p);
+  tp_select_kernel<<<dim3(kClusterCtas, units), kThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -18,7 +18,7 @@ namespace {
 // One row = LPR lanes x 8 bf16.  Rows are processed UNROLL at a time per
 // lane group so that several 16-byte loads are in flight per thread.
 template <int LPR, int UNROLL>
-__global__ void __launch_bounds__(256) vquant_kernel(const uint4* __restrict__ v,
+__global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict__ v,
                                                       uint2* __restrict__ vq,
                                                       float* __restrict__ gamma, int64_t rows,
                                                       float qmax) {
@@ -57,7 +57,7 @@ __global__ void __launch_bounds__(256) vquant_kernel(const uint4* __restrict__ v
 // V, kUnroll slot groups per warp with their loads in flight together; idx < 0
 // marks an unused slot (zero-filled).
 template <int LPR>
-__global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherParams p) {
+__global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ GatherParams p) {
   constexpr int SPW = 32 / (2 * LPR);  // slots per warp instruction
   constexpr int UNR = 4;
   const int lane = threadIdx.x & 31;
@@ -114,9 +114,9 @@ cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t r
   const uint4* vv = reinterpret_cast<const uint4*>(v);
   uint2* qq = reinterpret_cast<uint2*>(vq);
   if (head_dim == 128)
-    vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+    tp_vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
   else
-    vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+    tp_vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
   return cudaGetLastError();
 }
 
@@ -128,9 +128,9 @@ cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
             p.batch);
   if (p.head_dim == 128)
-    gather_kernel<16><<<grid, threads, 0, s>>>(p);
+    tp_gather_kernel<16><<<grid, threads, 0, s>>>(p);
   else
-    gather_kernel<8><<<grid, threads, 0, s>>>(p);
+    tp_gather_kernel<8><<<grid, threads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -340,4 +340,21 @@ def pin_ragged_docs_independent(O):
             assert np.array_equal(whole["scores"][(b, h)], single["scores"][(0, h)])
 
 
+def pin_gather_rows(O):
+    """Compaction reads row (head, doc_lo + idx) of every tensor: rows here encode
+    their own (head, token), so the gathered values name where they came from."""
+    hkv, n, d = 3, 40, 4
+    tok = np.arange(n)[None, :, None]
+    head = np.arange(hkv)[:, None, None]
+    k = (head * 1000 + tok + np.zeros((1, 1, d))).astype(np.uint16)
+    v = (head * 1000 + tok + 500 + np.zeros((1, 1, d))).astype(np.uint16)
+    gamma = (np.arange(hkv)[:, None] * 1000 + np.arange(n)[None, :]).astype(np.float32)
+    vq = ((np.arange(n)[None, :, None] % 100) + np.zeros((hkv, 1, d))).astype(np.int8)
+    idx = np.array([0, 3, 4, 9])
+    kc, vc, vqc, gc = O.gather_rows(k, v, gamma, vq, 10, 2, idx)
+    want_tok = 10 + idx
+    assert np.array_equal(kc[:, 0], 2000 + want_tok) and np.array_equal(vc[:, 0], 2500 + want_tok)
+    assert np.array_equal(gc, 2000 + want_tok) and np.array_equal(vqc[:, 0], want_tok % 100)
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -36,6 +36,7 @@ MUTATIONS = {
     "kept indices not ascending": ("return np.sort(order[:k]).astype(np.int64)", "return order[:k].astype(np.int64)"),
     "naive ceil budget": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.ceil(keep_ratio * float(n))"),
     "budget rounds down": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.floor(keep_ratio * float(n))"),
+    "gather ignores the document offset": ("tok = doc_lo + np.asarray(idx, dtype=np.int64)", "tok = np.asarray(idx, dtype=np.int64)"),
     "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma) if", "s_key = key_scores(qg, k_all[h, 0:n], sigma) if"),
 }
 
