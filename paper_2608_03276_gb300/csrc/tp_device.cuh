@@ -79,6 +79,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of the phase with parity `parity` (never suspends the
+// thread; for event loops that poll several barriers).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits for the phase of `bar` with parity `parity` to complete.  Gives up
 // after kWaitLimitNs of wall time or as soon as another thread of the CTA
 // raised `abort_flag`; returns false then (the caller unwinds).
@@ -332,13 +346,39 @@ __device__ __forceinline__ int block_sum(int v, int* warp_tot) {
 
 // ---------------------------------------------------------------------------
 // Eq. 2 codes: round-half-even of the IEEE fp32 quotient v / gamma, clamped to
-// +-qmax; gamma = 0 gives 0.  __fdiv_rn keeps the quotient correctly rounded.
+// +-qmax; gamma = 0 gives 0.
+//
+// quant_code divides exactly (__fdiv_rn).  quant_code_fast reaches the same
+// integer from one correctly rounded reciprocal per row: t = v * fl(1/gamma)
+// differs from v/gamma by at most ~2 ulp (|t - v/gamma| < 3.1e-5 for
+// |v/gamma| <= 127.5), and the correctly rounded quotient Q lies within half
+// an ulp (< 3.9e-6) of v/gamma, so |t - Q| < 3.5e-5.  rint(t) = rint(Q) unless
+// a rounding boundary k + 1/2 lies within 4e-5 of t; only then (and for
+// scales so small that 1/gamma is not finite) the exact division is taken.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int8_t quant_code(float v, float gamma, float qmax) {
   if (!(gamma > 0.f)) return 0;
   float q = rintf(__fdiv_rn(v, gamma));
   q = fminf(fmaxf(q, -qmax), qmax);
   return static_cast<int8_t>(static_cast<int>(q));
+}
+
+// inv = __fdiv_rn(1, gamma) for the row, computed once by the caller.  The
+// rounding uses the fp32 adder: t + 1.5*2^23 rounds t to an integer (ties to
+// even) for |t| < 2^22, and the sum's low bits are that integer.
+__device__ __forceinline__ int quant_code_fast(float v, float gamma, float inv, float qmax) {
+  if (!(gamma > 0.f)) return 0;
+  const float t = v * inv;
+  const float tb = t + 12582912.0f;  // 1.5 * 2^23
+  const float r = tb - 12582912.0f;  // rint(t)
+  int q;
+  if (fabsf(fabsf(t - r) - 0.5f) < 4e-5f || !(fabsf(inv) < 3.0e38f)) {
+    q = static_cast<int>(rintf(__fdiv_rn(v, gamma)));
+  } else {
+    q = __float_as_int(tb) - 0x4B400000;
+  }
+  const int qm = static_cast<int>(qmax);
+  return q < -qm ? -qm : (q > qm ? qm : q);
 }
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&f)[8]) {
@@ -351,11 +391,12 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&f)[8]) {
 }
 
 __device__ __forceinline__ uint2 quant8(const float (&f)[8], float gamma, float qmax) {
+  const float inv = gamma > 0.f ? __fdiv_rn(1.0f, gamma) : 0.f;
   uint32_t lo = 0, hi = 0;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[i], gamma, qmax))) << (8 * i);
-    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[4 + i], gamma, qmax))) << (8 * i);
+    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code_fast(f[i], gamma, inv, qmax))) << (8 * i);
+    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code_fast(f[4 + i], gamma, inv, qmax))) << (8 * i);
   }
   return make_uint2(lo, hi);
 }
