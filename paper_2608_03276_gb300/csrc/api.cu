@@ -296,6 +296,22 @@ void fill_gather(const Plan& P, GatherParams* gp) {
 
 }  // namespace
 
+cudaError_t set_smem_once(const void* kernel, int slot) {
+  constexpr int kSlots = 32, kDevs = 64;
+  static std::mutex mu;
+  static bool done[kSlots][kDevs];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (slot < 0 || slot >= kSlots || dev < 0 || dev >= kDevs)
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+  std::lock_guard<std::mutex> lock(mu);
+  if (done[slot][dev]) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+  if (e == cudaSuccess) done[slot][dev] = true;
+  return e;
+}
+
 // ---------------------------------------------------------------------------
 // Fixed device scratch for tp_guide_lse_static: the status word, the per-
 // (document, head) counters and the per-CTA partial sums of pass 1.  Every

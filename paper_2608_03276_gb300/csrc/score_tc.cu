@@ -634,9 +634,8 @@ size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
 template <int D, int NRB>
 cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
                          dim3 grid, size_t smem, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(tp_lse_kernel<D, NRB>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_lse_kernel<D, NRB>),
+                                1 + (D == 128 ? 3 : 0) + (NRB == 1 ? 0 : NRB == 2 ? 1 : 2));
   if (e != cudaSuccess) return e;
   tp_lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, p);
   return cudaGetLastError();
@@ -658,13 +657,11 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             cudaStream_t s) {
   if (head_dim == 128) {
-    cudaError_t e = cudaFuncSetAttribute(
-        tp_keyscore_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<128>), 8);
     if (e != cudaSuccess) return e;
     tp_keyscore_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
   } else {
-    cudaError_t e = cudaFuncSetAttribute(
-        tp_keyscore_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<64>), 9);
     if (e != cudaSuccess) return e;
     tp_keyscore_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
   }

@@ -37,15 +37,6 @@ __device__ __forceinline__ uint32_t score_key(float s) {
   return (s > 0.f) ? __float_as_uint(s) : 0u;  // -0, +0, NaN and negatives -> 0
 }
 
-// Adds one to hist[bin] for every active lane, one shared atomic per distinct
-// bin in the warp (keys concentrate in few bins).  All 32 lanes must call it.
-__device__ __forceinline__ void hist_add(int* hist, uint32_t bin, bool active) {
-  const unsigned mask = __ballot_sync(0xffffffffu, active);
-  if (!active) return;
-  const unsigned peers = __match_any_sync(mask, bin);
-  if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
-}
-
 constexpr int kSliceKeys = 16384;  // keys of a CTA's slice kept in shared memory
 constexpr int kMaxHalf = 16;       // largest pooling half-window of the staging strip
 
@@ -55,41 +46,86 @@ struct SelectSmem {
   int hist1[kBins1];
   int hist2[kBins2];
   int hist3[kBins3];
+  int red[kBins1 / kClusterCtas];  // this CTA's slice of the cluster-summed histogram
+  int red_total;
   int counts[2];  // (> T, == T) in this CTA's slice
   int scratch[33];
   int result[2];
 };
 
+// Address of `local` (a shared-memory object of this CTA) in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t dsmem(const void* local, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ int ld_dsmem(uint32_t addr) {
+  int v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+  return v;
+}
+
 // Bin holding the `need`-th largest key (1-based) of the cluster-wide
-// histogram (the sum of every CTA's shared histogram at byte offset `off`);
-// *above = keys in higher bins.  Called by the whole block.
+// histogram, i.e. the sum over the cluster of every CTA's `local_hist`;
+// *above = keys in higher bins.  Called by every thread of every CTA of the
+// cluster (it contains cluster barriers).
+//   1. CTA r sums its slice of nbins/8 bins over the 8 CTAs (remote loads).
+//   2. Every CTA reads the 8 slice totals, finds the slice holding the target
+//      (highest bins first), and scans that slice's bins from its owner.
 __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const int* local_hist,
                              int nbins, int need, int* above) {
-  const int per = nbins / kThreads;  // 2 or 4 bins per thread, highest bins first
-  int cnt[4] = {0, 0, 0, 0};
-  for (int r = 0; r < kClusterCtas; ++r) {
-    const int* h = cluster.map_shared_rank(local_hist, r);
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int slice = nbins / kClusterCtas;  // 256 or 128 bins
+  if (threadIdx.x < slice) {
+    const int bin = rank * slice + threadIdx.x;
+    int v[kClusterCtas];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (i < per) cnt[i] += h[nbins - 1 - (threadIdx.x * per + i)];
+    for (int r = 0; r < kClusterCtas; ++r) v[r] = ld_dsmem(dsmem(local_hist + bin, r));
+    int t = 0;
+#pragma unroll
+    for (int r = 0; r < kClusterCtas; ++r) t += v[r];
+    sm.red[threadIdx.x] = t;
   }
-  int local = 0;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    int t = 0;
+    for (int i = threadIdx.x; i < slice; i += 32) t += sm.red[i];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) local += cnt[i];
-  int total;
-  int before = block_excl_scan(local, sm.scratch, &total);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    if (i < per && before < need && before + cnt[i] >= need) {
-      sm.result[0] = nbins - 1 - (threadIdx.x * per + i);
-      sm.result[1] = before;
+    for (int o = 16; o >= 1; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (threadIdx.x == 0) sm.red_total = t;
+  }
+  cluster.sync();  // every slice reduced
+  // slice totals, highest slice first, and the slice that holds the target
+  if (threadIdx.x == 0) {
+    int before = 0, s_hit = 0, s_before = 0;
+    for (int r = kClusterCtas - 1; r >= 0; --r) {
+      const int t = ld_dsmem(dsmem(&sm.red_total, r));
+      if (before < need && before + t >= need) {
+        s_hit = r;
+        s_before = before;
+      }
+      before += t;
     }
-    before += cnt[i];
+    sm.result[0] = s_hit;
+    sm.result[1] = s_before;
+  }
+  __syncthreads();
+  const int s_hit = sm.result[0], s_before = sm.result[1];
+  __syncthreads();
+  // scan the hit slice's bins, highest first (one bin per thread)
+  int cnt = 0;
+  if (threadIdx.x < slice) cnt = ld_dsmem(dsmem(&sm.red[slice - 1 - threadIdx.x], s_hit));
+  int total;
+  const int before = s_before + block_excl_scan(cnt, sm.scratch, &total);
+  if (threadIdx.x < slice && before < need && before + cnt >= need) {
+    sm.result[0] = s_hit * slice + (slice - 1 - threadIdx.x);
+    sm.result[1] = before;
   }
   __syncthreads();
   *above = sm.result[1];
   const int d = sm.result[0];
-  __syncthreads();
+  cluster.sync();  // no CTA overwrites red / red_total while others still read them
   return d;
 }
 
@@ -126,6 +162,19 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
   const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
   for (int c0 = s0; c0 < s1; c0 += kSliceKeys) {
     const int c1 = min(c0 + kSliceKeys, s1);
+    // this thread's first round of scale (or score) loads go out before the
+    // key-score strip is staged, so the two global round trips overlap
+    float sv[8];
+    auto load_round = [&](int base) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = base + u * kThreads + threadIdx.x;
+        sv[u] = 0.f;
+        if (i < c1) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
+                                        : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
+      }
+    };
+    load_round(c0);
     if (!p.scores_in) {
       const float* sk = p.skey + row;
       const int len = c1 - c0 + 2 * half;
@@ -143,33 +192,25 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
       __syncthreads();
     }
     for (int base = c0; base < c1; base += 8 * kThreads) {
-      float sv[8];
-      bool live[8];
+      if (base != c0) load_round(base);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const int i = base + u * kThreads + threadIdx.x;
-        live[u] = i < c1;
-        sv[u] = 0.f;
-        if (live[u]) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
-                                         : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int i = base + u * kThreads + threadIdx.x;
+        const bool live = i < c1;
         uint32_t key = 0;
-        if (live[u]) {
-          float s = sv[u];
+        if (live) {
+          float sc = sv[u];
           if (!p.scores_in) {
             float acc = 0.f;
             const float* w = sm.strip + (i - c0);
             for (int o = 0; o <= 2 * half; ++o) acc += w[o];
-            s = p.key_only ? acc * inv_k : (acc * inv_k) * sv[u];
-            if (p.scores_out) p.scores_out[row + i] = s;
+            sc = p.key_only ? acc * inv_k : (acc * inv_k) * sv[u];
+            if (p.scores_out) p.scores_out[row + i] = sc;
           }
-          key = score_key(s);
+          key = score_key(sc);
           keys_base[i - kofs] = key;
         }
-        if (!p.scores_only) hist_add(sm.hist1, key >> 21, live[u]);
+        if (!p.scores_only && live) atomicAdd(&sm.hist1[key >> 21], 1);
       }
     }
     __syncthreads();
@@ -191,7 +232,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
     for (int base = s0; base < s1; base += kThreads) {
       const int i = base + threadIdx.x;
       const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
-      hist_add(sm.hist2, (key >> 10) & 0x7FF, i < s1 && (key >> 21) == static_cast<uint32_t>(d1));
+      if (i < s1 && (key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
     }
     cluster.sync();
     const int d2 = cluster_digit(cluster, sm, sm.hist2, kBins2, need, &above);
@@ -200,16 +241,17 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
     for (int base = s0; base < s1; base += kThreads) {
       const int i = base + threadIdx.x;
       const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
-      hist_add(sm.hist3, key & 0x3FF, i < s1 && (key >> 10) == pre);
+      if (i < s1 && (key >> 10) == pre) atomicAdd(&sm.hist3[key & 0x3FF], 1);
     }
     cluster.sync();
     const int d3 = cluster_digit(cluster, sm, sm.hist3, kBins3, need, &above);
     need_eq = need - above;
     thr = (pre << 10) | static_cast<uint32_t>(d3);
   } else {
-    // the cluster-wide barriers must match on every CTA
-    cluster.sync();
-    cluster.sync();
+    // the cluster-wide barriers must match on every CTA: two per digit search
+    // (three searches) and one after each of the two later histograms
+#pragma unroll 1
+    for (int i = 0; i < 8; ++i) cluster.sync();
   }
 
   // D: counts of this slice, then prefix over the slices before it
@@ -254,9 +296,12 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
         else if (kv[e] == thr) ++neq;
       }
     }
-    int tot_gt, tot_eq;
-    int gt_rank = gt_before + block_excl_scan(ngt, sm.scratch, &tot_gt);
-    int eq_rank = eq_before + block_excl_scan(neq, sm.scratch, &tot_eq);
+    // one scan of packed counts: (> T) in the high 16 bits, (== T) in the low
+    int tot;
+    const int pre = block_excl_scan((ngt << 16) | neq, sm.scratch, &tot);
+    const int tot_gt = tot >> 16, tot_eq = tot & 0xFFFF;
+    int gt_rank = gt_before + (pre >> 16);
+    int eq_rank = eq_before + (pre & 0xFFFF);
 #pragma unroll
     for (int e = 0; e < kPer; ++e) {
       const int j = j0 + e;
@@ -284,8 +329,7 @@ cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
   if (units <= 0) return cudaSuccess;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
   const size_t smem = sizeof(SelectSmem);
-  cudaError_t e = cudaFuncSetAttribute(tp_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel), 0);
   if (e != cudaSuccess) return e;
   tp_select_kernel<<<dim3(kClusterCtas, units), kThreads, smem, s>>>(p);
   return cudaGetLastError();

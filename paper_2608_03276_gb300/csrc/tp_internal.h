@@ -67,7 +67,7 @@ struct KeyScoreParams {
   int* status;
 };
 
-constexpr int kChunk = 4096;       // tokens per compaction round in the selection kernel
+constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
 constexpr int kClusterCtas = 8;    // CTAs (one cluster) per (document, head) in the selection
 
 struct SelectParams {
@@ -117,6 +117,10 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t s);
+
+// Raises a kernel's dynamic shared-memory limit to the device maximum, once per
+// (kernel slot, device); `slot` names the kernel in a small registry.
+cudaError_t set_smem_once(const void* kernel, int slot);
 
 // Shared-memory layout sizes of the scoring kernels (host side).
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages);
