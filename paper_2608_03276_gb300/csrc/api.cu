@@ -111,6 +111,9 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->stages2 = 4;
   while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
   P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
+  // pass 1 stages the guide block through its K ring
+  if (size_t(P->stages1) * (P->d / 64) * 16384 < size_t(P->d / 64) * P->rows_pad * 128)
+    return TP_ERR_UNSUPPORTED_SHAPE;
   P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
   if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
 
@@ -203,8 +206,8 @@ DocTable doc_table(const Plan& P) {
 // Pass 1: row normalisers into `lse` ([batch, H_kv, rows]), and the Eq. 2
 // scales of every token into `gamma` when v/gamma are given.  The counters and
 // the status word at the head of the workspace must be zero.
-int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, const void* v, float* gamma,
-            float* lse, char* ws, cudaStream_t s) {
+int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const void* q,
+            const void* v, float* gamma, float* lse, char* ws, cudaStream_t s) {
   CUtensorMap tmv = tmk;
   if (gamma && !encode_3d(&tmv, v, P.d, P.n_total, P.hkv, 128)) return TP_ERR_CUDA;
   int* status = reinterpret_cast<int*>(ws + P.ws_status);
@@ -226,7 +229,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const void* q, const void* v,
   lp.lse = lse;
   lp.counters = status + 1;
   lp.status = status;
-  return cuda_status(launch_lse(tmk, tmv, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
+  return cuda_status(launch_lse(tmk, tmv, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
 }
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
@@ -258,7 +261,7 @@ int run_scoring(const Plan& P, const void* q, const void* k, const void* v, floa
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
-  int st = run_lse(P, tmk, q, v, gamma, lse, ws, s);
+  int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s);
   if (st != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), s);
@@ -423,7 +426,7 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_lse(P, tmk, q, v, gamma, lse, w, s);
+  return run_lse(P, tmk, tmq, q, v, gamma, lse, w, s);
 }
 
 int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const void* v,
@@ -442,7 +445,7 @@ int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_lse(P, tmk, q, v, gamma, lse, w, s);
+  return run_lse(P, tmk, tmq, q, v, gamma, lse, w, s);
 }
 
 int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,

@@ -181,7 +181,7 @@ __device__ __forceinline__ void load_guide(uint8_t* sQ, const CUtensorMap* tmq, 
 template <int D, int NRB>
 __global__ void __launch_bounds__(kLseThreads, 1)
     tp_lse_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
-               const __grid_constant__ LseParams p) {
+               const __grid_constant__ CUtensorMap tmq, const __grid_constant__ LseParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
   constexpr int NKH = D / 64;
@@ -200,6 +200,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   uint64_t* drain = tempty + 3;
   uint64_t* full_v = drain + 1;        // [kVStages]
   uint64_t* empty_v = full_v + kVStages;  // [kVStages], one arrival per V warp
+  uint64_t* q_full = empty_v + kVStages;   // the guide block has landed in the K ring
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   int* last_flag = reinterpret_cast<int*>(smem + L.misc + 8);
@@ -230,6 +231,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
       mbar_init(&full_v[i], 1);
       mbar_init(&empty_v[i], 2);
     }
+    mbar_init(q_full, 1);
     *abort_flag = 0;
     *last_flag = 0;
     fence_barrier_init();
@@ -243,21 +245,31 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // Guide rows -> TMEM columns [0, ACOLS): warpgroup g writes row block g,
-  // warp quadrant q its 32 rows, one row per thread (rows >= M are zero).
+  // Guide rows -> TMEM columns [0, ACOLS).  The block arrives by TMA in the
+  // (still idle) K ring, 128-byte swizzled; warpgroup g then writes row block
+  // g, warp quadrant q its 32 rows, one row per thread (rows >= M arrive as
+  // zeros).  The swizzle puts 16-byte chunk c of row r at chunk c ^ (r & 7),
+  // so a warp's 32 rows read conflict-free.
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmq);
+    const int qbox = rows_pad < 256 ? rows_pad : 256;
+    mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(NKH * rows_pad * 128));
+#pragma unroll
+    for (int kh = 0; kh < NKH; ++kh)
+      for (int r0 = 0; r0 < rows_pad; r0 += qbox)
+        tma_load_3d(sK + (kh * rows_pad + r0) * 128, &tmq, kh * 64, r0, b * p.n_heads_kv + h, q_full);
+  }
   if (warp >= kEpiWarp0 && warp < kVWarp0) {
     const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
-    if (g < NRB) {
+    if (g < NRB && mbar_wait(q_full, 0, abort_flag)) {
       const int row = g * 128 + quad * 32 + lane;
-      const uint4* src = reinterpret_cast<const uint4*>(
-          p.q + ((static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows + row) * D);
-      const bool live = row < p.rows;
 #pragma unroll
       for (int part = 0; part < D / 64; ++part) {
+        const uint8_t* src = sK + (part * rows_pad + row) * 128;
         uint32_t r[32];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          const uint4 v = live ? __ldg(src + part * 8 + i) : make_uint4(0, 0, 0, 0);
+          const uint4 v = *reinterpret_cast<const uint4*>(src + ((i ^ (row & 7)) << 4));
           r[4 * i] = v.x;
           r[4 * i + 1] = v.y;
           r[4 * i + 2] = v.z;
@@ -266,7 +278,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         tmem_st32(tmem + (static_cast<uint32_t>(quad * 32) << 16) + g * (D / 2) + part * 32, r);
       }
     }
+    fence_proxy_async_smem();  // the K stream overwrites the block next
   }
+  if (warp == 0 && lane == 0 && *abort_flag) mbar_drain(q_full, 0);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -423,10 +437,16 @@ __global__ void __launch_bounds__(kLseThreads, 1)
       const float2* part =
           p.partials + (static_cast<size_t>(h) * gridDim.x + p.docs.cta[b]) * rows_pad;
       for (int r = threadIdx.x; r < p.rows; r += blockDim.x) {
+        // merged in CTA order, eight partials in flight at a time
         float2 acc = make_float2(-INFINITY, 0.f);
-        for (int cc = 0; cc < ncta_doc; ++cc) {
-          const float2 v = __ldcg(part + static_cast<size_t>(cc) * rows_pad + r);
-          acc = lse_merge(acc, v);
+        for (int c0 = 0; c0 < ncta_doc; c0 += 8) {
+          float2 v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (c0 + u < ncta_doc) v[u] = __ldcg(part + static_cast<size_t>(c0 + u) * rows_pad + r);
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (c0 + u < ncta_doc) acc = lse_merge(acc, v[u]);
         }
         p.lse[(static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows + r] =
             (acc.x + lg2(acc.y)) * 0.69314718055994531f;
@@ -632,25 +652,25 @@ size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
 }
 
 template <int D, int NRB>
-cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
-                         dim3 grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                         const LseParams& p, dim3 grid, size_t smem, cudaStream_t s) {
   cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_lse_kernel<D, NRB>),
                                 1 + (D == 128 ? 3 : 0) + (NRB == 1 ? 0 : NRB == 2 ? 1 : 2));
   if (e != cudaSuccess) return e;
-  tp_lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, p);
+  tp_lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, tmq, p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
-                       int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                       const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
   if (head_dim == 128) {
-    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, tmv, p, grid, smem, s);
-    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, tmv, p, grid, smem, s);
-    return launch_lse_t<128, 4>(tmk, tmv, p, grid, smem, s);
+    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, tmv, tmq, p, grid, smem, s);
+    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, tmv, tmq, p, grid, smem, s);
+    return launch_lse_t<128, 4>(tmk, tmv, tmq, p, grid, smem, s);
   }
-  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, tmv, p, grid, smem, s);
-  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, tmv, p, grid, smem, s);
-  return launch_lse_t<64, 4>(tmk, tmv, p, grid, smem, s);
+  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, tmv, tmq, p, grid, smem, s);
+  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, tmv, tmq, p, grid, smem, s);
+  return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, s);
 }
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,

@@ -110,8 +110,8 @@ struct GatherParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int num_sms, cudaStream_t s);
-cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const LseParams& p,
-                       int head_dim, dim3 grid, size_t smem, cudaStream_t s);
+cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                       const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s);
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             cudaStream_t s);
