@@ -106,13 +106,15 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->grid_x = P->cta[P->batch];
 
   // Deepest K-tile ring that fits next to the resident guide block.
-  P->stages1 = 6;  // K ring of pass 1 (next to its 2-stage V ring)
+  P->stages1 = 6;  // K ring of pass 1 (next to its V ring)
   while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
   P->stages2 = 4;
   while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
   P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
-  // pass 1 stages the guide block through its K ring
-  if (size_t(P->stages1) * (P->d / 64) * 16384 < size_t(P->d / 64) * P->rows_pad * 128)
+  // pass 1 stages the guide block, and at the end its row statistics, through
+  // its K ring
+  if (size_t(P->stages1) * (P->d / 64) * 16384 <
+      std::max(size_t(P->d / 64) * P->rows_pad * 128, size_t(4) * P->rows_pad * sizeof(float2)))
     return TP_ERR_UNSUPPORTED_SHAPE;
   P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
   if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;

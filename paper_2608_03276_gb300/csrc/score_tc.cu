@@ -29,7 +29,7 @@ namespace {
 constexpr int kThreads = 576;      // pass 2: TMA, MMA, 16 epilogue warps
 constexpr int kLseThreads = 640;   // pass 1: the same plus 2 V-scale warps
 constexpr int kVWarp0 = 18;        // first V-scale warp of pass 1
-constexpr int kVStages = 2;        // V-tile ring depth of pass 1
+constexpr int kVStages = 3;        // V-tile ring depth of pass 1
 constexpr int kEpiWarp0 = 2;  // first epilogue warp
 constexpr int kEpiWarps = 16;  // four warpgroups
 constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
@@ -50,6 +50,13 @@ __host__ __device__ inline ScoreSmem score_layout(int head_dim, int rows_pad, in
   L.extra = (L.misc + 16 + 15) & ~15u;
   L.total = L.extra + extra_bytes;
   return L;
+}
+
+// Pass 2 extras after its barriers: up to 1 KB of alignment, the row-offset
+// operands of the extra K step (key side 128 x 32 B, guide side rows x 32 B),
+// the warpgroup partials [2][4][128].
+__host__ __device__ inline uint32_t keyscore_extra_bytes(int rows_pad) {
+  return 1024u + 128u * 32u + static_cast<uint32_t>(rows_pad) * 32u + 2u * 4u * 128u * 4u;
 }
 
 __device__ __forceinline__ uint8_t* aligned_smem(uint8_t* raw) {
@@ -130,22 +137,17 @@ __device__ __forceinline__ void lse_chunk(const uint32_t (&r)[32], int col0, int
   }
 }
 
-// One 32-column chunk of a key's logits in pass 2: sum_r 2^(x_r*c2 - l_r),
-// with the negated row normalisers -l_r read from shared memory.
-__device__ __forceinline__ float key_chunk(const uint32_t (&r)[32], const float* nl, float c2) {
+// One 32-column chunk of a key's logits in pass 2: sum_r 2^(D_r * c2), where
+// the accumulator D already holds logit_r - lse_r / sigma (the row offset
+// enters the contraction as an extra K step).
+__device__ __forceinline__ float key_chunk(const uint32_t (&r)[32], float c2) {
   float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                  make_float2(0.f, 0.f)};
   const float2 cc = make_float2(c2, c2);
-  const float4* nl4 = reinterpret_cast<const float4*>(nl);
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float4 l = nl4[i];
-    const float2 y0 = ffma2(make_float2(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1])),
-                            cc, make_float2(l.x, l.y));
-    const float2 y1 = ffma2(make_float2(__uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3])),
-                            cc, make_float2(l.z, l.w));
-    a[(2 * i) & 3] = fadd2(a[(2 * i) & 3], make_float2(ex2(y0.x), ex2(y0.y)));
-    a[(2 * i + 1) & 3] = fadd2(a[(2 * i + 1) & 3], make_float2(ex2(y1.x), ex2(y1.y)));
+  for (int i = 0; i < 16; ++i) {
+    const float2 y = fmul2(make_float2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1])), cc);
+    a[i & 3] = fadd2(a[i & 3], make_float2(ex2(y.x), ex2(y.y)));
   }
   const float2 t = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
   return t.x + t.y;
@@ -190,7 +192,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   constexpr int NB = (512 - ACOLS) / 128 < 3 ? (512 - ACOLS) / 128 : 3;  // accumulator buffers
   const int stages = p.stages, rows_pad = NRB * 128;
   const bool with_v = p.gamma != nullptr;
-  const ScoreSmem L = score_layout(D, 0, stages + kVStages, 4 * 512 * sizeof(float2));
+  const ScoreSmem L = score_layout(D, 0, stages + kVStages, 0);
   uint8_t* sK = smem + L.k;
   uint8_t* sV = sK + stages * KT;
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
@@ -204,7 +206,8 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   int* last_flag = reinterpret_cast<int*>(smem + L.misc + 8);
-  float2* stats = reinterpret_cast<float2*>(smem + L.extra);  // [4 warpgroups][rows_pad]
+  // [4 warpgroups][rows_pad] row statistics, written once the K ring is idle
+  float2* stats = reinterpret_cast<float2*>(sK);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -250,8 +253,20 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   // g, warp quadrant q its 32 rows, one row per thread (rows >= M arrive as
   // zeros).  The swizzle puts 16-byte chunk c of row r at chunk c ^ (r & 7),
   // so a warp's 32 rows read conflict-free.
+  // The V ring is idle meanwhile: its first tiles are requested right away.
+  const int v_pre = with_v ? min(kVStages, nt) : 0;
+  auto issue_v = [&](int lt) {
+    const int vs = lt % kVStages;
+    mbar_arrive_expect_tx(&full_v[vs], KT);
+    const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
+#pragma unroll
+    for (int kh = 0; kh < NKH; ++kh)
+      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+  };
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmq);
+    if (with_v) prefetch_tensormap(&tmv);
+    for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
     const int qbox = rows_pad < 256 ? rows_pad : 256;
     mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(NKH * rows_pad * 128));
 #pragma unroll
@@ -285,11 +300,17 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   __syncthreads();
   tc_fence_after();
 
+  float m[NRB], z[NRB];  // epilogue: running (offset, sum) per row block
+#pragma unroll
+  for (int rb = 0; rb < NRB; ++rb) {
+    m[rb] = -INFINITY;
+    z[rb] = 0.f;
+  }
+
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmk);
-      if (with_v) prefetch_tensormap(&tmv);
-      int issued = 0, issued_v = 0;
+      int issued = 0, issued_v = v_pre;
       for (int lt = 0; lt < nt; ++lt) {
         const int s = lt % stages, use = lt / stages;
         if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
@@ -299,13 +320,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         for (int kh = 0; kh < NKH; ++kh)
           tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
         issued = lt + 1;
-        if (with_v) {
-          const int vs = lt % kVStages, vuse = lt / kVStages;
-          if (vuse > 0 && !mbar_wait(&empty_v[vs], (vuse - 1) & 1, abort_flag)) break;
-          mbar_arrive_expect_tx(&full_v[vs], KT);
-#pragma unroll
-          for (int kh = 0; kh < NKH; ++kh)
-            tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+        if (lt >= v_pre && with_v) {
+          if (!mbar_wait(&empty_v[lt % kVStages], (lt / kVStages - 1) & 1, abort_flag)) break;
+          issue_v(lt);
           issued_v = lt + 1;
         }
       }
@@ -385,12 +402,6 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   } else {
     const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
     const float c2 = p.c2;
-    float m[NRB], z[NRB];
-#pragma unroll
-    for (int rb = 0; rb < NRB; ++rb) {
-      m[rb] = -INFINITY;
-      z[rb] = 0.f;
-    }
     const uint32_t tcol = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ACOLS + g * 32;
     bool ok = true;
     for (int lt = 0; ok && lt < nt; ++lt) {
@@ -410,15 +421,21 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         lse_chunk(r, g * 32, valid, c2, m[rb], z[rb]);
       }
     }
-#pragma unroll
-    for (int rb = 0; rb < NRB; ++rb) stats[g * rows_pad + rb * 128 + quad * 32 + lane] = make_float2(m[rb], z[rb]);
   }
+  // Every stream has landed and every MMA has finished: the K ring is free.
   __syncthreads();
 
   const bool aborted = *abort_flag != 0;
   if (aborted) {
     if (threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
   } else {
+    if (warp >= kEpiWarp0 && warp < kVWarp0) {
+      const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
+#pragma unroll
+      for (int rb = 0; rb < NRB; ++rb)
+        stats[g * rows_pad + rb * 128 + quad * 32 + lane] = make_float2(m[rb], z[rb]);
+    }
+    __syncthreads();
     for (int r = threadIdx.x; r < rows_pad; r += blockDim.x) {
       float2 acc = make_float2(-INFINITY, 0.f);
 #pragma unroll
@@ -480,7 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr uint32_t KT = NKH * kHalfTileBytes;
   const int stages = p.stages, rows_pad = p.rows_pad, rows_mma = p.rows_mma;
   const int nh = (rows_mma + 255) / 256;
-  const ScoreSmem L = score_layout(D, rows_pad, stages, rows_pad * sizeof(float) + 2 * 4 * 128 * sizeof(float));
+  const ScoreSmem L = score_layout(D, rows_pad, stages, keyscore_extra_bytes(rows_pad));
   uint8_t* sQ = smem + L.q;
   uint8_t* sK = smem + L.k;
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
@@ -491,8 +508,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
-  float* l2s = reinterpret_cast<float*>(smem + L.extra);              // -lse*log2(e) per row
-  float* part = reinterpret_cast<float*>(smem + L.extra + rows_pad * sizeof(float));  // [2][4][128]
+  // Row offsets as an extra K step of the contraction (32-byte swizzled,
+  // K-major): key side [1, 1, 1, 0, ...], guide side (hi, mid, lo, 0, ...) with
+  // hi + mid + lo = -lse[row] / sigma (three bf16 parts, exact to ~2^-24).
+  uint8_t* a_aug = smem + ((L.extra + 1023u) & ~1023u);               // [128 keys][32 B]
+  uint8_t* b_aug = a_aug + 128 * 32;                                  // [rows_pad][32 B]
+  float* part = reinterpret_cast<float*>(b_aug + rows_pad * 32);      // [2][4][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -520,8 +541,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
-    for (int r = threadIdx.x; r < rows_pad; r += blockDim.x)
-      l2s[r] = r < p.rows ? -(lse[r] * 1.4426950408889634f) : -INFINITY;
+    for (int r = threadIdx.x; r < 128 + rows_pad; r += blockDim.x) {
+      uint4 c0;
+      uint8_t* row;
+      if (r < 128) {  // key side: three ones
+        row = a_aug + r * 32;
+        c0 = make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u);
+      } else {        // guide side: the row's offset in three parts
+        const int g = r - 128;
+        row = b_aug + g * 32;
+        const float v = g < p.rows ? -(lse[g] * 1.4426950408889634f) / p.c2 : -1.0e30f;
+        const uint32_t hi = bf16_bits_rn(v);
+        const float r1 = v - __uint_as_float(hi << 16);
+        const uint32_t mid = bf16_bits_rn(r1);
+        const uint32_t lo = bf16_bits_rn(r1 - __uint_as_float(mid << 16));
+        c0 = make_uint4(hi | (mid << 16), lo, 0u, 0u);
+      }
+      const int rr = r < 128 ? r : r - 128;
+      const int pos = (rr >> 2) & 1;  // 32-byte swizzle: chunk c at c ^ ((row >> 2) & 1)
+      *reinterpret_cast<uint4*>(row + pos * 16) = c0;
+      *reinterpret_cast<uint4*>(row + (pos ^ 1) * 16) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async_smem();  // read by the tensor core
   }
   if (warp == 0) {
     tmem_alloc(tmem_slot, 512);
@@ -580,6 +621,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 sdesc_k128(smem_u32(sQ + (kh * rows_pad + hh * 256) * 128 + k16 * 32));
             mma_bf16_ss(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
           }
+          mma_bf16_ss(dt, sdesc_k32(smem_u32(a_aug)), sdesc_k32(smem_u32(b_aug + hh * 256 * 32)),
+                      idesc, 1u);
           mma_commit(&tfull[buf]);
         }
         mma_commit(&empty_k[s]);
@@ -602,7 +645,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const int nch = min(256, rows_mma - 256 * hh) / 32;
         const uint32_t tb = tlane + buf * 256;
-        const float* nl = l2s + hh * 256;
         const int c0 = g, c1 = g + 4;
         uint32_t ra[32], rb[32];
         if (c0 < nch) tmem_ld32_async(tb + c0 * 32, ra);
@@ -612,8 +654,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
-        if (c0 < nch) acc += key_chunk(ra, nl + c0 * 32, c2);
-        if (c1 < nch) acc += key_chunk(rb, nl + c1 * 32, c2);
+        if (c0 < nch) acc += key_chunk(ra, c2);
+        if (c1 < nch) acc += key_chunk(rb, c2);
       }
       // fixed-order sum of the four warpgroups' partials for this tile's keys
       float* slot = part + (lt & 1) * 4 * 128;
@@ -642,13 +684,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
-  (void)rows_pad;  // the guide rows live in tensor memory; V has its own 2-stage ring
-  return score_layout(head_dim, 0, stages + kVStages, 4 * 512 * sizeof(float2)).total + 1024;
+  (void)rows_pad;  // the guide rows live in tensor memory; V has its own ring
+  return score_layout(head_dim, 0, stages + kVStages, 0).total + 1024;
 }
 
 size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
-  return score_layout(head_dim, rows_pad, stages,
-                      rows_pad * sizeof(float) + 2 * 4 * 128 * sizeof(float)).total + 1024;
+  return score_layout(head_dim, rows_pad, stages, keyscore_extra_bytes(rows_pad)).total + 1024;
 }
 
 template <int D, int NRB>

@@ -257,6 +257,25 @@ __device__ __forceinline__ uint64_t sdesc_k128(uint32_t addr) {
   return d;
 }
 
+// Descriptor of a K-major bf16 operand with 32-byte rows (one K=16 step) in the
+// 32-byte swizzle: 8-row atoms of 256 bytes; within an atom, 16-byte chunk c of
+// row r sits at chunk position c ^ ((r >> 2) & 1).
+__device__ __forceinline__ uint64_t sdesc_k32(uint32_t addr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((addr & 0x3FFFFu) >> 4);  // start address
+  d |= static_cast<uint64_t>(1) << 16;                 // leading byte offset (unused here)
+  d |= static_cast<uint64_t>(256 >> 4) << 32;          // stride byte offset: 8 rows x 32 B
+  d |= static_cast<uint64_t>(1) << 46;                 // descriptor version
+  d |= static_cast<uint64_t>(6) << 61;                 // 32-byte swizzle
+  return d;
+}
+
+// bf16 bits of x rounded to nearest, ties to even (finite x).
+__device__ __forceinline__ uint32_t bf16_bits_rn(float x) {
+  const uint32_t u = __float_as_uint(x);
+  return (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
+}
+
 // Issues a load of 32 consecutive TMEM columns of this warp's 32 lanes (one
 // lane per thread) without waiting; the registers become valid at the next
 // tmem_wait() that names them.
@@ -333,6 +352,16 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
       "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
       "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
       : "=f"(d.x), "=f"(d.y)
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return d;
