@@ -27,6 +27,7 @@ this path) on the same workload and metric.
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import math
@@ -80,7 +81,9 @@ def measured_peaks():
 # Clock sampling during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi clock and throttle-reason samples every 20 ms, time-stamped;
+    summary() keeps the samples that fall inside the marked timed window."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -88,6 +91,7 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.path = None
+        self.t_start = self.t_end = None
 
     def __enter__(self):
         fd, self.path = tempfile.mkstemp(suffix=".csv")
@@ -95,14 +99,21 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
         time.sleep(0.3)
         return self
 
+    def mark_start(self):
+        self.t_start = datetime.datetime.now()
+
+    def mark_end(self):
+        self.t_end = datetime.datetime.now()
+
     def __exit__(self, *a):
+        time.sleep(0.05)
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -113,25 +124,37 @@ class ClockSampler:
     def summary(self):
         if self.proc is None or not self.path:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        sm, smax, reasons = [], [], set()
+        rows = []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         with open(self.path) as f:
             for line in f:
                 parts = [x.strip() for x in line.split(",")]
-                if len(parts) < 9:
+                if len(parts) < 10:
                     continue
                 try:
-                    sm.append(float(parts[1]))
-                    smax.append(float(parts[2]))
+                    ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f")
+                    rows.append((ts, float(parts[2]), float(parts[3]),
+                                 {nm for nm, val in zip(names, parts[6:10]) if val.lower().startswith("active")}))
                 except ValueError:
                     continue
-                for nm, val in zip(names, parts[5:9]):
-                    if val.lower().startswith("active"):
-                        reasons.add(nm)
         os.unlink(self.path)
-        if not sm:
+        if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "samples": len(sm),
+        margin = datetime.timedelta(milliseconds=25)
+        inside = rows
+        if self.t_start is not None and self.t_end is not None:
+            inside = [r for r in rows if self.t_start - margin <= r[0] <= self.t_end + margin]
+        window = len(inside)
+        if not inside:  # timed region shorter than the sampling period: nearest sample after its start
+            later = [r for r in rows if self.t_start is None or r[0] >= self.t_start]
+            inside = later[:1] or rows[-1:]
+        reasons = set()
+        for r in inside:
+            reasons |= r[3]
+        return {"sm_mhz": statistics.median(r[1] for r in inside), "sm_max_mhz": max(r[2] for r in inside),
+                "samples": len(inside), "samples_in_window": window,
+                "window_ms": round((self.t_end - self.t_start).total_seconds() * 1e3, 1)
+                if self.t_start and self.t_end else None,
                 "reasons": sorted(reasons)}
 
 
@@ -288,11 +311,13 @@ def run_ours(args, w):
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clocks:
+        clocks.mark_start()
         ev0.record(stream)
         for _ in range(args.steps):
             step()
         ev1.record(stream)
         torch.cuda.synchronize()
+        clocks.mark_end()
     if world > 1:
         dist.barrier()
     ms = ev0.elapsed_time(ev1) / args.steps

@@ -336,8 +336,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     __syncwarp();
   } else if (warp >= kVWarp0) {
     // Eq. 2 scales: each thread reduces 2 of the tile's 128 V rows.  The 128-byte
-    // swizzle only permutes 16-byte chunks within a row, so a row's absmax reads
-    // its own 8 chunks of each K half in any order.
+    // swizzle only permutes 16-byte chunks within a row, so a row's absmax may
+    // read its 8 chunks of each K half in any order: lane l reads chunk position
+    // cc ^ (row & 7), so eight consecutive rows cover all banks at every step.
     if (with_v) {
       const int vw = warp - kVWarp0;
       for (int lt = 0; lt < nt; ++lt) {
@@ -352,7 +353,8 @@ __global__ void __launch_bounds__(kLseThreads, 1)
           for (int kh = 0; kh < NKH; ++kh)
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
-              const uint4 u = *reinterpret_cast<const uint4*>(tile + kh * kHalfTileBytes + r * 128 + c * 16);
+              const uint4 u =
+                  *reinterpret_cast<const uint4*>(tile + kh * kHalfTileBytes + r * 128 + ((c ^ (r & 7)) << 4));
               mx = __vmaxu2(mx, u.x & 0x7FFF7FFFu);
               mx = __vmaxu2(mx, u.y & 0x7FFF7FFFu);
               mx = __vmaxu2(mx, u.z & 0x7FFF7FFFu);
