@@ -487,6 +487,44 @@ __device__ __forceinline__ uint2 quant8(const float (&f)[8], float gamma, float 
   return make_uint2(lo, hi);
 }
 
+// Eight codes of one 16-byte bf16 vector (the same rule as quant_code), in
+// packed arithmetic: t = v * fl(1/gamma) rounded by the 1.5*2^23 adder, the
+// code read from the low byte of the sum.  The whole vector takes the exact
+// per-value path when gamma is not a positive finite scale, 1/gamma
+// overflows, any |t| reaches qmax + 1/2 (a clamp), or any t lies within 4e-5 of a
+// rounding boundary k + 1/2 (the bound of quant_code_fast).
+__device__ __forceinline__ uint2 quant8_packed(const uint4& u, float gamma, float qmax) {
+  float f[8];
+  bf16x8_to_f32(u, f);
+  const float inv = gamma > 0.f ? __fdiv_rn(1.0f, gamma) : 0.f;
+  const float2 iv = make_float2(inv, inv);
+  const float2 big = make_float2(12582912.0f, 12582912.0f), nbig = make_float2(-12582912.0f, -12582912.0f);
+  uint32_t code[8];
+  float dmax = 0.f, tmax = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 t = fmul2(make_float2(f[2 * i], f[2 * i + 1]), iv);
+    const float2 tb = fadd2(t, big);
+    const float2 r = fadd2(tb, nbig);
+    dmax = fmax3(dmax, fabsf(t.x - r.x), fabsf(t.y - r.y));
+    tmax = fmax3(tmax, fabsf(t.x), fabsf(t.y));
+    code[2 * i] = __float_as_uint(tb.x);
+    code[2 * i + 1] = __float_as_uint(tb.y);
+  }
+  if (gamma > 0.f && gamma < 3.0e38f && inv < 3.0e38f && dmax < 0.5f - 4e-5f && tmax < qmax + 0.5f) {
+    const uint32_t lo = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
+    const uint32_t hi = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
+    return make_uint2(lo, hi);
+  }
+  uint32_t lo = 0, hi = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    lo |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[i], gamma, qmax))) << (8 * i);
+    hi |= static_cast<uint32_t>(static_cast<uint8_t>(quant_code(f[4 + i], gamma, qmax))) << (8 * i);
+  }
+  return make_uint2(lo, hi);
+}
+
 __device__ __forceinline__ uint2 quant8_bf16(const uint4& u, float gamma, float qmax) {
   float f[8];
   bf16x8_to_f32(u, f);

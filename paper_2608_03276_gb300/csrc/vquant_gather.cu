@@ -46,30 +46,34 @@ __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict_
       for (int o = LPR / 2; o >= 1; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
       const float g = __fdiv_rn(a, qmax);
       if (row < rows) {
-        if (vq) vq[row * LPR + part] = quant8(f, g, qmax);
+        if (vq) vq[row * LPR + part] = quant8_packed(u[k], g, qmax);
         if (part == 0) gamma[row] = g;
       }
     }
   }
 }
 
-// Compaction: one (document, head, slot) per LPR-lane group for K and one for
-// V, kUnroll slot groups per warp with their loads in flight together; idx < 0
-// marks an unused slot (zero-filled).
+// Compaction: a group of LPR lanes moves one (document, head, slot): lane
+// `part` copies the 16-byte part `part` of both the K and the V row and forms
+// the int8 codes of its 8 V values, so every lane runs the same code.  Each
+// lane keeps kUnroll slots in flight; idx < 0 marks an unused slot
+// (zero-filled).
 template <int LPR>
 __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ GatherParams p) {
-  constexpr int SPW = 32 / (2 * LPR);  // slots per warp instruction
+  constexpr int SPW = 32 / LPR;  // slots per warp instruction
   constexpr int UNR = 4;
   const int lane = threadIdx.x & 31;
-  const int lp = lane % (2 * LPR), part = lp % LPR;
-  const bool is_v = lp >= LPR;  // K lanes then V lanes
+  const int part = lane % LPR;
   const int b = blockIdx.z, h = blockIdx.y;
   const int64_t unit = static_cast<int64_t>(b) * p.n_heads_kv + h;
   const int64_t warp_global = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int64_t t0 = warp_global * SPW * UNR + lane / (2 * LPR);
-  const uint4* src = reinterpret_cast<const uint4*>(is_v ? p.v : p.k);
+  const int64_t t0 = warp_global * SPW * UNR + lane / LPR;
+  const uint4* kin = reinterpret_cast<const uint4*>(p.k);
+  const uint4* vin = reinterpret_cast<const uint4*>(p.v);
+  const int64_t tok0 = static_cast<int64_t>(h) * p.n_total + p.off[b];
   int32_t j[UNR];
-  uint4 val[UNR];
+  uint4 kv[UNR], vv[UNR];
+  float g[UNR];
 #pragma unroll
   for (int u = 0; u < UNR; ++u) {
     const int64_t t = t0 + u * SPW;
@@ -77,10 +81,13 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
   }
 #pragma unroll
   for (int u = 0; u < UNR; ++u) {
-    val[u] = make_uint4(0, 0, 0, 0);
+    kv[u] = vv[u] = make_uint4(0, 0, 0, 0);
+    g[u] = 0.f;
     if (j[u] >= 0) {
-      const int64_t tok = static_cast<int64_t>(h) * p.n_total + p.off[b] + j[u];
-      val[u] = __ldcs(src + tok * LPR + part);
+      const int64_t tok = tok0 + j[u];
+      kv[u] = __ldcs(kin + tok * LPR + part);
+      vv[u] = __ldcs(vin + tok * LPR + part);
+      g[u] = p.gamma[tok];
     }
   }
 #pragma unroll
@@ -88,14 +95,11 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
     if (j[u] == -2) continue;
     const int64_t slot = unit * p.cap + t0 + u * SPW;
     const int64_t dst = slot * LPR + part;
-    if (!is_v) {
-      if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = val[u];
-    } else {
-      const float g = j[u] >= 0 ? p.gamma[static_cast<int64_t>(h) * p.n_total + p.off[b] + j[u]] : 0.f;
-      if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = val[u];
-      if (p.vqc) reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_bf16(val[u], g, p.qmax) : make_uint2(0, 0);
-      if (p.gammac && part == 0) p.gammac[slot] = g;
-    }
+    if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = kv[u];
+    if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = vv[u];
+    if (p.vqc)
+      reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_packed(vv[u], g[u], p.qmax) : make_uint2(0, 0);
+    if (p.gammac && part == 0) p.gammac[slot] = g[u];
   }
 }
 
@@ -124,7 +128,7 @@ cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
   if (p.cap <= 0) return cudaSuccess;
   const int threads = 256;
   const int lpr = p.head_dim / 8;
-  const int64_t slots_per_block = (threads / 32) * (32 / (2 * lpr)) * 4;
+  const int64_t slots_per_block = (threads / 32) * (32 / lpr) * 4;
   dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
             p.batch);
   if (p.head_dim == 128)
