@@ -390,14 +390,35 @@ def run_ours(args, w):
     h2d = sum(t.numel() * t.element_size() for l in range(Le) for t in hq[l])
     d2h = sum(t.numel() * t.element_size() for l in range(Le) for t in host_out[l])
 
+    # Three streams: uploads, compression, downloads.  Layer l's upload waits
+    # for the previous compression that read its device buffers, layer l's
+    # compression waits for its upload and for the previous download of its
+    # outputs, and its download waits for its compression.
+    s_up, s_down = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev_up = [torch.cuda.Event() for _ in range(Le)]
+    ev_done = [torch.cuda.Event() for _ in range(Le)]
+    ev_down = [torch.cuda.Event() for _ in range(Le)]
+    for l in range(Le):  # every event starts recorded
+        ev_done[l].record(stream)
+        ev_down[l].record(stream)
+
     def e2e_step():
         for l in range(Le):
-            for dst, src in zip(dq[l], hq[l]):
-                dst.copy_(src, non_blocking=True)
+            s_up.wait_event(ev_done[l])
+            with torch.cuda.stream(s_up):
+                for dst, src in zip(dq[l], hq[l]):
+                    dst.copy_(src, non_blocking=True)
+            ev_up[l].record(s_up)
+            stream.wait_event(ev_up[l])
+            stream.wait_event(ev_down[l])
             o = outs[l]
             binding.compress(p, *dq[l], w.keep_ratio, w.budget, o, stream)
-            for dst, src in zip(host_out[l], (o.idx, o.kc, o.vc, o.vqc, o.gammac)):
-                dst.copy_(src, non_blocking=True)
+            ev_done[l].record(stream)
+            s_down.wait_event(ev_done[l])
+            with torch.cuda.stream(s_down):
+                for dst, src in zip(host_out[l], (o.idx, o.kc, o.vc, o.vqc, o.gammac)):
+                    dst.copy_(src, non_blocking=True)
+            ev_down[l].record(s_down)
 
     for _ in range(2):
         e2e_step()
@@ -406,9 +427,13 @@ def run_ours(args, w):
         dist.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    s_up.wait_event(e0)
+    s_down.wait_event(e0)
     esteps = max(1, args.steps)
     for _ in range(esteps):
         e2e_step()
+    for l in range(Le):  # the timed region ends when every download has landed
+        stream.wait_event(ev_down[l])
     e1.record(stream)
     torch.cuda.synchronize()
     ems = e0.elapsed_time(e1) / esteps
