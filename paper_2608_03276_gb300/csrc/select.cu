@@ -8,7 +8,9 @@
 // kept set is every key > T plus the first (k - above) keys equal to T in
 // token order (the lowest-index tie-break), written in ascending order.
 //
-// One thread-block cluster of kClusterCtas CTAs handles one (document, head):
+// One thread-block cluster of CL CTAs (8; 4 when 8 per unit would not fit in
+// one wave and every slice still fits in shared memory) handles one
+// (document, head):
 // CTA r owns a contiguous slice of the tokens.  Histograms and per-slice
 // counts live in each CTA's shared memory and are summed across the cluster
 // through distributed shared memory, separated by hardware cluster barriers,
@@ -18,6 +20,7 @@
 //   D  (> T, == T) counts per slice, then the ordered compaction into idx.
 // The kept rows are then copied by the grid-wide gather kernel.
 #include <cooperative_groups.h>
+
 
 #include "tp_device.cuh"
 
@@ -46,7 +49,7 @@ struct SelectSmem {
   int hist1[kBins1];
   int hist2[kBins2];
   int hist3[kBins3];
-  int red[kBins1 / kClusterCtas];  // this CTA's slice of the cluster-summed histogram
+  int red[kBins1 / 4];  // this CTA's slice of the cluster-summed histogram
   int red_total;
   int counts[2];  // (> T, == T) in this CTA's slice
   int scratch[33];
@@ -70,21 +73,22 @@ __device__ __forceinline__ int ld_dsmem(uint32_t addr) {
 // histogram, i.e. the sum over the cluster of every CTA's `local_hist`;
 // *above = keys in higher bins.  Called by every thread of every CTA of the
 // cluster (it contains cluster barriers).
-//   1. CTA r sums its slice of nbins/8 bins over the 8 CTAs (remote loads).
-//   2. Every CTA reads the 8 slice totals, finds the slice holding the target
+//   1. CTA r sums its slice of nbins/CL bins over the CL CTAs (remote loads).
+//   2. Every CTA reads the CL slice totals, finds the slice holding the target
 //      (highest bins first), and scans that slice's bins from its owner.
+template <int CL>
 __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const int* local_hist,
                              int nbins, int need, int* above) {
   const int rank = static_cast<int>(cluster.block_rank());
-  const int slice = nbins / kClusterCtas;  // 256 or 128 bins
+  const int slice = nbins / CL;  // at most 512 bins (CL >= 4): one per thread
   if (threadIdx.x < slice) {
     const int bin = rank * slice + threadIdx.x;
-    int v[kClusterCtas];
+    int v[CL];
 #pragma unroll
-    for (int r = 0; r < kClusterCtas; ++r) v[r] = ld_dsmem(dsmem(local_hist + bin, r));
+    for (int r = 0; r < CL; ++r) v[r] = ld_dsmem(dsmem(local_hist + bin, r));
     int t = 0;
 #pragma unroll
-    for (int r = 0; r < kClusterCtas; ++r) t += v[r];
+    for (int r = 0; r < CL; ++r) t += v[r];
     sm.red[threadIdx.x] = t;
   }
   __syncthreads();
@@ -99,7 +103,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   // slice totals, highest slice first, and the slice that holds the target
   if (threadIdx.x == 0) {
     int before = 0, s_hit = 0, s_before = 0;
-    for (int r = kClusterCtas - 1; r >= 0; --r) {
+    for (int r = CL - 1; r >= 0; --r) {
       const int t = ld_dsmem(dsmem(&sm.red_total, r));
       if (before < need && before + t >= need) {
         s_hit = r;
@@ -129,8 +133,8 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   return d;
 }
 
-__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads, 1)
-    tp_select_kernel(const __grid_constant__ SelectParams p) {
+template <int CL>
+__global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_constant__ SelectParams p) {
   extern __shared__ uint8_t smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
@@ -142,7 +146,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
   const int k = p.kept[b];
   const size_t row = static_cast<size_t>(h) * p.n_total + lo;
   // this CTA's slice [s0, s1) of the document's tokens
-  const int per_cta = (((n + kClusterCtas - 1) / kClusterCtas) + 3) & ~3;
+  const int per_cta = (((n + CL - 1) / CL) + 3) & ~3;
   const int s0 = min(rank * per_cta, n), s1 = min(s0 + per_cta, n);
   // the slice's keys: in shared memory when they fit, else in the global scratch
   const bool in_smem = (s1 - s0 <= kSliceKeys);
@@ -227,7 +231,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
   int need_eq = -1;  // -1: keep every token of the document
   if (kk > 0 && kk < n) {
     int above;
-    const int d1 = cluster_digit(cluster, sm, sm.hist1, kBins1, kk, &above);
+    const int d1 = cluster_digit<CL>(cluster, sm, sm.hist1, kBins1, kk, &above);
     int need = kk - above;
     for (int base = s0; base < s1; base += kThreads) {
       const int i = base + threadIdx.x;
@@ -235,7 +239,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
       if (i < s1 && (key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
     }
     cluster.sync();
-    const int d2 = cluster_digit(cluster, sm, sm.hist2, kBins2, need, &above);
+    const int d2 = cluster_digit<CL>(cluster, sm, sm.hist2, kBins2, need, &above);
     need -= above;
     const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
     for (int base = s0; base < s1; base += kThreads) {
@@ -244,7 +248,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
       if (i < s1 && (key >> 10) == pre) atomicAdd(&sm.hist3[key & 0x3FF], 1);
     }
     cluster.sync();
-    const int d3 = cluster_digit(cluster, sm, sm.hist3, kBins3, need, &above);
+    const int d3 = cluster_digit<CL>(cluster, sm, sm.hist3, kBins3, need, &above);
     need_eq = need - above;
     thr = (pre << 10) | static_cast<uint32_t>(d3);
   } else {
@@ -324,15 +328,41 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreads,
 
 size_t select_smem_bytes() { return sizeof(SelectSmem); }
 
+template <int CL>
+cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(CL, units);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL>, p);
+}
+
 cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
   const int units = p.batch * p.n_heads_kv;
   if (units <= 0) return cudaSuccess;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
   const size_t smem = sizeof(SelectSmem);
-  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel), 0);
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t n_max = 0;
+  for (int b = 0; b < p.batch; ++b) n_max = p.off[b + 1] - p.off[b] > n_max ? p.off[b + 1] - p.off[b] : n_max;
+  // Fewer, larger slices when eight CTAs per unit would need more than one wave.
+  if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys) {
+    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<4>), 11);
+    if (e != cudaSuccess) return e;
+    return launch_select_t<4>(p, units, smem, s);
+  }
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<8>), 0);
   if (e != cudaSuccess) return e;
-  tp_select_kernel<<<dim3(kClusterCtas, units), kThreads, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_select_t<8>(p, units, smem, s);
 }
 
 }  // namespace tp

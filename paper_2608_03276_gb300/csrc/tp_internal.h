@@ -68,7 +68,6 @@ struct KeyScoreParams {
 };
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
-constexpr int kClusterCtas = 8;    // CTAs (one cluster) per (document, head) in the selection
 
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
