@@ -103,6 +103,68 @@ __device__ __forceinline__ float sum_exp2(const float (&x)[32], float c2, float 
   return t.x + t.y;
 }
 
+// Value i of a 64-column span held as two 32-register chunks.
+#define TP_X64(i) __uint_as_float((i) < 32 ? ra[(i) & 31] : rb[(i) & 31])
+
+__device__ __forceinline__ float max64(const uint32_t (&ra)[32], const uint32_t (&rb)[32]) {
+  float t[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    t[k] = fmax3(TP_X64(8 * k), TP_X64(8 * k + 1), TP_X64(8 * k + 2));
+    t[k] = fmax3(t[k], TP_X64(8 * k + 3), TP_X64(8 * k + 4));
+    t[k] = fmax3(t[k], TP_X64(8 * k + 5), TP_X64(8 * k + 6));
+    t[k] = fmaxf(t[k], TP_X64(8 * k + 7));
+  }
+  return fmaxf(fmax3(fmax3(t[0], t[1], t[2]), fmax3(t[3], t[4], t[5]), t[6]), t[7]);
+}
+
+// sum_i 2^(x_i * c2 + off) over a 64-column span, four packed partial sums.
+__device__ __forceinline__ float sum_exp2_64(const uint32_t (&ra)[32], const uint32_t (&rb)[32],
+                                             float c2, float off) {
+  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                 make_float2(0.f, 0.f)};
+  const float2 cc = make_float2(c2, c2), oo = make_float2(off, off);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const float2 y = ffma2(make_float2(TP_X64(2 * i), TP_X64(2 * i + 1)), cc, oo);
+    a[i & 3] = fadd2(a[i & 3], make_float2(ex2(y.x), ex2(y.y)));
+  }
+  const float2 t = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
+  return t.x + t.y;
+}
+#undef TP_X64
+
+// lse_chunk (below) for a 64-column span given as two 32-column chunks: one
+// offset decision for all 64 values; columns >= `valid` are masked in place.
+__device__ __forceinline__ void lse_chunk64(uint32_t (&ra)[32], uint32_t (&rb)[32], int col0,
+                                            int valid, float c2, float& m, float& z) {
+  if (valid < col0 + 64) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      if (col0 + i >= valid) ra[i] = 0xFF800000u;  // -inf
+      if (col0 + 32 + i >= valid) rb[i] = 0xFF800000u;
+    }
+  }
+  float s = 0.f;
+  bool exact = (m == -INFINITY);
+  if (!exact) {
+    s = sum_exp2_64(ra, rb, c2, -m);
+    exact = !(s <= 0x1p64f);
+  }
+  if (exact) {
+    const float mn = fmaxf(m, max64(ra, rb) * c2);
+    if (mn == -INFINITY) return;
+    s = sum_exp2_64(ra, rb, c2, -mn);
+    z *= ex2(m - mn);
+    m = mn;
+  }
+  z += s;
+  if (z > 0x1p64f) {
+    z *= 0x1p-64f;
+    m += 64.f;
+  }
+}
+
 // One 32-column chunk of a guide row's logits into the running (offset m,
 // sum z) of pass 1, both in log2 units: z = sum 2^(x*c2 - m).  The offset is
 // refreshed from the exact chunk maximum only when it is unset or the chunk
@@ -227,7 +289,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     }
     for (int i = 0; i < NB; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], kEpiWarps);
+      mbar_init(&tempty[i], kEpiWarps / 2);  // one group of eight warps drains a buffer
     }
     mbar_init(drain, 1);
     for (int i = 0; i < kVStages; ++i) {
@@ -300,12 +362,8 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   __syncthreads();
   tc_fence_after();
 
-  float m[NRB], z[NRB];  // epilogue: running (offset, sum) per row block
-#pragma unroll
-  for (int rb = 0; rb < NRB; ++rb) {
-    m[rb] = -INFINITY;
-    z[rb] = 0.f;
-  }
+  // epilogue: running (offset, sum) per row block this warp sees (two with NRB = 4)
+  float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f};
 
   if (warp == 0) {
     if (lane == 0) {
@@ -402,26 +460,34 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     }
     __syncwarp();
   } else {
-    const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
+    // Two groups of eight warps take alternate jobs (group G = jobs j with
+    // j % 2 == G), so one group's TMEM loads overlap the other's arithmetic.
+    // In a group, warpgroup half h owns columns 64h..64h+63 of the job.
+    const int wg = (warp - kEpiWarp0) >> 2, grp = wg >> 1, hcol = wg & 1, quad = warp & 3;
     const float c2 = p.c2;
-    const uint32_t tcol = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ACOLS + g * 32;
+    const uint32_t tcol = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ACOLS + hcol * 64;
+    const int njobs = nt * NRB;
     bool ok = true;
-    for (int lt = 0; ok && lt < nt; ++lt) {
-      const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
-#pragma unroll
-      for (int rb = 0; rb < NRB; ++rb) {
-        const int j = lt * NRB + rb, buf = j % NB;
-        if (ok && !mbar_wait(&tfull[buf], (j / NB) & 1, abort_flag)) ok = false;
-        if (!ok) break;
-        tc_fence_after();
-        uint32_t r[32];
-        tmem_ld32_async(tcol + buf * 128, r);
-        tmem_wait(r);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[buf]);
-        lse_chunk(r, g * 32, valid, c2, m[rb], z[rb]);
+    for (int j = grp; ok && j < njobs; j += 2) {
+      const int buf = j % NB, lt = j / NRB;
+      if (!mbar_wait(&tfull[buf], (j / NB) & 1, abort_flag)) {
+        ok = false;
+        break;
       }
+      tc_fence_after();
+      uint32_t ra[32], rb[32];
+      tmem_ld32_async(tcol + buf * 128, ra);
+      tmem_ld32_async(tcol + buf * 128 + 32, rb);
+      tmem_wait(ra);
+      tmem_wait(rb);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
+      const int valid = min(kKeyTile, n - (t0 + lt) * kKeyTile);
+      // row block j % NRB: this group sees rb = grp, grp + 2 (NRB = 4), grp (NRB = 2), 0 (NRB = 1)
+      const int slot = NRB == 4 ? (j % NRB) >> 1 : 0;
+      if (slot == 0) lse_chunk64(ra, rb, hcol * 64, valid, c2, m[0], z[0]);
+      else lse_chunk64(ra, rb, hcol * 64, valid, c2, m[NRB == 4 ? 1 : 0], z[NRB == 4 ? 1 : 0]);
     }
   }
   // Every stream has landed and every MMA has finished: the K ring is free.
@@ -432,10 +498,16 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     if (threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
   } else {
     if (warp >= kEpiWarp0 && warp < kVWarp0) {
-      const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
+      const int g = (warp - kEpiWarp0) >> 2, grp = g >> 1, quad = warp & 3;
 #pragma unroll
-      for (int rb = 0; rb < NRB; ++rb)
-        stats[g * rows_pad + rb * 128 + quad * 32 + lane] = make_float2(m[rb], z[rb]);
+      for (int rb = 0; rb < NRB; ++rb) {
+        // this warp's (offset, sum) for row block rb, or the empty pair
+        float2 st = make_float2(-INFINITY, 0.f);
+        if (NRB == 1) st = make_float2(m[0], z[0]);
+        else if (NRB == 2 && rb == grp) st = make_float2(m[0], z[0]);
+        else if (NRB == 4 && (rb & 1) == grp) st = make_float2(m[rb >> 1], z[rb >> 1]);
+        stats[g * rows_pad + rb * 128 + quad * 32 + lane] = st;
+      }
     }
     __syncthreads();
     for (int r = threadIdx.x; r < rows_pad; r += blockDim.x) {
