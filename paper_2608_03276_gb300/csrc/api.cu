@@ -236,7 +236,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
 int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const float* lse,
-                 float* skey, int* status, cudaStream_t s) {
+                 float* skey, int* status, bool dependent, cudaStream_t s) {
   KeyScoreParams kp;
   memset(&kp, 0, sizeof(kp));
   kp.docs = doc_table(P);
@@ -252,7 +252,8 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
   kp.lse = lse;
   kp.skey = skey;
   kp.status = status;
-  return cuda_status(launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, s));
+  return cuda_status(
+      launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
 }
 
 // Both scoring passes (with the Eq. 2 scales fused into the first when gamma
@@ -266,7 +267,7 @@ int run_scoring(const Plan& P, const void* q, const void* k, const void* v, floa
   int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s);
   if (st != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
-                      reinterpret_cast<int*>(ws + P.ws_status), s);
+                      reinterpret_cast<int*>(ws + P.ws_status), true, s);
 }
 
 void fill_select(const Plan& P, char* ws, SelectParams* sp) {
@@ -410,7 +411,7 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
   sp.gamma = gamma;
   sp.scores_out = scores;
   sp.scores_only = 1;
-  return cuda_status(launch_select(sp, s));
+  return cuda_status(launch_select(sp, true, s));
 }
 
 int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* v, float* lse,
@@ -459,7 +460,8 @@ int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_keyscore(P, tmk, tmq, lse, key_scores, nullptr, static_cast<cudaStream_t>(stream));
+  return run_keyscore(P, tmk, tmq, lse, key_scores, nullptr, false,
+                      static_cast<cudaStream_t>(stream));
 }
 
 int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64_t budget,
@@ -477,7 +479,7 @@ int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64
   fill_select(P, w, &sp);
   sp.scores_in = scores;
   sp.idx = idx;
-  return cuda_status(launch_select(sp, s));
+  return cuda_status(launch_select(sp, false, s));
 }
 
 int tp_compact(const tp_problem* p, const void* k, const void* v, const float* gamma,
@@ -501,7 +503,7 @@ int tp_compact(const tp_problem* p, const void* k, const void* v, const float* g
   gp.vc = static_cast<uint16_t*>(vc);
   gp.vqc = vqc;
   gp.gammac = gammac;
-  return cuda_status(launch_gather(gp, static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_gather(gp, false, static_cast<cudaStream_t>(stream)));
 }
 
 int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
@@ -531,7 +533,7 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
   sp.gamma = g;
   sp.scores_out = scores;
   sp.idx = idx;
-  cudaError_t e2 = launch_select(sp, s);
+  cudaError_t e2 = launch_select(sp, true, s);
   if (e2 != cudaSuccess) return TP_ERR_CUDA;
   if (P.cap == 0) return TP_OK;
   GatherParams gp;
@@ -544,7 +546,7 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
   gp.vc = static_cast<uint16_t*>(vc);
   gp.vqc = vqc;
   gp.gammac = gammac;
-  return cuda_status(launch_gather(gp, s));
+  return cuda_status(launch_gather(gp, true, s));
 }
 
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {

@@ -281,6 +281,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   const int ntiles = (n + kKeyTile - 1) / kKeyTile;
   const int t0 = c * p.tiles_per_cta;
   const int nt = min(p.tiles_per_cta, ntiles - t0);
+  grid_dep_launch();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -613,6 +614,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
+  grid_dep_launch();
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  // The guide block and the first K tiles are inputs of the whole layer: they
+  // may load while pass 1 (this kernel's predecessor) finishes.
+  const int k_pre = min(stages, nt);
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmk);
+    prefetch_tensormap(&tmq);
+    load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
+    for (int lt = 0; lt < k_pre; ++lt) {
+      mbar_arrive_expect_tx(&full_k[lt], KT);
+      const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
+#pragma unroll
+      for (int kh = 0; kh < NKH; ++kh)
+        tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[lt]);
+    }
+  }
+  grid_dep_wait();  // the row normalisers come from pass 1
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
     for (int r = threadIdx.x; r < 128 + rows_pad; r += blockDim.x) {
@@ -638,22 +663,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     fence_proxy_async_smem();  // read by the tensor core
   }
-  if (warp == 0) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
   __syncthreads();
-  tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
     if (lane == 0) {
-      prefetch_tensormap(&tmk);
-      prefetch_tensormap(&tmq);
-      load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
-      int issued = 0;
-      for (int lt = 0; lt < nt; ++lt) {
+      int issued = k_pre;
+      for (int lt = k_pre; lt < nt; ++lt) {
         const int s = lt % stages, use = lt / stages;
         if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
         mbar_arrive_expect_tx(&full_k[s], KT);
@@ -790,17 +806,23 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUt
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
-                            cudaStream_t s) {
-  if (head_dim == 128) {
-    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<128>), 8);
-    if (e != cudaSuccess) return e;
-    tp_keyscore_kernel<128><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
-  } else {
-    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<64>), 9);
-    if (e != cudaSuccess) return e;
-    tp_keyscore_kernel<64><<<grid, kThreads, smem, s>>>(tmk, tmq, p);
-  }
-  return cudaGetLastError();
+                            bool dependent, cudaStream_t s) {
+  const void* fn = head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_kernel<128>)
+                                   : reinterpret_cast<const void*>(tp_keyscore_kernel<64>);
+  cudaError_t e = set_smem_once(fn, head_dim == 128 ? 8 : 9);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 1 : 0;
+  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<128>, tmk, tmq, p)
+                         : cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<64>, tmk, tmq, p);
 }
 
 }  // namespace tp

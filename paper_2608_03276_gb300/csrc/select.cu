@@ -153,11 +153,13 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   uint32_t* const keys_base = in_smem ? sm.keys : p.keys + row;
   const int kofs = in_smem ? s0 : 0;  // keys of token i live at keys_base[i - kofs]
 
+  grid_dep_launch();
   for (int i = threadIdx.x; i < kBins1; i += kThreads) {
     sm.hist1[i] = 0;
     sm.hist2[i] = 0;
   }
   for (int i = threadIdx.x; i < kBins3; i += kThreads) sm.hist3[i] = 0;
+  grid_dep_wait();  // key scores and scales come from the scoring kernels
   __syncthreads();
 
   // A: keys of the slice (scores formed here in the fused path) + digit-1 histogram,
@@ -329,23 +331,26 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 size_t select_smem_bytes() { return sizeof(SelectSmem); }
 
 template <int CL>
-cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, cudaStream_t s) {
+cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool dependent,
+                            cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(CL, units);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = CL;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = dependent ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL>, p);
 }
 
-cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
+cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s) {
   const int units = p.batch * p.n_heads_kv;
   if (units <= 0) return cudaSuccess;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
@@ -358,11 +363,11 @@ cudaError_t launch_select(const SelectParams& p, cudaStream_t s) {
   if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys) {
     cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<4>), 11);
     if (e != cudaSuccess) return e;
-    return launch_select_t<4>(p, units, smem, s);
+    return launch_select_t<4>(p, units, smem, dependent, s);
   }
   cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<8>), 0);
   if (e != cudaSuccess) return e;
-  return launch_select_t<8>(p, units, smem, s);
+  return launch_select_t<8>(p, units, smem, dependent, s);
 }
 
 }  // namespace tp

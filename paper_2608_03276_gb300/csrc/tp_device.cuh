@@ -40,6 +40,15 @@ __device__ __forceinline__ float lg2(float x) {
   return y;
 }
 
+// Programmatic dependent launch: a kernel launched as a dependent may start
+// while its predecessor in the stream finishes; grid_dep_wait() returns once
+// the predecessor has completed and its writes are visible (at once when the
+// kernel was not launched as a dependent).  grid_dep_launch() lets this
+// kernel's own dependent be scheduled as soon as every CTA of this grid has
+// issued it.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;"); }
+
 // Records a device-side failure in the workspace status word (first writer wins).
 __device__ __forceinline__ void set_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);

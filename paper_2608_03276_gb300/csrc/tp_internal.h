@@ -111,11 +111,14 @@ cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t r
                           float qmax, int num_sms, cudaStream_t s);
 cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                        const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s);
+// `dependent`: launch as a programmatic dependent of the previous kernel in
+// the stream (only where that kernel and this one belong to one layer's
+// sequence, whose inputs were written before its first kernel started).
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
-                            cudaStream_t s);
-cudaError_t launch_select(const SelectParams& p, cudaStream_t s);
-cudaError_t launch_gather(const GatherParams& p, cudaStream_t s);
+                            bool dependent, cudaStream_t s);
+cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
+cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once per
 // (kernel slot, device); `slot` names the kernel in a small registry.

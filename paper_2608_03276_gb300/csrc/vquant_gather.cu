@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
   const uint4* kin = reinterpret_cast<const uint4*>(p.k);
   const uint4* vin = reinterpret_cast<const uint4*>(p.v);
   const int64_t tok0 = static_cast<int64_t>(h) * p.n_total + p.off[b];
+  grid_dep_wait();  // idx comes from the selection kernel
   int32_t j[UNR];
   uint4 kv[UNR], vv[UNR];
   float g[UNR];
@@ -124,18 +125,24 @@ cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t r
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather(const GatherParams& p, cudaStream_t s) {
+cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s) {
   if (p.cap <= 0) return cudaSuccess;
   const int threads = 256;
   const int lpr = p.head_dim / 8;
   const int64_t slots_per_block = (threads / 32) * (32 / lpr) * 4;
   dim3 grid(static_cast<unsigned>((p.cap + slots_per_block - 1) / slots_per_block), p.n_heads_kv,
             p.batch);
-  if (p.head_dim == 128)
-    tp_gather_kernel<16><<<grid, threads, 0, s>>>(p);
-  else
-    tp_gather_kernel<8><<<grid, threads, 0, s>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(threads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 1 : 0;
+  return p.head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_gather_kernel<16>, p)
+                           : cudaLaunchKernelEx(&cfg, tp_gather_kernel<8>, p);
 }
 
 }  // namespace tp
