@@ -25,7 +25,9 @@ Readings of the paper used here (where it is silent or ambiguous):
   +-(2^(b-1) - 1); gamma = 0 gives all-zero codes;
 * scale - softmax scale 1/sqrt(d) unless given;
 * budget - kept = ceil(ratio * n - 1e-9 * n) clamped to [0, n];
-* ties - equal scores keep the lower token index; kept indices ascend.
+* ties - equal scores keep the lower token index; kept indices ascend;
+* blends - the aggregation ablation's normalised add uses L2 norms over one
+  (document, head); its harmonic mean reads the printed ',' as '+'.
 
 Parity pins for every function live in tests/test_oracle_pins.py.
 """
@@ -132,6 +134,22 @@ def key_scores(q_group: np.ndarray, k_ctx: np.ndarray, sigma: float) -> np.ndarr
     return a.sum(axis=0) / g
 
 
+def key_scores_given_lse(q_group: np.ndarray, k_ctx: np.ndarray, sigma: float,
+                         lse_rows: np.ndarray) -> np.ndarray:
+    """key_scores with each row's softmax normaliser supplied by the caller.
+
+    s[i] = (1/G) * sum_r exp(sigma * q_r . k_i - lse_r) over the G*L_t rows
+    r = (g, j).  The method slices A out of the full prefill attention map
+    (Sec. 3.2), whose row normaliser also covers the guide's own causal prefix;
+    a caller that keeps the prefill's per-row log-sum-exp passes it here, which
+    gives that literal normaliser and needs no normalisation pass.  With lse_r =
+    guide_lse(...) this equals key_scores.
+    """
+    g, lt, d = q_group.shape
+    x = (q_group.reshape(g * lt, d) @ k_ctx.T) * sigma
+    return np.exp(x - np.asarray(lse_rows, dtype=np.float64)[:, None]).sum(axis=0) / g
+
+
 def pool(s: np.ndarray, kernel: int) -> np.ndarray:
     """Eq. 1's 1-D average pooling with window K (odd), zero outside [0, n)."""
     if kernel < 1 or kernel % 2 == 0:
@@ -146,11 +164,37 @@ def pool(s: np.ndarray, kernel: int) -> np.ndarray:
     return out / kernel
 
 
-def combine(pooled: np.ndarray, gamma: np.ndarray, key_only: bool = False) -> np.ndarray:
-    """Eq. 3: s_i = s_key_i * s_value_i with s_value_i = gamma_i (Sec. 3.3-3.4)."""
+COMBINE_MODES = ("mul", "normadd", "harmonic")
+
+
+def combine(pooled: np.ndarray, gamma: np.ndarray, key_only: bool = False,
+            mode: str = "mul") -> np.ndarray:
+    """Eq. 3: s_i = s_key_i * s_value_i with s_value_i = gamma_i (Sec. 3.3-3.4).
+
+    The two other blends of the aggregation ablation (Sec. 6, "Score
+    aggregation strategy"), over one (document, head):
+      normadd   s_key_i / ||s_key||_2 + s_value_i / ||s_value||_2, a term whose
+                norm is 0 contributing 0;
+      harmonic  2 s_key_i s_value_i / (s_key_i + s_value_i), 0 where the sum
+                is 0 (the printed formula has ',' for '+').
+    key_only drops s_value (Sec. 6, the key-only row of the ablation).
+    """
     if key_only:
         return pooled.copy()
-    return pooled * np.asarray(gamma, dtype=np.float64)
+    a = np.asarray(pooled, dtype=np.float64)
+    b = np.asarray(gamma, dtype=np.float64)
+    if mode == "mul":
+        return a * b
+    if mode == "normadd":
+        na, nb = math.sqrt(float(np.sum(a * a))), math.sqrt(float(np.sum(b * b)))
+        return (a / na if na > 0 else 0.0 * a) + (b / nb if nb > 0 else 0.0 * b)
+    if mode == "harmonic":
+        den = a + b
+        out = np.zeros_like(a)
+        nz = den != 0
+        out[nz] = 2.0 * a[nz] * b[nz] / den[nz]
+        return out
+    raise ValueError(f"unknown combine mode {mode!r}")
 
 
 # --------------------------------------------------------------------------
@@ -168,12 +212,15 @@ def select_topk(scores: np.ndarray, k: int) -> np.ndarray:
 def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
                    n_heads_q: int, n_heads_kv: int, keep_ratio: float = 0.25,
                    fixed_budget: int = -1, pool_kernel: int = 5, quant_bits: int = 8,
-                   softmax_scale: float = 0.0, key_only: bool = False,
-                   heads: Optional[Sequence[int]] = None, docs: Optional[Sequence[int]] = None):
+                   softmax_scale: float = 0.0, key_only: bool = False, combine_mode: str = "mul",
+                   lse=None, heads: Optional[Sequence[int]] = None,
+                   docs: Optional[Sequence[int]] = None):
     """The whole compression of one layer (Sec. 3.1-3.4 with Sec. 4 budgets).
 
     q_bits [batch, H_q, L_t, d], k_bits / v_bits [H_kv, N_total, d] (bf16 bits),
-    doc_offsets [batch+1].  Returns a dict:
+    doc_offsets [batch+1].  ``lse`` [batch, H_kv, G*L_t] (natural log), when
+    given, replaces each guide row's normaliser (key_scores_given_lse);
+    ``combine_mode`` selects the blend of ``combine``.  Returns a dict:
       gamma  [H_kv, N_total] float32, vq [H_kv, N_total, d] int8,
       scores {(b, h): float64 [n_b]}  combined scores s_i,
       key    {(b, h): float64 [n_b]}  unpooled key scores,
@@ -198,8 +245,13 @@ def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
         for h in heads:
             qg = q[b, h * g:(h + 1) * g]
             # an empty document has no context tokens: nothing to score or keep
-            s_key = key_scores(qg, k_all[h, lo:hi], sigma) if n > 0 else np.zeros(0)
-            s = combine(pool(s_key, pool_kernel), gamma[h, lo:hi], key_only)
+            if n == 0:
+                s_key = np.zeros(0)
+            elif lse is None:
+                s_key = key_scores(qg, k_all[h, lo:hi], sigma)
+            else:
+                s_key = key_scores_given_lse(qg, k_all[h, lo:hi], sigma, np.asarray(lse)[b, h])
+            s = combine(pool(s_key, pool_kernel), gamma[h, lo:hi], key_only, combine_mode)
             out["key"][(b, h)] = s_key
             out["scores"][(b, h)] = s
             out["idx"][(b, h)] = select_topk(s, kb)

@@ -237,6 +237,47 @@ def pin_combine_product(O):
     assert list(O.combine(a, g, key_only=True)) == [0.5, 2.0, 0.0, 3.0]
 
 
+def pin_key_scores_given_lse(O):
+    """With Q = 0 every logit is 0, so exp(x - lse_r) = 1/(n + c_r) when the
+    caller's normaliser lse_r = log(n + c_r) also counts guide-prefix mass c_r
+    (the literal prefill normaliser, Sec. 3.2): s_i = (1/G) sum_r 1/(n + c_r).
+    A shift of every normaliser by D scales every score by exp(-D); with the
+    context-only normaliser the scores equal key_scores (uniform: L_t / n)."""
+    g, lt, d, n = 2, 3, 8, 10
+    q = np.zeros((g, lt, d))
+    k = _rand(1, (n, d))
+    c = np.array([0.0, 1.0, 2.0, 5.0, 0.5, 3.0])
+    s = O.key_scores_given_lse(q, k, 0.3, np.log(n + c))
+    want = sum(1.0 / (n + cr) for cr in c) / g
+    assert np.allclose(s, want, rtol=1e-13, atol=0)
+    s0 = O.key_scores_given_lse(q, k, 0.3, np.full(g * lt, math.log(n)))
+    assert np.allclose(s0, lt / n, rtol=1e-13, atol=0)
+    qr = _rand(2, (g, lt, d))
+    lse = np.linspace(2.0, 4.0, g * lt)
+    a = O.key_scores_given_lse(qr, k, 0.25, lse)
+    b = O.key_scores_given_lse(qr, k, 0.25, lse + 0.75)
+    assert np.allclose(b, a * math.exp(-0.75), rtol=1e-12, atol=0)
+
+
+def pin_combine_normadd(O):
+    """Normalised add (Sec. 6 aggregation ablation): L2 norms over the vector.
+    (3, 4) and (5, 12) have norms 5 and 13; each term is scale-free; a zero
+    vector contributes nothing."""
+    a, g = np.array([3.0, 4.0]), np.array([5.0, 12.0])
+    s = O.combine(a, g, mode="normadd")
+    assert np.allclose(s, [0.6 + 5 / 13, 0.8 + 12 / 13], rtol=1e-15, atol=0)
+    assert np.allclose(O.combine(7.0 * a, 0.01 * g, mode="normadd"), s, rtol=1e-14, atol=0)
+    assert np.allclose(O.combine(a, np.zeros(2), mode="normadd"), [0.6, 0.8], rtol=1e-15, atol=0)
+
+
+def pin_combine_harmonic(O):
+    """Harmonic mean 2ab/(a+b): (1,1) -> 1, (1,3) -> 3/2, (2,6) -> 3, (0,x) -> 0,
+    and 0 where both are 0."""
+    a = np.array([1.0, 1.0, 2.0, 0.0, 0.0])
+    g = np.array([1.0, 3.0, 6.0, 5.0, 0.0])
+    assert list(O.combine(a, g, mode="harmonic")) == [1.0, 1.5, 3.0, 0.0, 0.0]
+
+
 def _brute_topk(scores, k):
     """Max-sum subset of size k; among equal sums the lexicographically smallest."""
     best, best_set = None, None

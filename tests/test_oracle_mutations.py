@@ -30,14 +30,19 @@ MUTATIONS = {
     "quant rounds half away from zero": ("q = np.clip(np.rint(quot), -qmax, qmax)", "q = np.clip(np.trunc(quot + np.copysign(0.5, quot)), -qmax, qmax)"),
     "quant truncates": ("q = np.clip(np.rint(quot), -qmax, qmax)", "q = np.clip(np.trunc(quot), -qmax, qmax)"),
     "quant uses mean |v|": ("a = np.max(np.abs(v), axis=-1)", "a = np.mean(np.abs(v), axis=-1)"),
-    "additive combine": ("return pooled * np.asarray(gamma, dtype=np.float64)", "return pooled + np.asarray(gamma, dtype=np.float64)"),
+    "additive combine": ("        return a * b\n", "        return a + b\n"),
     "ties keep the higher index": ("order = np.lexsort((np.arange(n), -scores))", "order = np.lexsort((-np.arange(n), -scores))"),
     "selects the smallest scores": ("order = np.lexsort((np.arange(n), -scores))", "order = np.lexsort((np.arange(n), scores))"),
     "kept indices not ascending": ("return np.sort(order[:k]).astype(np.int64)", "return order[:k].astype(np.int64)"),
     "naive ceil budget": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.ceil(keep_ratio * float(n))"),
     "budget rounds down": ("k = math.ceil(keep_ratio * float(n) - 1e-9 * float(n))", "k = math.floor(keep_ratio * float(n))"),
     "gather ignores the document offset": ("tok = doc_lo + np.asarray(idx, dtype=np.int64)", "tok = np.asarray(idx, dtype=np.int64)"),
-    "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma) if", "s_key = key_scores(qg, k_all[h, 0:n], sigma) if"),
+    "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma)\n", "s_key = key_scores(qg, k_all[h, 0:n], sigma)\n"),
+    "given normaliser added": ("np.exp(x - np.asarray(lse_rows", "np.exp(x + np.asarray(lse_rows"),
+    "given-normaliser scores not averaged over G": ("[:, None]).sum(axis=0) / g", "[:, None]).sum(axis=0)"),
+    "normalised add with L1 norms": ("na, nb = math.sqrt(float(np.sum(a * a))), math.sqrt(float(np.sum(b * b)))", "na, nb = float(np.sum(np.abs(a))), float(np.sum(np.abs(b)))"),
+    "harmonic mean without the factor 2": ("out[nz] = 2.0 * a[nz] * b[nz] / den[nz]", "out[nz] = a[nz] * b[nz] / den[nz]"),
+    "harmonic mean divides by a zero sum": ("nz = den != 0", "nz = den == den"),
 }
 
 
