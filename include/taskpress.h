@@ -55,6 +55,14 @@ extern "C" {
 
 /* Flags (tp_problem.flags). */
 #define TP_SCORE_KEY_ONLY 0x1u /* s_i = pooled key score only (Sec. 4.3.1 ablation) */
+/* The other blends of the Sec. 6 aggregation ablation (at most one flag):
+ *   TP_SCORE_NORM_ADD  s_i = s_key_i / ||s_key||_2 + gamma_i / ||gamma||_2, the
+ *                      L2 norms taken over one document and KV head (a zero
+ *                      norm drops its term);
+ *   TP_SCORE_HARMONIC  s_i = 2 s_key_i gamma_i / (s_key_i + gamma_i), 0 where
+ *                      the sum is 0 (the paper prints ',' for '+'). */
+#define TP_SCORE_NORM_ADD 0x2u
+#define TP_SCORE_HARMONIC 0x4u
 
 /* Limits. */
 #define TP_MAX_BATCH 256   /* documents per call                              */
@@ -72,7 +80,8 @@ extern "C" {
  *   pool_kernel           : K of Eq. 1's average pooling; odd, 1..33 (default 5)
  *   quant_bits            : b of Eq. 2; only 8 is supported
  *   softmax_scale         : logit scale; <= 0 means 1/sqrt(d)
- *   flags                 : TP_SCORE_KEY_ONLY or 0
+ *   flags                 : 0 (Eq. 3 product), or one of TP_SCORE_KEY_ONLY,
+ *                           TP_SCORE_NORM_ADD, TP_SCORE_HARMONIC
  */
 typedef struct tp_problem {
   int32_t n_heads_q;
@@ -126,7 +135,8 @@ int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, 
  *   s_key_i = (1/K) sum_{k=-K/2..K/2} (1/G) sum_{rows r of the group} A[r, i+k]
  *       (Eq. 1; rows are the G*L_t guide rows of the KV head's query heads,
  *       terms outside the document are zero),
- *   s_i = s_key_i * gamma_i (Eq. 3), or s_key_i with TP_SCORE_KEY_ONLY.
+ *   s_i = s_key_i * gamma_i (Eq. 3), or s_key_i with TP_SCORE_KEY_ONLY, or
+ *   the TP_SCORE_NORM_ADD / TP_SCORE_HARMONIC blend.
  * q: [batch, H_q, L_t, d] bf16; k: [H_kv, N, d] bf16; gamma: [H_kv, N] fp32
  * (may be NULL only with TP_SCORE_KEY_ONLY); scores: [H_kv, N] fp32 out.
  * ws / ws_bytes: workspace of at least tp_workspace_bytes(p, 0, 0).
@@ -214,6 +224,22 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
                       double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
                       int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
                       size_t ws_bytes, void* stream);
+
+/*
+ * tp_compress_layer with the caller's row normalisers: `lse` ([batch, H_kv, M]
+ * fp32, natural log, rows ordered as in tp_guide_lse) replaces the normalising
+ * pass, so the scores take one pass over K (Sec. 3.2; survey row f2).  The
+ * method slices A out of the full prefill attention map; a caller that keeps
+ * that attention's per-row log-sum-exp for the guide rows passes it here and
+ * gets the paper's literal normaliser, which also counts the guide's own
+ * causal prefix.  With lse from tp_guide_lse the result equals
+ * tp_compress_layer's.  The Eq. 2 scales come from a separate pass over V.
+ * Other arguments, outputs and workspace as in tp_compress_layer.
+ */
+int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, const void* v,
+                          const float* lse, double keep_ratio, int64_t budget, int32_t* idx,
+                          void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
+                          float* gamma, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * Synchronises `stream`, then reads the device status word that the kernels of

@@ -23,6 +23,8 @@ TP_ERR_UNSUPPORTED_SHAPE = -3
 TP_ERR_CUDA = -4
 TP_ERR_TIMEOUT = -5
 TP_SCORE_KEY_ONLY = 0x1
+TP_SCORE_NORM_ADD = 0x2
+TP_SCORE_HARMONIC = 0x4
 TP_MAX_BATCH = 256
 TP_MAX_ROWS = 512
 #: kernels one tp_compress_layer call launches (scoring pass 1 with the V
@@ -33,7 +35,7 @@ KERNELS_PER_COMPRESS = 4
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
            "tp_select", "tp_compact",
-           "tp_compress_layer", "tp_check_status", "tp_status_string")
+           "tp_compress_layer", "tp_compress_layer_lse", "tp_check_status", "tp_status_string")
 
 
 class TpProblem(ctypes.Structure):
@@ -99,6 +101,10 @@ def load(path: Optional[str] = None):
     lib.tp_compress_layer.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_double,
                                       c_int64, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                       c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
+    lib.tp_compress_layer_lse.restype = c_int
+    lib.tp_compress_layer_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
+                                          c_double, c_int64, c_void_p, c_void_p, c_void_p, c_void_p,
+                                          c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
     lib.tp_check_status.restype = c_int
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
@@ -279,6 +285,28 @@ def tp_compress_layer(p: Problem, q, k, v, keep_ratio: float, budget: int, idx, 
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 
+def tp_compress_layer_lse(p: Problem, q, k, v, lse, keep_ratio: float, budget: int, idx, kc, vc, vqc,
+                          gammac, scores, gamma, ws, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    rows = (hq // hkv) * lt
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+    _check("tp_compress_layer_lse", load().tp_compress_layer_lse(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
+        _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
+        keep_ratio, budget,
+        _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
+        _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
+        _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
+        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _ptr(gammac, torch.float32, m, "gammac", nullable=True),
+        _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
 def tp_check_status(ws, stream=None) -> int:
     return int(load().tp_check_status(c_void_p(ws.data_ptr()), ws.numel(), _stream(stream)))
 
@@ -308,7 +336,14 @@ class CompressOutputs:
                               device=device)
 
 
-def compress(p: Problem, q, k, v, keep_ratio: float, budget: int, out: CompressOutputs, stream=None):
-    tp_compress_layer(p, q, k, v, keep_ratio, budget, out.idx, out.kc, out.vc, out.vqc, out.gammac,
-                      out.scores, out.gamma, out.ws, stream)
+def compress(p: Problem, q, k, v, keep_ratio: float, budget: int, out: CompressOutputs, stream=None,
+             lse=None):
+    """One layer through tp_compress_layer, or through tp_compress_layer_lse
+    with the caller's row normalisers `lse`."""
+    if lse is None:
+        tp_compress_layer(p, q, k, v, keep_ratio, budget, out.idx, out.kc, out.vc, out.vqc,
+                          out.gammac, out.scores, out.gamma, out.ws, stream)
+    else:
+        tp_compress_layer_lse(p, q, k, v, lse, keep_ratio, budget, out.idx, out.kc, out.vc, out.vqc,
+                              out.gammac, out.scores, out.gamma, out.ws, stream)
     return out

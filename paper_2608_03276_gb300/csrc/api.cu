@@ -57,7 +57,10 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0 || p->pool_kernel > 33)
     return TP_ERR_UNSUPPORTED_SHAPE;
   if (p->quant_bits != 8) return TP_ERR_UNSUPPORTED_SHAPE;
-  if (p->flags & ~TP_SCORE_KEY_ONLY) return TP_ERR_INVALID_ARG;
+  const uint32_t score_flags = TP_SCORE_KEY_ONLY | TP_SCORE_NORM_ADD | TP_SCORE_HARMONIC;
+  if (p->flags & ~score_flags) return TP_ERR_INVALID_ARG;
+  const uint32_t f = p->flags;
+  if ((f & (f - 1)) != 0) return TP_ERR_INVALID_ARG;  // at most one score flag
   memset(P, 0, sizeof(*P));
   P->hq = p->n_heads_q;
   P->hkv = p->n_heads_kv;
@@ -270,6 +273,12 @@ int run_scoring(const Plan& P, const void* q, const void* k, const void* v, floa
                       reinterpret_cast<int*>(ws + P.ws_status), true, s);
 }
 
+int blend_of(uint32_t flags) {
+  if (flags & TP_SCORE_NORM_ADD) return kBlendNormAdd;
+  if (flags & TP_SCORE_HARMONIC) return kBlendHarmonic;
+  return kBlendProduct;
+}
+
 void fill_select(const Plan& P, char* ws, SelectParams* sp) {
   memset(sp, 0, sizeof(*sp));
   for (int b = 0; b <= P.batch; ++b) sp->off[b] = P.off[b];
@@ -298,6 +307,64 @@ void fill_gather(const Plan& P, GatherParams* gp) {
   gp->n_total = P.n_total;
   gp->cap = P.cap;
   gp->qmax = 127.0f;
+}
+
+// The fused layer.  Without `lse`: two scoring passes (the first also forms
+// the Eq. 2 scales).  With the caller's row normalisers `lse`: one pass over
+// V for the scales, then the key-score pass with those normalisers.
+int compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
+                   const float* lse_in, double keep_ratio, int64_t budget, int32_t* idx, void* kc,
+                   void* vc, int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
+                   size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k || !v || (!idx && P.cap > 0) || !aligned16(q) || !aligned16(k) || !aligned16(v))
+    return TP_ERR_INVALID_ARG;
+  if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
+      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
+    return TP_ERR_INVALID_ARG;
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
+  if (!lse_in) {
+    if ((st = run_scoring(P, q, k, v, g, w, s)) != TP_OK) return st;
+  } else if (P.n_total > 0 && P.grid_x > 0) {
+    if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
+                      127.0f, num_sms(), s) != cudaSuccess)
+      return TP_ERR_CUDA;
+    CUtensorMap tmk, tmq;
+    if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+    if ((st = run_keyscore(P, tmk, tmq, lse_in, reinterpret_cast<float*>(w + P.ws_skey),
+                           reinterpret_cast<int*>(w + P.ws_status), false, s)) != TP_OK)
+      return st;
+  }
+  SelectParams sp;
+  fill_select(P, w, &sp);
+  sp.pool_kernel = p->pool_kernel;
+  sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
+  sp.blend = blend_of(p->flags);
+  sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
+  sp.gamma = g;
+  sp.scores_out = scores;
+  sp.idx = idx;
+  cudaError_t e2 = launch_select(sp, true, s);
+  if (e2 != cudaSuccess) return TP_ERR_CUDA;
+  if (P.cap == 0) return TP_OK;
+  GatherParams gp;
+  fill_gather(P, &gp);
+  gp.k = static_cast<const uint16_t*>(k);
+  gp.v = static_cast<const uint16_t*>(v);
+  gp.gamma = g;
+  gp.idx = idx;
+  gp.kc = static_cast<uint16_t*>(kc);
+  gp.vc = static_cast<uint16_t*>(vc);
+  gp.vqc = vqc;
+  gp.gammac = gammac;
+  return cuda_status(launch_gather(gp, true, s));
 }
 
 }  // namespace
@@ -407,6 +474,7 @@ int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const flo
   fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;
   sp.key_only = key_only ? 1 : 0;
+  sp.blend = blend_of(p->flags);
   sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
   sp.gamma = gamma;
   sp.scores_out = scores;
@@ -510,43 +578,17 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
                       double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
                       int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
                       size_t ws_bytes, void* stream) {
-  Plan P;
-  int st = make_plan(p, keep_ratio, budget, true, &P);
-  if (st != TP_OK) return st;
-  if (!q || !k || !v || (!idx && P.cap > 0) || !aligned16(q) || !aligned16(k) || !aligned16(v))
-    return TP_ERR_INVALID_ARG;
-  if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
-      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
-    return TP_ERR_INVALID_ARG;
-  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
-    return TP_ERR_WORKSPACE;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  char* w = static_cast<char*>(ws);
-  float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
-  if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  if ((st = run_scoring(P, q, k, v, g, w, s)) != TP_OK) return st;
-  SelectParams sp;
-  fill_select(P, w, &sp);
-  sp.pool_kernel = p->pool_kernel;
-  sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
-  sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
-  sp.gamma = g;
-  sp.scores_out = scores;
-  sp.idx = idx;
-  cudaError_t e2 = launch_select(sp, true, s);
-  if (e2 != cudaSuccess) return TP_ERR_CUDA;
-  if (P.cap == 0) return TP_OK;
-  GatherParams gp;
-  fill_gather(P, &gp);
-  gp.k = static_cast<const uint16_t*>(k);
-  gp.v = static_cast<const uint16_t*>(v);
-  gp.gamma = g;
-  gp.idx = idx;
-  gp.kc = static_cast<uint16_t*>(kc);
-  gp.vc = static_cast<uint16_t*>(vc);
-  gp.vqc = vqc;
-  gp.gammac = gammac;
-  return cuda_status(launch_gather(gp, true, s));
+  return compress_layer(p, q, k, v, nullptr, keep_ratio, budget, idx, kc, vc, vqc, gammac, scores,
+                        gamma, ws, ws_bytes, stream);
+}
+
+int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, const void* v,
+                          const float* lse, double keep_ratio, int64_t budget, int32_t* idx,
+                          void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
+                          float* gamma, void* ws, size_t ws_bytes, void* stream) {
+  if (!lse) return TP_ERR_INVALID_ARG;
+  return compress_layer(p, q, k, v, lse, keep_ratio, budget, idx, kc, vc, vqc, gammac, scores,
+                        gamma, ws, ws_bytes, stream);
 }
 
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {

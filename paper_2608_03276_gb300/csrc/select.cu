@@ -54,7 +54,29 @@ struct SelectSmem {
   int counts[2];  // (> T, == T) in this CTA's slice
   int scratch[33];
   int result[2];
+  float norm2[2];  // this CTA's sums of squares of pooled key scores and scales
+  float inv_norm[2];
 };
+
+// Sum of v over the block in a fixed order (warp trees, then warp totals).
+__device__ __forceinline__ float block_sum_f(float v, float* warp_part) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) warp_part[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+  if (warp == 0) {
+    t = lane < static_cast<int>(blockDim.x >> 5) ? warp_part[lane] : 0.f;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) warp_part[32] = t;
+  }
+  __syncthreads();
+  t = warp_part[32];
+  __syncthreads();
+  return t;
+}
 
 // Address of `local` (a shared-memory object of this CTA) in cluster CTA `rank`.
 __device__ __forceinline__ uint32_t dsmem(const void* local, int rank) {
@@ -163,64 +185,111 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   __syncthreads();
 
   // A: keys of the slice (scores formed here in the fused path) + digit-1 histogram,
-  // in sub-slices of kSliceKeys tokens whose key scores are staged with their halo
+  // in sub-slices of kSliceKeys tokens whose key scores are staged with their halo.
+  // The normalised-add blend first sweeps the slice for the sums of squares of
+  // the pooled key scores and of the scales, reduced over the cluster.
   const int half = p.pool_kernel / 2;
   const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
-  for (int c0 = s0; c0 < s1; c0 += kSliceKeys) {
-    const int c1 = min(c0 + kSliceKeys, s1);
-    // this thread's first round of scale (or score) loads go out before the
-    // key-score strip is staged, so the two global round trips overlap
-    float sv[8];
-    auto load_round = [&](int base) {
+  const bool fused = !p.scores_in;
+  float inv_na = 0.f, inv_nb = 0.f;
+  auto sweep = [&](bool norms_only) {
+    float sa = 0.f, sb = 0.f;
+    for (int c0 = s0; c0 < s1; c0 += kSliceKeys) {
+      const int c1 = min(c0 + kSliceKeys, s1);
+      // this thread's first round of scale (or score) loads go out before the
+      // key-score strip is staged, so the two global round trips overlap
+      float sv[8];
+      auto load_round = [&](int base) {
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int i = base + u * kThreads + threadIdx.x;
-        sv[u] = 0.f;
-        if (i < c1) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
-                                        : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
-      }
-    };
-    load_round(c0);
-    if (!p.scores_in) {
-      const float* sk = p.skey + row;
-      const int len = c1 - c0 + 2 * half;
-      for (int j0 = threadIdx.x; j0 < len; j0 += 8 * kThreads) {
-        float v[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {  // eight independent loads in flight
-          const int j = j0 + u * kThreads, i = c0 - half + j;
-          v[u] = (j < len && i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
+        for (int u = 0; u < 8; ++u) {
+          const int i = base + u * kThreads + threadIdx.x;
+          sv[u] = 0.f;
+          if (i < c1) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
+                                          : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
         }
+      };
+      load_round(c0);
+      if (fused) {
+        const float* sk = p.skey + row;
+        const int len = c1 - c0 + 2 * half;
+        for (int j0 = threadIdx.x; j0 < len; j0 += 8 * kThreads) {
+          float v[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          if (j0 + u * kThreads < len) sm.strip[j0 + u * kThreads] = v[u];
+          for (int u = 0; u < 8; ++u) {  // eight independent loads in flight
+            const int j = j0 + u * kThreads, i = c0 - half + j;
+            v[u] = (j < len && i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            if (j0 + u * kThreads < len) sm.strip[j0 + u * kThreads] = v[u];
+        }
+        __syncthreads();
+      }
+      for (int base = c0; base < c1; base += 8 * kThreads) {
+        if (base != c0) load_round(base);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int i = base + u * kThreads + threadIdx.x;
+          const bool live = i < c1;
+          uint32_t key = 0;
+          if (live) {
+            float sc = sv[u];
+            if (fused) {
+              float acc = 0.f;
+              const float* w = sm.strip + (i - c0);
+              for (int o = 0; o <= 2 * half; ++o) acc += w[o];
+              const float a = acc * inv_k, g = sv[u];
+              if (norms_only) {
+                sa += a * a;
+                sb += g * g;
+                continue;
+              }
+              if (p.key_only) {
+                sc = a;
+              } else if (p.blend == kBlendNormAdd) {
+                sc = a * inv_na + g * inv_nb;
+              } else if (p.blend == kBlendHarmonic) {
+                const float den = a + g;
+                sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
+              } else {
+                sc = a * g;
+              }
+              if (p.scores_out) p.scores_out[row + i] = sc;
+            }
+            key = score_key(sc);
+            keys_base[i - kofs] = key;
+          }
+          if (!p.scores_only && live) atomicAdd(&sm.hist1[key >> 21], 1);
+        }
       }
       __syncthreads();
     }
-    for (int base = c0; base < c1; base += 8 * kThreads) {
-      if (base != c0) load_round(base);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int i = base + u * kThreads + threadIdx.x;
-        const bool live = i < c1;
-        uint32_t key = 0;
-        if (live) {
-          float sc = sv[u];
-          if (!p.scores_in) {
-            float acc = 0.f;
-            const float* w = sm.strip + (i - c0);
-            for (int o = 0; o <= 2 * half; ++o) acc += w[o];
-            sc = p.key_only ? acc * inv_k : (acc * inv_k) * sv[u];
-            if (p.scores_out) p.scores_out[row + i] = sc;
-          }
-          key = score_key(sc);
-          keys_base[i - kofs] = key;
-        }
-        if (!p.scores_only && live) atomicAdd(&sm.hist1[key >> 21], 1);
+    if (norms_only) {
+      sa = block_sum_f(sa, reinterpret_cast<float*>(sm.scratch));
+      sb = block_sum_f(sb, reinterpret_cast<float*>(sm.scratch));
+      if (threadIdx.x == 0) {
+        sm.norm2[0] = sa;
+        sm.norm2[1] = sb;
       }
     }
-    __syncthreads();
+  };
+  if (fused && !p.key_only && p.blend == kBlendNormAdd) {
+    sweep(true);
+    cluster.sync();  // every CTA's sums are in place
+    if (threadIdx.x == 0) {
+      float ta = 0.f, tb = 0.f;  // summed in rank order: the same on every CTA
+      for (int r = 0; r < CL; ++r) {
+        ta += __int_as_float(ld_dsmem(dsmem(&sm.norm2[0], r)));
+        tb += __int_as_float(ld_dsmem(dsmem(&sm.norm2[1], r)));
+      }
+      sm.inv_norm[0] = ta > 0.f ? __fdiv_rn(1.f, sqrtf(ta)) : 0.f;
+      sm.inv_norm[1] = tb > 0.f ? __fdiv_rn(1.f, sqrtf(tb)) : 0.f;
+    }
+    cluster.sync();  // no CTA moves on (or leaves) while another still reads its sums
+    inv_na = sm.inv_norm[0];
+    inv_nb = sm.inv_norm[1];
   }
+  sweep(false);
   if (p.scores_only) return;  // no cluster-wide exchange follows
 
   const int64_t unit_slot0 = static_cast<int64_t>(unit) * p.cap;

@@ -69,6 +69,13 @@ struct KeyScoreParams {
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
 
+// Blends of the pooled key score a and the scale g (Eq. 3 and the Sec. 6
+// aggregation ablation): a * g; a / ||a||_2 + g / ||g||_2 per (document,
+// head); 2 a g / (a + g).
+constexpr int kBlendProduct = 0;
+constexpr int kBlendNormAdd = 1;
+constexpr int kBlendHarmonic = 2;
+
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
   int32_t kept[kMaxBatch];   // k_b per document
@@ -79,6 +86,7 @@ struct SelectParams {
   int64_t cap;
   int pool_kernel;           // >= 1, odd
   int key_only;
+  int blend;                 // kBlendProduct (Eq. 3), kBlendNormAdd or kBlendHarmonic
   int scores_only;           // form the scores (and keys) and stop
   const float* scores_in;    // combined scores (tp_select) or null
   const float* skey;         // unpooled key scores (fused path) or null

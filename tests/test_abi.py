@@ -29,7 +29,7 @@ def declared_symbols():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_symbols()
-    assert len(names) == 13, names
+    assert len(names) == 14, names
     assert sorted(lib.EXPORTS) == names
     cdll = lib.load()
     for n in names:
@@ -77,11 +77,21 @@ def test_rejects_bad_offsets(lib):
     assert lib.tp_kept_capacity(_prob(lib, list(range(0, 258))), 0.5, -1) == -1
 
 
+def test_score_flags(lib):
+    for f in (0, lib.TP_SCORE_KEY_ONLY, lib.TP_SCORE_NORM_ADD, lib.TP_SCORE_HARMONIC):
+        assert lib.tp_kept_capacity(_prob(lib, [0, 100], flags=f), 0.5, -1) == 50
+    for f in (lib.TP_SCORE_NORM_ADD | lib.TP_SCORE_HARMONIC, lib.TP_SCORE_KEY_ONLY | lib.TP_SCORE_NORM_ADD,
+              0x8, 0x100):
+        assert lib.tp_kept_capacity(_prob(lib, [0, 100], flags=f), 0.5, -1) == -1
+
+
 def test_null_pointers_rejected_before_any_launch(lib):
     cdll = lib.load()
     p = _prob(lib, [0, 100])
     assert cdll.tp_quantize_v(p.ref(), None, None, None, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_compress_layer(p.ref(), None, None, None, 0.5, -1, None, None, None, None, None,
                                   None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_compress_layer_lse(p.ref(), None, None, None, None, 0.5, -1, None, None, None, None,
+                                      None, None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_select(p.ref(), None, 0.5, -1, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_status_string(-5) == b"device-side wait timed out"

@@ -1,0 +1,115 @@
+"""Scoring variants through the C ABI, against the oracle.
+
+- The aggregation ablation's blends (Sec. 6): normalised add and harmonic
+  mean (TP_SCORE_NORM_ADD, TP_SCORE_HARMONIC), through the fused layer and
+  through tp_guide_scores.
+- Single-pass scoring with the caller's row normalisers
+  (tp_compress_layer_lse): with the context-only normaliser it must reproduce
+  the two-pass result; with a normaliser that also counts extra guide-prefix
+  mass per row (the literal prefill normaliser of Sec. 3.2) it must follow
+  the oracle given the same normalisers.
+"""
+import math
+
+import numpy as np
+import pytest
+
+from oracle import taskpress_oracle as O
+from paper_2608_03276_gb300 import synth
+from tests import parity
+from tests.test_gpu_parity import SMALL, _check_layer, _oracle, _problem, _run_compress
+
+pytestmark = pytest.mark.gpu
+
+BLENDS = {"normadd": "TP_SCORE_NORM_ADD", "harmonic": "TP_SCORE_HARMONIC"}
+
+
+@pytest.mark.parametrize("mode", sorted(BLENDS))
+@pytest.mark.parametrize("name", ["c1-tiny-2k", "c2-llama-4133", "c5-ragged"])
+def test_blend_fused_layer(cuda_lib, name, mode):
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    out = _run_compress(binding, w, x, flags=getattr(binding, BLENDS[mode]))
+    ref = _oracle(w, x, combine_mode=mode)
+    _check_layer(w, x, out, ref)
+
+
+@pytest.mark.parametrize("mode", sorted(BLENDS))
+def test_blend_guide_scores(cuda_lib, mode):
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL["c4-gqa7-3001"]
+    x = synth.make_layer(w)
+    ref = _oracle(w, x, combine_mode=mode)
+    p = _problem(binding, w, x.doc_offsets, flags=getattr(binding, BLENDS[mode]))
+    s = torch.empty((w.n_heads_kv, p.n_total), dtype=torch.float32, device="cuda")
+    ws = torch.empty(binding.tp_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    binding.tp_guide_scores(p, parity.to_device_bf16(x.q), parity.to_device_bf16(x.k),
+                            torch.tensor(ref["gamma"], device="cuda"), s, ws)
+    sc = s.cpu().numpy()
+    for b in range(len(x.doc_offsets) - 1):
+        lo, hi = x.doc_offsets[b], x.doc_offsets[b + 1]
+        for h in range(w.n_heads_kv):
+            parity.assert_scores_close(sc[h, lo:hi], ref["scores"][(b, h)], f"{mode} {b},{h}")
+
+
+def _context_lse(w, x):
+    """Each guide row's context-only normaliser [batch, H_kv, G*L_t], fp32."""
+    q, k = O.decode_bf16(x.q), O.decode_bf16(x.k)
+    g = w.n_heads_q // w.n_heads_kv
+    sigma = 1.0 / math.sqrt(w.head_dim)
+    offs = x.doc_offsets
+    out = np.zeros((len(offs) - 1, w.n_heads_kv, g * w.guide_len), np.float32)
+    for b in range(len(offs) - 1):
+        lo, hi = int(offs[b]), int(offs[b + 1])
+        if hi == lo:
+            continue
+        for h in range(w.n_heads_kv):
+            rows = q[b, h * g:(h + 1) * g].reshape(g * w.guide_len, w.head_dim)
+            out[b, h] = O.guide_lse(rows, k[h, lo:hi], sigma)
+    return out
+
+
+def _run_lse(binding, w, x, lse):
+    import torch
+    p = _problem(binding, w, x.doc_offsets)
+    out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+    binding.compress(p, parity.to_device_bf16(x.q), parity.to_device_bf16(x.k),
+                     parity.to_device_bf16(x.v), w.keep_ratio, w.budget, out,
+                     lse=torch.tensor(lse, device="cuda"))
+    assert binding.tp_check_status(out.ws) == 0
+    return out
+
+
+@pytest.mark.parametrize("name", ["c2-llama-4133", "c3-guide128-2053", "c5-ragged"])
+def test_caller_lse_context_normaliser(cuda_lib, name):
+    """The context-only normaliser supplied by the caller reproduces the
+    two-pass layer (the oracle's default)."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    lse = _context_lse(w, x)
+    out = _run_lse(binding, w, x, lse)
+    ref = _oracle(w, x, lse=lse.astype(np.float64))
+    _check_layer(w, x, out, ref)
+    ref2 = _oracle(w, x)
+    for key in ref2["scores"]:
+        parity.assert_scores_close(ref["scores"][key], ref2["scores"][key], f"oracle {key}")
+
+
+@pytest.mark.parametrize("name", ["c2-llama-4133", "c4-gqa7-3001"])
+def test_caller_lse_literal_normaliser(cuda_lib, name):
+    """A normaliser that also counts guide-prefix mass (different per row, up
+    to e^3 times the context mass) changes the scores and the kept sets; the
+    GPU follows the oracle given the same normalisers."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    lse_ctx = _context_lse(w, x)
+    rng = np.random.Generator(np.random.PCG64(9))
+    extra = rng.uniform(-2.0, 3.0, lse_ctx.shape)  # log of the prefix mass relative to the context
+    lse = np.logaddexp(lse_ctx.astype(np.float64), lse_ctx + extra).astype(np.float32)
+    out = _run_lse(binding, w, x, lse)
+    ref = _oracle(w, x, lse=lse.astype(np.float64))
+    _check_layer(w, x, out, ref)
