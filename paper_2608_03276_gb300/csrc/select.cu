@@ -155,7 +155,10 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   return d;
 }
 
-template <int CL>
+// CL: CTAs per (document, head) cluster.  BLEND: how the fused path combines
+// the pooled key score with the scale (a compile-time choice, so the product
+// kernel's per-token loop carries nothing for the other blends).
+template <int CL, int BLEND>
 __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_constant__ SelectParams p) {
   extern __shared__ uint8_t smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
@@ -246,9 +249,9 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
               }
               if (p.key_only) {
                 sc = a;
-              } else if (p.blend == kBlendNormAdd) {
+              } else if constexpr (BLEND == kBlendNormAdd) {
                 sc = a * inv_na + g * inv_nb;
-              } else if (p.blend == kBlendHarmonic) {
+              } else if constexpr (BLEND == kBlendHarmonic) {
                 const float den = a + g;
                 sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
               } else {
@@ -273,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
       }
     }
   };
-  if (fused && !p.key_only && p.blend == kBlendNormAdd) {
+  if (BLEND == kBlendNormAdd && fused && !p.key_only) {
     sweep(true);
     cluster.sync();  // every CTA's sums are in place
     if (threadIdx.x == 0) {
@@ -399,9 +402,11 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 
 size_t select_smem_bytes() { return sizeof(SelectSmem); }
 
-template <int CL>
+template <int CL, int BLEND>
 cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool dependent,
-                            cudaStream_t s) {
+                            cudaStream_t s, int slot) {
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND>), slot);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(CL, units);
   cfg.blockDim = dim3(kThreads);
@@ -416,7 +421,17 @@ cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool 
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL>, p);
+  return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL, BLEND>, p);
+}
+
+template <int CL>
+cudaError_t launch_select_blend(const SelectParams& p, int units, size_t smem, bool dependent,
+                                cudaStream_t s, int slot0) {
+  switch (p.blend) {
+    case kBlendNormAdd: return launch_select_t<CL, kBlendNormAdd>(p, units, smem, dependent, s, slot0 + 1);
+    case kBlendHarmonic: return launch_select_t<CL, kBlendHarmonic>(p, units, smem, dependent, s, slot0 + 2);
+    default: return launch_select_t<CL, kBlendProduct>(p, units, smem, dependent, s, slot0);
+  }
 }
 
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s) {
@@ -429,14 +444,10 @@ cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s)
   int64_t n_max = 0;
   for (int b = 0; b < p.batch; ++b) n_max = p.off[b + 1] - p.off[b] > n_max ? p.off[b + 1] - p.off[b] : n_max;
   // Fewer, larger slices when eight CTAs per unit would need more than one wave.
-  if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys) {
-    cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<4>), 11);
-    if (e != cudaSuccess) return e;
-    return launch_select_t<4>(p, units, smem, dependent, s);
-  }
-  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<8>), 0);
-  if (e != cudaSuccess) return e;
-  return launch_select_t<8>(p, units, smem, dependent, s);
+  // shared-memory attribute slots: 12..14 for four-CTA clusters, 15..17 for eight
+  if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys)
+    return launch_select_blend<4>(p, units, smem, dependent, s, 12);
+  return launch_select_blend<8>(p, units, smem, dependent, s, 15);
 }
 
 }  // namespace tp
