@@ -55,7 +55,7 @@ extern "C" {
 
 /* Flags (tp_problem.flags). */
 #define TP_SCORE_KEY_ONLY 0x1u /* s_i = pooled key score only (Sec. 4.3.1 ablation) */
-/* The other blends of the Sec. 6 aggregation ablation (at most one flag):
+/* The other blends of the Sec. 4.4 aggregation ablation (at most one flag):
  *   TP_SCORE_NORM_ADD  s_i = s_key_i / ||s_key||_2 + gamma_i / ||gamma||_2, the
  *                      L2 norms taken over one document and KV head (a zero
  *                      norm drops its term);

@@ -13,9 +13,11 @@ reach the same integers.
 
 Readings of the paper used here (where it is silent or ambiguous):
 
-* softmax normaliser - each guide row is normalised over the context keys only
-  (the attention block the method slices out of the prefill map, Sec. 3.2;
-  guide keys are never given to the compression step);
+* softmax normaliser - by default each guide row is normalised over the
+  context keys only (the attention block the method slices out of the prefill
+  map, Sec. 3.2, renormalised); given the guide's keys, the literal row of
+  that causal map, context plus guide prefix (guide_lse_literal); or a
+  normaliser the caller supplies;
 * reduction - Eq. 1 sums over the L_t guide tokens; the G query heads sharing
   a KV head are averaged (the paper budgets per KV head, Sec. 4 "Eviction");
 * pooling - the Eq. 1 window has 2*floor(K/2)+1 terms, so K must be odd; terms
@@ -150,6 +152,30 @@ def key_scores_given_lse(q_group: np.ndarray, k_ctx: np.ndarray, sigma: float,
     return np.exp(x - np.asarray(lse_rows, dtype=np.float64)[:, None]).sum(axis=0) / g
 
 
+def guide_lse_literal(q_group: np.ndarray, k_ctx: np.ndarray, k_guide: np.ndarray,
+                      sigma: float) -> np.ndarray:
+    """Each guide row's normaliser over its whole causal row of the prefill map.
+
+    The prefill attends over the context followed by the guide, causally, so
+    guide token j sees every context key and the guide keys 0..j (itself
+    included).  A is sliced out of that map (Sec. 3.2), so row r = (g, j) of
+    the stacked group (query head-major, then guide token) is normalised by
+      lse[r] = log( sum_i exp(sigma q_r . k_i) + sum_{j' <= j} exp(sigma q_r . kg_j') ).
+    q_group [G, L_t, d], k_ctx [n, d], k_guide [L_t, d] float64 (post-RoPE).
+    Each row is written out as its own logit vector: context part, then the
+    guide prefix; then max, exp, sum, log.
+    """
+    g, lt, d = q_group.shape
+    out = np.empty(g * lt)
+    for gi in range(g):
+        for j in range(lt):
+            qr = q_group[gi, j]
+            x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma
+            m = np.max(x)
+            out[gi * lt + j] = m + math.log(float(np.sum(np.exp(x - m))))
+    return out
+
+
 def pool(s: np.ndarray, kernel: int) -> np.ndarray:
     """Eq. 1's 1-D average pooling with window K (odd), zero outside [0, n)."""
     if kernel < 1 or kernel % 2 == 0:
@@ -171,13 +197,13 @@ def combine(pooled: np.ndarray, gamma: np.ndarray, key_only: bool = False,
             mode: str = "mul") -> np.ndarray:
     """Eq. 3: s_i = s_key_i * s_value_i with s_value_i = gamma_i (Sec. 3.3-3.4).
 
-    The two other blends of the aggregation ablation (Sec. 6, "Score
+    The two other blends of the aggregation ablation (Sec. 4.4, "Score
     aggregation strategy"), over one (document, head):
       normadd   s_key_i / ||s_key||_2 + s_value_i / ||s_value||_2, a term whose
                 norm is 0 contributing 0;
       harmonic  2 s_key_i s_value_i / (s_key_i + s_value_i), 0 where the sum
                 is 0 (the printed formula has ',' for '+').
-    key_only drops s_value (Sec. 6, the key-only row of the ablation).
+    key_only drops s_value (Sec. 4.3.1, the key-only row of Tab. 8).
     """
     if key_only:
         return pooled.copy()
@@ -213,13 +239,15 @@ def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
                    n_heads_q: int, n_heads_kv: int, keep_ratio: float = 0.25,
                    fixed_budget: int = -1, pool_kernel: int = 5, quant_bits: int = 8,
                    softmax_scale: float = 0.0, key_only: bool = False, combine_mode: str = "mul",
-                   lse=None, heads: Optional[Sequence[int]] = None,
+                   lse=None, k_guide_bits=None, heads: Optional[Sequence[int]] = None,
                    docs: Optional[Sequence[int]] = None):
     """The whole compression of one layer (Sec. 3.1-3.4 with Sec. 4 budgets).
 
     q_bits [batch, H_q, L_t, d], k_bits / v_bits [H_kv, N_total, d] (bf16 bits),
     doc_offsets [batch+1].  ``lse`` [batch, H_kv, G*L_t] (natural log), when
     given, replaces each guide row's normaliser (key_scores_given_lse);
+    ``k_guide_bits`` [batch, H_kv, L_t, d] (bf16 bits), when given, gives each
+    row the literal normaliser of guide_lse_literal instead (not with ``lse``);
     ``combine_mode`` selects the blend of ``combine``.  Returns a dict:
       gamma  [H_kv, N_total] float32, vq [H_kv, N_total, d] int8,
       scores {(b, h): float64 [n_b]}  combined scores s_i,
@@ -228,8 +256,11 @@ def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
       k      {b: k_b}.
     ``heads`` / ``docs`` restrict the (expensive) scoring to a subset.
     """
+    if lse is not None and k_guide_bits is not None:
+        raise ValueError("give either lse or k_guide_bits")
     q = decode_bf16(q_bits)
     k_all = decode_bf16(k_bits)
+    kg = None if k_guide_bits is None else decode_bf16(k_guide_bits)
     batch, hq, lt, d = q.shape
     g = n_heads_q // n_heads_kv
     sigma = softmax_scale if softmax_scale > 0 else 1.0 / math.sqrt(d)
@@ -247,6 +278,9 @@ def compress_layer(q_bits, k_bits, v_bits, doc_offsets: Sequence[int], *,
             # an empty document has no context tokens: nothing to score or keep
             if n == 0:
                 s_key = np.zeros(0)
+            elif kg is not None:
+                lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, h], sigma)
+                s_key = key_scores_given_lse(qg, k_all[h, lo:hi], sigma, lse_rows)
             elif lse is None:
                 s_key = key_scores(qg, k_all[h, lo:hi], sigma)
             else:

@@ -69,7 +69,7 @@ struct KeyScoreParams {
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
 
-// Blends of the pooled key score a and the scale g (Eq. 3 and the Sec. 6
+// Blends of the pooled key score a and the scale g (Eq. 3 and the Sec. 4.4
 // aggregation ablation): a * g; a / ||a||_2 + g / ||g||_2 per (document,
 // head); 2 a g / (a + g).
 constexpr int kBlendProduct = 0;

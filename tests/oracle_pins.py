@@ -259,8 +259,80 @@ def pin_key_scores_given_lse(O):
     assert np.allclose(b, a * math.exp(-0.75), rtol=1e-12, atol=0)
 
 
+def pin_literal_lse_closed_form(O):
+    """Q = 0: every logit is 0, so row r = (g, j) of the causal prefill map has
+    n context terms and j + 1 guide terms: lse_r = log(n + j + 1), rows ordered
+    query head-major (Sec. 3.2).  With no context keys only the prefix is left."""
+    g, lt, d, n = 3, 4, 8, 11
+    q = np.zeros((g, lt, d))
+    got = O.guide_lse_literal(q, _rand(1, (n, d)), _rand(2, (lt, d)), 0.4)
+    want = np.array([math.log(n + j + 1) for _ in range(g) for j in range(lt)])
+    assert np.allclose(got, want, rtol=1e-14, atol=0)
+    got0 = O.guide_lse_literal(q, np.zeros((0, d)), _rand(2, (lt, d)), 0.4)
+    assert np.allclose(got0, [math.log(j + 1) for _ in range(g) for j in range(lt)], rtol=1e-14, atol=1e-15)
+
+
+def pin_literal_lse_causal(O):
+    """One scalar channel: q_r = a_g e1, context keys +-e1, guide keys c_j e1.
+    Row (g, j) sums exp(+-sigma a_g) and exp(sigma a_g c_j') for j' <= j, written
+    out term by term; a huge later guide key leaves earlier rows unchanged."""
+    g, lt, d, sigma = 2, 3, 4, 0.5
+    a = [0.7, -1.3]
+    c = [2.0, -0.5, 30.0]
+    q = np.zeros((g, lt, d))
+    for gi in range(g):
+        q[gi, :, 0] = a[gi]
+    k = np.zeros((2, d))
+    k[0, 0], k[1, 0] = 1.0, -1.0
+    kg = np.zeros((lt, d))
+    kg[:, 0] = c
+    got = O.guide_lse_literal(q, k, kg, sigma)
+    for gi in range(g):
+        for j in range(lt):
+            z = math.exp(sigma * a[gi]) + math.exp(-sigma * a[gi])
+            for jj in range(j + 1):
+                z += math.exp(sigma * a[gi] * c[jj])
+            assert math.isclose(got[gi * lt + j], math.log(z), rel_tol=1e-13), (gi, j)
+
+
+def pin_literal_key_scores_brute_force(O):
+    """compress_layer with guide keys against a brute-force literal prefill row:
+    for every (document, head, g, j), the causal row over [context, guide 0..j]
+    is built with explicit loops, exponentiated and normalised; its context
+    part, summed over rows and averaged over the group, is the key score.
+    Two documents and two KV heads with distinct guide keys pin the [b, h]
+    indexing of the guide keys."""
+    batch, hkv, g, lt, d = 2, 2, 2, 3, 8
+    offs = [0, 5, 12]
+    rng = np.random.Generator(np.random.PCG64(31))
+    q = rng.integers(-4, 5, (batch, hkv * g, lt, d)).astype(np.float32) / 4
+    k = rng.integers(-4, 5, (hkv, offs[-1], d)).astype(np.float32) / 4
+    v = rng.integers(-4, 5, (hkv, offs[-1], d)).astype(np.float32) / 4
+    kg = rng.integers(-8, 9, (batch, hkv, lt, d)).astype(np.float32) / 4
+    sigma = 0.5
+    out = O.compress_layer(exact_bf16(q), exact_bf16(k), exact_bf16(v), offs, n_heads_q=hkv * g,
+                           n_heads_kv=hkv, keep_ratio=0.5, softmax_scale=sigma,
+                           k_guide_bits=exact_bf16(kg))
+    for b in range(batch):
+        lo, hi = offs[b], offs[b + 1]
+        for h in range(hkv):
+            s = [0.0] * (hi - lo)
+            for gi in range(g):
+                for j in range(lt):
+                    qr = [float(x) for x in q[b, h * g + gi, j]]
+                    ctx = [math.exp(sigma * sum(qr[c] * float(k[h, i, c]) for c in range(d)))
+                           for i in range(lo, hi)]
+                    pre = [math.exp(sigma * sum(qr[c] * float(kg[b, h, jj, c]) for c in range(d)))
+                           for jj in range(j + 1)]
+                    z = sum(ctx) + sum(pre)
+                    for i in range(hi - lo):
+                        s[i] += ctx[i] / z
+            want = np.array(s) / g
+            assert np.allclose(out["key"][(b, h)], want, rtol=1e-12, atol=0), (b, h)
+
+
 def pin_combine_normadd(O):
-    """Normalised add (Sec. 6 aggregation ablation): L2 norms over the vector.
+    """Normalised add (Sec. 4.4 aggregation ablation): L2 norms over the vector.
     (3, 4) and (5, 12) have norms 5 and 13; each term is scale-free; a zero
     vector contributes nothing."""
     a, g = np.array([3.0, 4.0]), np.array([5.0, 12.0])

@@ -1,6 +1,6 @@
 """Scoring variants through the C ABI, against the oracle.
 
-- The aggregation ablation's blends (Sec. 6): normalised add and harmonic
+- The aggregation ablation's blends (Sec. 4.4): normalised add and harmonic
   mean (TP_SCORE_NORM_ADD, TP_SCORE_HARMONIC), through the fused layer and
   through tp_guide_scores.
 - Single-pass scoring with the caller's row normalisers

@@ -40,6 +40,12 @@ MUTATIONS = {
     "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma)\n", "s_key = key_scores(qg, k_all[h, 0:n], sigma)\n"),
     "given normaliser added": ("np.exp(x - np.asarray(lse_rows", "np.exp(x + np.asarray(lse_rows"),
     "given-normaliser scores not averaged over G": ("[:, None]).sum(axis=0) / g", "[:, None]).sum(axis=0)"),
+    "guide prefix excludes the token itself": ("x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma", "x = np.concatenate([k_ctx @ qr, k_guide[:j] @ qr]) * sigma"),
+    "whole guide, no causal mask": ("x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma", "x = np.concatenate([k_ctx @ qr, k_guide @ qr]) * sigma"),
+    "literal normaliser drops the context": ("x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma", "x = k_guide[: j + 1] @ qr * sigma"),
+    "literal rows token-major": ("out[gi * lt + j] = m", "out[j * g + gi] = m"),
+    "guide keys of document 0": ("lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, h], sigma)", "lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[0, h], sigma)"),
+    "guide keys of head 0": ("lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, h], sigma)", "lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, 0], sigma)"),
     "normalised add with L1 norms": ("na, nb = math.sqrt(float(np.sum(a * a))), math.sqrt(float(np.sum(b * b)))", "na, nb = float(np.sum(np.abs(a))), float(np.sum(np.abs(b)))"),
     "harmonic mean without the factor 2": ("out[nz] = 2.0 * a[nz] * b[nz] / den[nz]", "out[nz] = a[nz] * b[nz] / den[nz]"),
     "harmonic mean divides by a zero sum": ("nz = den != 0", "nz = den == den"),
