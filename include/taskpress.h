@@ -228,7 +228,7 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
 /*
  * tp_compress_layer with the caller's row normalisers: `lse` ([batch, H_kv, M]
  * fp32, natural log, rows ordered as in tp_guide_lse) replaces the normalising
- * pass, so the scores take one pass over K (Sec. 3.2; survey row f2).  The
+ * pass, so the scores take one pass over K (Sec. 3.2).  The
  * method slices A out of the full prefill attention map; a caller that keeps
  * that attention's per-row log-sum-exp for the guide rows passes it here and
  * gets the paper's literal normaliser, which also counts the guide's own
@@ -240,6 +240,33 @@ int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, con
                           const float* lse, double keep_ratio, int64_t budget, int32_t* idx,
                           void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
                           float* gamma, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * The literal row normaliser (Sec. 3.2).  A is sliced out of the causal
+ * prefill map over the context followed by the guide, so guide row
+ * r = (g, j) (rows ordered as in tp_guide_lse, j = r mod L_t) is normalised
+ * over every context key of its document and over the guide keys 0..j:
+ *   lse[b, h, r] <- log( exp(lse[b, h, r]) + sum_{j' <= j} exp(sigma q_r . kg[b, h, j']) ).
+ * Folds the guide-prefix term into `lse` in place ([batch, H_kv, M] fp32,
+ * natural log, as tp_guide_lse writes it).  For an empty document the input
+ * row is ignored and the output is the prefix term alone.
+ * q: [batch, H_q, L_t, d] bf16; k_guide: [batch, H_kv, L_t, d] bf16, the
+ * guide's post-RoPE keys from the same prefill (16-byte aligned, as q).
+ * The arithmetic is fp32 (exact bf16 products, fp32 sums, expf / logf).
+ */
+int tp_guide_prefix_lse(const tp_problem* p, const void* q, const void* k_guide, float* lse,
+                        void* stream);
+
+/*
+ * tp_compress_layer with the literal normaliser: between the two scoring
+ * passes the guide prefix is folded into each row's normaliser as in
+ * tp_guide_prefix_lse.  k_guide: [batch, H_kv, L_t, d] bf16 device pointer.
+ * Other arguments, outputs and workspace as in tp_compress_layer.
+ */
+int tp_compress_layer_guide(const tp_problem* p, const void* q, const void* k, const void* v,
+                            const void* k_guide, double keep_ratio, int64_t budget, int32_t* idx,
+                            void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
+                            float* gamma, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * Synchronises `stream`, then reads the device status word that the kernels of

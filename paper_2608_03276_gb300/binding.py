@@ -35,7 +35,8 @@ KERNELS_PER_COMPRESS = 4
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
            "tp_select", "tp_compact",
-           "tp_compress_layer", "tp_compress_layer_lse", "tp_check_status", "tp_status_string")
+           "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
+           "tp_compress_layer_guide", "tp_check_status", "tp_status_string")
 
 
 class TpProblem(ctypes.Structure):
@@ -105,6 +106,10 @@ def load(path: Optional[str] = None):
     lib.tp_compress_layer_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
                                           c_double, c_int64, c_void_p, c_void_p, c_void_p, c_void_p,
                                           c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
+    lib.tp_guide_prefix_lse.restype = c_int
+    lib.tp_guide_prefix_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p]
+    lib.tp_compress_layer_guide.restype = c_int
+    lib.tp_compress_layer_guide.argtypes = lib.tp_compress_layer_lse.argtypes
     lib.tp_check_status.restype = c_int
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
@@ -239,6 +244,17 @@ def tp_guide_key_scores(p: Problem, q, k, lse, key_scores, stream=None):
         _ptr(key_scores, torch.float32, hkv * n, "key_scores"), _stream(stream)))
 
 
+def tp_guide_prefix_lse(p: Problem, q, k_guide, lse, stream=None):
+    """Folds the guide's causal prefix into the row normalisers `lse`, in place."""
+    import torch
+    hq, hkv, d, lt = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len
+    rows = (hq // hkv) * lt
+    _check("tp_guide_prefix_lse", load().tp_guide_prefix_lse(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k_guide, torch.bfloat16, p.batch * hkv * lt * d, "k_guide"),
+        _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"), _stream(stream)))
+
+
 def tp_select(p: Problem, scores, keep_ratio: float, budget: int, idx, ws, stream=None):
     import torch
     hkv, n = p.c.n_heads_kv, p.n_total
@@ -307,6 +323,27 @@ def tp_compress_layer_lse(p: Problem, q, k, v, lse, keep_ratio: float, budget: i
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 
+def tp_compress_layer_guide(p: Problem, q, k, v, k_guide, keep_ratio: float, budget: int, idx, kc,
+                            vc, vqc, gammac, scores, gamma, ws, stream=None):
+    import torch
+    hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+    _check("tp_compress_layer_guide", load().tp_compress_layer_guide(
+        p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
+        _ptr(k, torch.bfloat16, hkv * n * d, "k"), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
+        _ptr(k_guide, torch.bfloat16, p.batch * hkv * lt * d, "k_guide"),
+        keep_ratio, budget,
+        _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
+        _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
+        _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
+        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _ptr(gammac, torch.float32, m, "gammac", nullable=True),
+        _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
 def tp_check_status(ws, stream=None) -> int:
     return int(load().tp_check_status(c_void_p(ws.data_ptr()), ws.numel(), _stream(stream)))
 
@@ -337,10 +374,16 @@ class CompressOutputs:
 
 
 def compress(p: Problem, q, k, v, keep_ratio: float, budget: int, out: CompressOutputs, stream=None,
-             lse=None):
-    """One layer through tp_compress_layer, or through tp_compress_layer_lse
-    with the caller's row normalisers `lse`."""
-    if lse is None:
+             lse=None, k_guide=None):
+    """One layer through tp_compress_layer; through tp_compress_layer_lse with
+    the caller's row normalisers `lse`; or through tp_compress_layer_guide with
+    the guide's keys `k_guide` (the literal normaliser)."""
+    if lse is not None and k_guide is not None:
+        raise ValueError("give either lse or k_guide")
+    if k_guide is not None:
+        tp_compress_layer_guide(p, q, k, v, k_guide, keep_ratio, budget, out.idx, out.kc, out.vc,
+                                out.vqc, out.gammac, out.scores, out.gamma, out.ws, stream)
+    elif lse is None:
         tp_compress_layer(p, q, k, v, keep_ratio, budget, out.idx, out.kc, out.vc, out.vqc,
                           out.gammac, out.scores, out.gamma, out.ws, stream)
     else:

@@ -26,7 +26,7 @@ struct Plan {
   int32_t cta[kMaxBatch + 1];
   int stages1, stages2;
   size_t smem1, smem2;
-  float c2, inv_group;
+  float c2, inv_group, sigma;
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
@@ -85,6 +85,7 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->rows_mma = (P->rows + 31) / 32 * 32;
   const double sigma = p->softmax_scale > 0 ? double(p->softmax_scale) : 1.0 / sqrt(double(P->d));
   P->c2 = static_cast<float>(sigma * 1.4426950408889634);
+  P->sigma = static_cast<float>(sigma);
   P->inv_group = 1.0f / static_cast<float>(P->g);
 
   // Key tiles per CTA: the smallest T whose CTA count fits one wave.
@@ -259,16 +260,36 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
       launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
 }
 
+// The guide-prefix fold of the literal normaliser (`lse` in place).
+int run_prefix(const Plan& P, const void* q, const void* k_guide, float* lse, bool dependent,
+               cudaStream_t s) {
+  PrefixParams pp;
+  memset(&pp, 0, sizeof(pp));
+  for (int b = 0; b <= P.batch; ++b) pp.off[b] = P.off[b];
+  pp.q = static_cast<const uint16_t*>(q);
+  pp.k_guide = static_cast<const uint16_t*>(k_guide);
+  pp.lse = lse;
+  pp.batch = P.batch;
+  pp.n_heads_kv = P.hkv;
+  pp.rows = P.rows;
+  pp.guide_len = P.lt;
+  pp.head_dim = P.d;
+  pp.sigma = P.sigma;
+  return cuda_status(launch_prefix(pp, dependent, s));
+}
+
 // Both scoring passes (with the Eq. 2 scales fused into the first when gamma
-// is given); leaves the unpooled key scores in the workspace.
+// is given, and the guide prefix folded into the normalisers between them when
+// k_guide is given); leaves the unpooled key scores in the workspace.
 int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
-                cudaStream_t s) {
+                cudaStream_t s, const void* k_guide = nullptr) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
   int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s);
   if (st != TP_OK) return st;
+  if (k_guide && (st = run_prefix(P, q, k_guide, lse, true, s)) != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), true, s);
 }
@@ -310,12 +331,13 @@ void fill_gather(const Plan& P, GatherParams* gp) {
 }
 
 // The fused layer.  Without `lse`: two scoring passes (the first also forms
-// the Eq. 2 scales).  With the caller's row normalisers `lse`: one pass over
-// V for the scales, then the key-score pass with those normalisers.
+// the Eq. 2 scales), with the guide prefix folded into the normalisers between
+// them when `k_guide` is given.  With the caller's row normalisers `lse`: one
+// pass over V for the scales, then the key-score pass with those normalisers.
 int compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
-                   const float* lse_in, double keep_ratio, int64_t budget, int32_t* idx, void* kc,
-                   void* vc, int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
-                   size_t ws_bytes, void* stream) {
+                   const float* lse_in, const void* k_guide, double keep_ratio, int64_t budget,
+                   int32_t* idx, void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
+                   float* gamma, void* ws, size_t ws_bytes, void* stream) {
   Plan P;
   int st = make_plan(p, keep_ratio, budget, true, &P);
   if (st != TP_OK) return st;
@@ -331,7 +353,7 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
   if (!lse_in) {
-    if ((st = run_scoring(P, q, k, v, g, w, s)) != TP_OK) return st;
+    if ((st = run_scoring(P, q, k, v, g, w, s, k_guide)) != TP_OK) return st;
   } else if (P.n_total > 0 && P.grid_x > 0) {
     if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
                       127.0f, num_sms(), s) != cudaSuccess)
@@ -578,8 +600,8 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
                       double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
                       int8_t* vqc, float* gammac, float* scores, float* gamma, void* ws,
                       size_t ws_bytes, void* stream) {
-  return compress_layer(p, q, k, v, nullptr, keep_ratio, budget, idx, kc, vc, vqc, gammac, scores,
-                        gamma, ws, ws_bytes, stream);
+  return compress_layer(p, q, k, v, nullptr, nullptr, keep_ratio, budget, idx, kc, vc, vqc, gammac,
+                        scores, gamma, ws, ws_bytes, stream);
 }
 
 int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, const void* v,
@@ -587,8 +609,26 @@ int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, con
                           void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
                           float* gamma, void* ws, size_t ws_bytes, void* stream) {
   if (!lse) return TP_ERR_INVALID_ARG;
-  return compress_layer(p, q, k, v, lse, keep_ratio, budget, idx, kc, vc, vqc, gammac, scores,
-                        gamma, ws, ws_bytes, stream);
+  return compress_layer(p, q, k, v, lse, nullptr, keep_ratio, budget, idx, kc, vc, vqc, gammac,
+                        scores, gamma, ws, ws_bytes, stream);
+}
+
+int tp_compress_layer_guide(const tp_problem* p, const void* q, const void* k, const void* v,
+                            const void* k_guide, double keep_ratio, int64_t budget, int32_t* idx,
+                            void* kc, void* vc, int8_t* vqc, float* gammac, float* scores,
+                            float* gamma, void* ws, size_t ws_bytes, void* stream) {
+  if (!k_guide || !aligned16(k_guide)) return TP_ERR_INVALID_ARG;
+  return compress_layer(p, q, k, v, nullptr, k_guide, keep_ratio, budget, idx, kc, vc, vqc, gammac,
+                        scores, gamma, ws, ws_bytes, stream);
+}
+
+int tp_guide_prefix_lse(const tp_problem* p, const void* q, const void* k_guide, float* lse,
+                        void* stream) {
+  Plan P;
+  int st = make_plan(p, 0.0, 0, false, &P);
+  if (st != TP_OK) return st;
+  if (!q || !k_guide || !lse || !aligned16(q) || !aligned16(k_guide)) return TP_ERR_INVALID_ARG;
+  return run_prefix(P, q, k_guide, lse, false, static_cast<cudaStream_t>(stream));
 }
 
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {

@@ -114,6 +114,21 @@ struct GatherParams {
   float* gammac;
 };
 
+// The literal normaliser: the guide's causal prefix folded into each guide
+// row's context normaliser, in place.
+struct PrefixParams {
+  int64_t off[kMaxBatch + 1];  // token offsets (an empty document has no context term)
+  const uint16_t* q;           // guide rows [batch * H_kv, rows, d] bf16
+  const uint16_t* k_guide;     // guide keys [batch * H_kv, L_t, d] bf16
+  float* lse;                  // [batch, H_kv, rows], read and rewritten
+  int batch;
+  int n_heads_kv;
+  int rows;                    // M = G * L_t, row r = (g, j) with j = r mod L_t
+  int guide_len;
+  int head_dim;
+  float sigma;                 // logit scale
+};
+
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int num_sms, cudaStream_t s);
@@ -127,6 +142,7 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             bool dependent, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
+cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once per
 // (kernel slot, device); `slot` names the kernel in a small registry.

@@ -255,6 +255,30 @@ def make_layer_torch(w: Workload, layer: int, device, generator=None):
     return q, k, v
 
 
+#: standard deviation of the synthetic guide keys.  With unit-variance guide
+#: queries and the 1/sqrt(d) scale, a guide-prefix logit is N(0, 4), so each
+#: prefix term has mean mass e^2, against e^(1/2) for a unit-variance context key
+GUIDE_KEY_STD = 2.0
+
+
+def make_guide_keys(w: Workload, layer: int = 0) -> np.ndarray:
+    """Seeded host guide keys [batch, H_kv, L_t, d] (bf16 bits): the post-RoPE
+    keys of the guide tokens themselves, N(0, GUIDE_KEY_STD^2)."""
+    rng = np.random.Generator(np.random.PCG64(w.seed + layer * 1000003 + 424243))
+    x = rng.standard_normal((w.batch, w.n_heads_kv, w.guide_len, w.head_dim), dtype=np.float32)
+    return f32_to_bf16_bits(x * np.float32(GUIDE_KEY_STD))
+
+
+def make_guide_keys_torch(w: Workload, layer: int, device):
+    """The guide-key recipe drawn with torch on ``device`` (bf16)."""
+    import torch
+
+    gen = torch.Generator(device=device)
+    gen.manual_seed(w.seed + layer * 1000003 + 424243)
+    x = torch.randn((w.batch, w.n_heads_kv, w.guide_len, w.head_dim), generator=gen, device=device)
+    return (x * GUIDE_KEY_STD).to(torch.bfloat16).contiguous()
+
+
 def small_variant(w: Workload, doc_lens: Sequence[int], layers: int = 1) -> Workload:
     """The same recipe at oracle-friendly sizes (spans shrink to fit)."""
     n_spans, span_len = w.spans

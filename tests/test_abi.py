@@ -29,7 +29,7 @@ def declared_symbols():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_symbols()
-    assert len(names) == 14, names
+    assert len(names) == 16, names
     assert sorted(lib.EXPORTS) == names
     cdll = lib.load()
     for n in names:
@@ -93,5 +93,8 @@ def test_null_pointers_rejected_before_any_launch(lib):
                                   None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_compress_layer_lse(p.ref(), None, None, None, None, 0.5, -1, None, None, None, None,
                                       None, None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_compress_layer_guide(p.ref(), None, None, None, None, 0.5, -1, None, None, None,
+                                        None, None, None, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_guide_prefix_lse(p.ref(), None, None, None, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_select(p.ref(), None, 0.5, -1, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_status_string(-5) == b"device-side wait timed out"

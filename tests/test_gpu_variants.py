@@ -113,3 +113,66 @@ def test_caller_lse_literal_normaliser(cuda_lib, name):
     out = _run_lse(binding, w, x, lse)
     ref = _oracle(w, x, lse=lse.astype(np.float64))
     _check_layer(w, x, out, ref)
+
+
+# ---------------------------------------------------------------------------
+# The literal normaliser: guide prefix folded in (tp_guide_prefix_lse,
+# tp_compress_layer_guide)
+# ---------------------------------------------------------------------------
+def _literal_lse(w, x, kg_bits):
+    q, k, kg = O.decode_bf16(x.q), O.decode_bf16(x.k), O.decode_bf16(kg_bits)
+    g = w.n_heads_q // w.n_heads_kv
+    sigma = 1.0 / math.sqrt(w.head_dim)
+    offs = x.doc_offsets
+    out = np.zeros((len(offs) - 1, w.n_heads_kv, g * w.guide_len))
+    for b in range(len(offs) - 1):
+        lo, hi = int(offs[b]), int(offs[b + 1])
+        for h in range(w.n_heads_kv):
+            out[b, h] = O.guide_lse_literal(q[b, h * g:(h + 1) * g], k[h, lo:hi], kg[b, h], sigma)
+    return out
+
+
+PREFIX_CASES = {
+    "c1-tiny-2k": SMALL["c1-tiny-2k"],
+    "c4-gqa7-3001": SMALL["c4-gqa7-3001"],
+    "ragged-empty": synth.small_variant(synth.WORKLOADS[5], [300, 0, 7, 129, 1]).with_(budget=50),
+    "guide-129": synth.small_variant(synth.WORKLOADS[2], [515]).with_(guide_len=129, n_heads_q=18,
+                                                                      n_heads_kv=6),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PREFIX_CASES))
+def test_guide_prefix_fold(cuda_lib, name):
+    """The fold alone, fed the oracle's context normalisers (fp32): each row
+    must equal the oracle's literal normaliser to fp32 accuracy.  Short
+    documents make one dropped or extra guide term visible (> 1e-2)."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = PREFIX_CASES[name]
+    x = synth.make_layer(w)
+    kg = synth.make_guide_keys(w)
+    p = _problem(binding, w, x.doc_offsets)
+    lse = torch.tensor(_context_lse(w, x), device="cuda")
+    binding.tp_guide_prefix_lse(p, parity.to_device_bf16(x.q), parity.to_device_bf16(kg), lse)
+    got = lse.cpu().numpy().astype(np.float64)
+    want = _literal_lse(w, x, kg)
+    err = np.abs(got - want) / np.maximum(1.0, np.abs(want))
+    assert err.max() <= 2e-5, f"max err {err.max():.3g} at {np.unravel_index(err.argmax(), err.shape)}"
+
+
+@pytest.mark.parametrize("name", ["c2-llama-4133", "c4-gqa7-3001", "c5-ragged"])
+def test_literal_normaliser_layer(cuda_lib, name):
+    """tp_compress_layer_guide (pass 1, the prefix fold, pass 2, selection,
+    compaction) against the oracle with the guide keys."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    kg = synth.make_guide_keys(w)
+    p = _problem(binding, w, x.doc_offsets)
+    out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+    binding.compress(p, parity.to_device_bf16(x.q), parity.to_device_bf16(x.k),
+                     parity.to_device_bf16(x.v), w.keep_ratio, w.budget, out,
+                     k_guide=parity.to_device_bf16(kg))
+    assert binding.tp_check_status(out.ws) == 0
+    ref = _oracle(w, x, k_guide_bits=kg)
+    _check_layer(w, x, out, ref)
