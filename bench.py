@@ -21,7 +21,9 @@ Also reported on the same JSON line:
   cpu_baseline  the CPU oracle on a bounded sample of one layer;
   clocks        nvidia-smi samples taken during the timed region;
   lse_given     the same stack through tp_compress_layer_lse, the row
-                normalisers supplied by the caller (one pass over K).
+                normalisers supplied by the caller (one pass over K);
+  literal_normaliser  the same stack through tp_compress_layer_guide (the
+                guide's causal prefix folded into the normalisers).
 
 `--impl reference` times the CPU oracle (the only other implementation of
 this path) on the same workload and metric.
@@ -387,6 +389,25 @@ def run_ours(args, w):
                  "path": "tp_compress_layer_lse: caller row normalisers, one pass over K"}
     del lses
 
+    # ---- the literal normaliser: guide keys given (tp_compress_layer_guide)
+    kgs = [synth.make_guide_keys_torch(wr, l, dev) for l in range(L)]
+
+    def step_literal():
+        for (q, k, v), o, kg in zip(layers, outs, kgs):
+            binding.compress(p, q, k, v, w.keep_ratio, w.budget, o, stream, k_guide=kg)
+
+    for _ in range(args.warmup):
+        step_literal()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step_literal()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms_lit = ev0.elapsed_time(ev1) / args.steps
+    literal = {"value": w.n_total * L * world / (ms_lit / 1e3), "unit": UNIT, "ms_per_step": ms_lit,
+               "path": "tp_compress_layer_guide: guide prefix folded into the normalisers"}
+    del kgs
+
     read_b, write_b, flops1 = layer_algorithmic(w, kept_tokens)
     dom = max(("lse+vscale", "keyscore"), key=lambda s: stage_ms[s])
     dom_ms = stage_ms[dom]
@@ -498,6 +519,7 @@ def run_ours(args, w):
                        "parallelism": f"replicas{world}"},
             "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms,
             "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk, "lse_given": lse_given,
+            "literal_normaliser": literal,
             "cpu_baseline": cpu,
         }
         print(json.dumps(line))

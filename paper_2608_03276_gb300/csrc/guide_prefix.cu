@@ -16,15 +16,13 @@ namespace tp {
 
 namespace {
 
-constexpr int kPrefixWarps = 8;
-constexpr int kRowsPerWarp = 4;
-constexpr int kRowsPerCta = kPrefixWarps * kRowsPerWarp;
-constexpr int kKeyChunk = 32;  // guide keys per shared-memory chunk (one per lane)
+constexpr int kPrefixThreads = 256;
+constexpr int kRowsPerCta = 32;   // 8 warps x 4 rows
+constexpr int kKeyBlock = 128;    // 32 lanes x 4 keys
 constexpr int kMaxD = 128;
 
-__device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
-  return __uint_as_float(static_cast<uint32_t>(b) << 16);
-}
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // Merge of two (max, sum) pairs of exp terms; an empty pair is (-inf, 0).
 __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
@@ -34,63 +32,115 @@ __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2)
   m = mm;
 }
 
-// grid (ceil(rows / 32), batch * H_kv), 256 threads.  Warp w takes rows
-// r0 + w + 8 i (i < 4) of unit (b, h) = blockIdx.y; in each chunk of 32 guide
-// keys, lane l takes key j0 + l for all four rows at once.  The guide keys of
-// the chunk sit transposed in shared memory ([d][33]: conflict-free for both
-// the staging writes and the per-lane reads); the query rows are broadcast.
-__global__ void __launch_bounds__(kPrefixWarps * 32) tp_prefix_kernel(const __grid_constant__ PrefixParams p) {
-  __shared__ float qs[kRowsPerCta][kMaxD];
-  __shared__ float kt[kMaxD][kKeyChunk + 1];
+// Stages `count` bf16 rows of d elements (row stride d) into a transposed fp32
+// tile t[c * ld + i] (i < count; rows past `count` are zero).  Each thread
+// moves 16-byte pieces; consecutive threads take consecutive rows, so the
+// transposed stores hit distinct banks.  All of a thread's loads are issued
+// before the first store.
+template <int PER>
+__device__ __forceinline__ void stage_transposed(float* t, int ld, const uint16_t* src, int count,
+                                                 int d) {
+  const int pieces = d / 8;  // 16-byte pieces per row
+  uint4 v[PER];
+#pragma unroll
+  for (int u = 0; u < PER; ++u) {
+    const int idx = threadIdx.x + u * kPrefixThreads;
+    const int i = idx % ld, c8 = idx / ld;
+    v[u] = make_uint4(0u, 0u, 0u, 0u);
+    if (c8 < pieces && i < count)
+      v[u] = *reinterpret_cast<const uint4*>(src + static_cast<size_t>(i) * d + c8 * 8);
+  }
+#pragma unroll
+  for (int u = 0; u < PER; ++u) {
+    const int idx = threadIdx.x + u * kPrefixThreads;
+    const int i = idx % ld, c8 = idx / ld;
+    if (c8 >= pieces) continue;
+    float* col = t + (c8 * 8) * ld + i;
+    col[0 * ld] = bf16_lo(v[u].x);
+    col[1 * ld] = bf16_hi(v[u].x);
+    col[2 * ld] = bf16_lo(v[u].y);
+    col[3 * ld] = bf16_hi(v[u].y);
+    col[4 * ld] = bf16_lo(v[u].z);
+    col[5 * ld] = bf16_hi(v[u].z);
+    col[6 * ld] = bf16_lo(v[u].w);
+    col[7 * ld] = bf16_hi(v[u].w);
+  }
+}
+
+// grid (ceil(rows / 32), batch * H_kv), 256 threads, 80 KB of dynamic shared
+// memory: the CTA's 32 query rows ([d][32]) and one block of 128 guide keys
+// ([d][128]), both fp32 and transposed.  Warp w owns rows r0 + 4w .. 4w+3 and
+// lane l keys kb + 4l .. 4l+3 of each key block: per feature c it reads one
+// broadcast float4 of queries and one float4 of keys and does 16 FMAs.  Each
+// lane keeps a running (max, sum) per row over its keys; the lanes merge at
+// the end, and lane 0 folds the result into the row's normaliser.
+__global__ void __launch_bounds__(kPrefixThreads) tp_prefix_kernel(const __grid_constant__ PrefixParams p) {
+  extern __shared__ float4 prefix_smem[];
+  float* qs = reinterpret_cast<float*>(prefix_smem);     // [kMaxD][kRowsPerCta]
+  float* kt = qs + kMaxD * kRowsPerCta;                  // [kMaxD][kKeyBlock]
   grid_dep_launch();
   const int unit = blockIdx.y;
   const int b = unit / p.n_heads_kv;
   const int r0 = blockIdx.x * kRowsPerCta;
   const int d = p.head_dim, lt = p.guide_len;
   const size_t unit_row0 = static_cast<size_t>(unit) * p.rows;
-  const uint16_t* qb = p.q + unit_row0 * d;
   const uint16_t* kg = p.k_guide + static_cast<size_t>(unit) * lt * d;
+  const int nrows = min(kRowsPerCta, p.rows - r0);
 
-  for (int i = threadIdx.x; i < kRowsPerCta * d; i += blockDim.x) {
-    const int rr = i / d, c = i - rr * d;
-    const int r = r0 + rr;
-    qs[rr][c] = r < p.rows ? bf16_bits_to_f32(qb[static_cast<size_t>(r) * d + c]) : 0.f;
-  }
+  stage_transposed<kRowsPerCta * kMaxD / 8 / kPrefixThreads>(qs, kRowsPerCta, p.q + (unit_row0 + r0) * d,
+                                                             nrows, d);
   int jmax = 0;  // the largest guide position among this CTA's rows
-  for (int rr = 0; rr < kRowsPerCta && r0 + rr < p.rows; ++rr) jmax = max(jmax, (r0 + rr) % lt);
+  for (int rr = 0; rr < nrows; ++rr) jmax = max(jmax, (r0 + rr) % lt);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float m[kRowsPerWarp], s[kRowsPerWarp];
-  int jrow[kRowsPerWarp];
+  float m[4], s[4];
+  int jrow[4];
 #pragma unroll
-  for (int i = 0; i < kRowsPerWarp; ++i) {
+  for (int i = 0; i < 4; ++i) {
     m[i] = -INFINITY;
     s[i] = 0.f;
-    const int r = r0 + warp + kPrefixWarps * i;
+    const int r = r0 + 4 * warp + i;
     jrow[i] = r < p.rows ? r % lt : -1;
   }
-  for (int j0 = 0; j0 <= jmax; j0 += kKeyChunk) {
-    __syncthreads();  // the previous chunk is consumed (and qs is complete)
-    for (int i = threadIdx.x; i < kKeyChunk * d; i += blockDim.x) {
-      const int l = i / d, c = i - l * d;
-      kt[c][l] = j0 + l < lt ? bf16_bits_to_f32(kg[static_cast<size_t>(j0 + l) * d + c]) : 0.f;
-    }
+  for (int kb = 0; kb <= jmax; kb += kKeyBlock) {
+    __syncthreads();  // the previous key block is consumed
+    stage_transposed<kKeyBlock * kMaxD / 8 / kPrefixThreads>(kt, kKeyBlock, kg + static_cast<size_t>(kb) * d,
+                                                             min(kKeyBlock, lt - kb), d);
     __syncthreads();
-    float acc[kRowsPerWarp] = {0.f, 0.f, 0.f, 0.f};
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[i][e] = 0.f;
 #pragma unroll 4
     for (int c = 0; c < d; ++c) {
-      const float kv = kt[c][lane];
+      const float4 qv = *reinterpret_cast<const float4*>(qs + c * kRowsPerCta + 4 * warp);
+      const float4 kv = *reinterpret_cast<const float4*>(kt + c * kKeyBlock + 4 * lane);
+      const float qa[4] = {qv.x, qv.y, qv.z, qv.w};
+      const float ka[4] = {kv.x, kv.y, kv.z, kv.w};
 #pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) acc[i] = fmaf(qs[warp + kPrefixWarps * i][c], kv, acc[i]);
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) acc[i][e] = fmaf(qa[i], ka[e], acc[i][e]);
     }
-    const int jj = j0 + lane;
 #pragma unroll
-    for (int i = 0; i < kRowsPerWarp; ++i) {
-      if (jj <= jrow[i]) merge_ms(m[i], s[i], acc[i] * p.sigma, 1.f);
+    for (int i = 0; i < 4; ++i) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = kb + 4 * lane + e;
+        if (key > jrow[i]) continue;  // causal: guide token j sees keys 0..j
+        const float x = acc[i][e] * p.sigma;
+        if (x > m[i]) {
+          s[i] = s[i] * expf(m[i] - x) + 1.f;
+          m[i] = x;
+        } else {
+          s[i] += expf(x - m[i]);
+        }
+      }
     }
   }
 #pragma unroll
-  for (int i = 0; i < kRowsPerWarp; ++i) {
+  for (int i = 0; i < 4; ++i) {
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) {
       const float m2 = __shfl_xor_sync(0xffffffffu, m[i], o);
@@ -99,15 +149,21 @@ __global__ void __launch_bounds__(kPrefixWarps * 32) tp_prefix_kernel(const __gr
     }
   }
   grid_dep_wait();  // the context normalisers come from scoring pass 1
-  if (lane == 0) {
-    const bool empty = p.off[b + 1] == p.off[b];
+  if (lane < 4) {
+    float mi = m[0], si = s[0];
+    int ji = jrow[0];
 #pragma unroll
-    for (int i = 0; i < kRowsPerWarp; ++i) {
-      if (jrow[i] < 0) continue;
-      const size_t at = unit_row0 + r0 + warp + kPrefixWarps * i;
-      const float pre = m[i] + logf(s[i]);  // every row sees at least its own key
+    for (int i = 1; i < 4; ++i)
+      if (lane == i) {
+        mi = m[i];
+        si = s[i];
+        ji = jrow[i];
+      }
+    if (ji >= 0) {
+      const size_t at = unit_row0 + r0 + 4 * warp + lane;
+      const float pre = mi + logf(si);  // every row sees at least its own key
       // an empty document has no context terms (pass 1 writes no normaliser for it)
-      const float ctx = empty ? -INFINITY : p.lse[at];
+      const float ctx = p.off[b + 1] == p.off[b] ? -INFINITY : p.lse[at];
       float out = pre;
       if (ctx != -INFINITY) {
         const float mm = fmaxf(ctx, pre);
@@ -123,11 +179,14 @@ __global__ void __launch_bounds__(kPrefixWarps * 32) tp_prefix_kernel(const __gr
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s) {
   const int units = p.batch * p.n_heads_kv;
   if (units <= 0 || p.rows <= 0) return cudaSuccess;
-  if (p.head_dim > kMaxD) return cudaErrorInvalidValue;
+  if (p.head_dim > kMaxD || p.head_dim % 8 != 0) return cudaErrorInvalidValue;
+  const size_t smem = sizeof(float) * kMaxD * (kRowsPerCta + kKeyBlock);
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_prefix_kernel), 18);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((p.rows + kRowsPerCta - 1) / kRowsPerCta, units);
-  cfg.blockDim = dim3(kPrefixWarps * 32);
-  cfg.dynamicSmemBytes = 0;
+  cfg.blockDim = dim3(kPrefixThreads);
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
