@@ -22,9 +22,10 @@ Readings of the paper used here (where it is silent or ambiguous):
   a KV head are averaged (the paper budgets per KV head, Sec. 4 "Eviction");
 * pooling - the Eq. 1 window has 2*floor(K/2)+1 terms, so K must be odd; terms
   outside [0, n) are zero and the divisor stays K;
-* quantiser - symmetric per-token absmax, b = 8 bits (Eq. 2); fp32 scale;
-  codes are round-half-even of the IEEE fp32 quotient v / gamma, clamped to
-  +-(2^(b-1) - 1); gamma = 0 gives all-zero codes;
+* quantiser - symmetric per-token absmax, b = 8 or 4 bits (Eq. 2); fp32
+  scale; codes are round-half-even of the IEEE fp32 quotient v / gamma,
+  clamped to +-(2^(b-1) - 1); gamma = 0 gives all-zero codes; 4-bit codes are
+  stored two per byte, the even channel in the low nibble;
 * scale - softmax scale 1/sqrt(d) unless given;
 * budget - kept = ceil(ratio * n - 1e-9 * n) clamped to [0, n];
 * ties - equal scores keep the lower token index; kept indices ascend;
@@ -98,6 +99,20 @@ def quantize_v(v_bits, quant_bits: int = 8):
     q = np.clip(np.rint(quot), -qmax, qmax)
     q = np.where(gamma[..., None] > 0, q, 0.0)
     return gamma, q.astype(np.int8)
+
+
+def pack_codes(q, quant_bits: int = 8) -> np.ndarray:
+    """Storage form of the Eq. 2 codes.  b = 8: one int8 per value.  b = 4 (the
+    4-bit KV of the paper's experiments, Sec. 4 "Quantization"): two codes per
+    byte, channel 2i in the low nibble and channel 2i+1 in the high nibble,
+    each in 4-bit two's complement.  Returns int8 [..., d] or uint8 [..., d/2]."""
+    q = np.asarray(q)
+    if quant_bits == 8:
+        return q.astype(np.int8)
+    if quant_bits == 4:
+        u = q.astype(np.int64) & 0xF
+        return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)
+    raise ValueError("quant_bits must be 4 or 8")
 
 
 # --------------------------------------------------------------------------

@@ -227,6 +227,41 @@ def pin_quant_bounds(O):
     assert np.all(np.sign(top) == np.sign(vv[np.arange(64), arg]))
 
 
+def pin_quant4_golden(O):
+    """b = 4 (tests/golden/quant4_cases.txt): hand-derived scales, codes and the
+    two-per-byte storage (even channel in the low nibble)."""
+    with open(os.path.join(GOLDEN, "quant4_cases.txt")) as f:
+        lines = [ln.split("#")[0].strip() for ln in f]
+    n = 0
+    for ln in (x for x in lines if x):
+        vals, gam, codes, packed = ln.split("|")
+        gam = gam.strip()
+        gw = float.fromhex(gam) if gam.startswith("0x") else float(gam)
+        g, q = O.quantize_v(exact_bf16([[float(x) for x in vals.split()]]), 4)
+        assert float(g[0]) == gw, (vals, g[0], gw)
+        assert list(q[0]) == [int(c) for c in codes.split()], (vals, list(q[0]))
+        pk = O.pack_codes(q, 4)
+        assert pk.dtype == np.uint8 and pk.shape == (1, len(q[0]) // 2)
+        assert [int(x) for x in pk[0]] == [int(x, 16) for x in packed.split()], (vals, list(pk[0]))
+        n += 1
+    assert n == 4
+
+
+def pin_quant4_bounds(O):
+    """Random rows at b = 4: |q| <= 7, absmax -> +-7, |v - q*gamma| <= gamma * (1/2 + 2^-18)."""
+    rng = np.random.Generator(np.random.PCG64(12))
+    v = (rng.standard_normal((48, 64)) * np.exp(rng.uniform(-20, 20, (48, 1)))).astype(np.float32)
+    bits = (v.view(np.uint32) >> 16).astype(np.uint16)
+    vv = (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    g, q = O.quantize_v(bits, 4)
+    assert np.all(np.abs(q.astype(np.int64)) <= 7)
+    assert np.allclose(g, np.abs(vv).max(axis=1) / 7.0, rtol=2 ** -23, atol=0)
+    err = np.abs(vv - q.astype(np.float64) * g.astype(np.float64)[:, None])
+    assert np.all(err <= g.astype(np.float64)[:, None] * (0.5 + 2 ** -18)), err.max()
+    arg = np.argmax(np.abs(vv), axis=1)
+    assert np.all(np.abs(q[np.arange(48), arg].astype(np.int64)) == 7)
+
+
 # -- Eq. 3 and Sec. 3.4 selection ---------------------------------------------
 
 def pin_combine_product(O):

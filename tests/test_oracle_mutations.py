@@ -46,6 +46,8 @@ MUTATIONS = {
     "literal rows token-major": ("out[gi * lt + j] = m", "out[j * g + gi] = m"),
     "guide keys of document 0": ("lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, h], sigma)", "lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[0, h], sigma)"),
     "guide keys of head 0": ("lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, h], sigma)", "lse_rows = guide_lse_literal(qg, k_all[h, lo:hi], kg[b, 0], sigma)"),
+    "4-bit nibbles swapped": ("return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)", "return (u[..., 1::2] | (u[..., 0::2] << 4)).astype(np.uint8)"),
+    "4-bit codes sign-magnitude": ("u = q.astype(np.int64) & 0xF", "u = np.abs(q).astype(np.int64) | np.where(q < 0, 8, 0)"),
     "normalised add with L1 norms": ("na, nb = math.sqrt(float(np.sum(a * a))), math.sqrt(float(np.sum(b * b)))", "na, nb = float(np.sum(np.abs(a))), float(np.sum(np.abs(b)))"),
     "harmonic mean without the factor 2": ("out[nz] = 2.0 * a[nz] * b[nz] / den[nz]", "out[nz] = a[nz] * b[nz] / den[nz]"),
     "harmonic mean divides by a zero sum": ("nz = den != 0", "nz = den == den"),
