@@ -18,14 +18,18 @@
  *        Q guide   [batch, H_q, L_t, d]   bf16, post-RoPE guide queries
  *        K, V      [H_kv, N, d]           bf16, documents packed along N
  *        gamma     [H_kv, N]              fp32 per-token V scale
- *        Vq        [H_kv, N, d]           int8 codes
+ *        Vq        [H_kv, N, d*b/8]       Eq. 2 codes (see below)
  *        scores    [H_kv, N]              fp32 combined scores s_i
  *        idx       [batch, H_kv, cap]     int32, doc-local kept indices
  *        Kc, Vc    [batch, H_kv, cap, d]  bf16 compressed cache
- *        Vqc       [batch, H_kv, cap, d]  int8
+ *        Vqc       [batch, H_kv, cap, d*b/8] Eq. 2 codes
  *        gammac    [batch, H_kv, cap]     fp32
  *    where cap = tp_kept_capacity(...).  Document b keeps k_b <= cap tokens;
  *    slots k_b..cap-1 of its rows are filled with idx = -1 and zero bytes.
+ *  - Codes (b = quant_bits): b = 8, one int8 per value; b = 4 (the 4-bit KV
+ *    of the paper's experiments, Sec. 4), two per byte, channel 2i in the
+ *    low nibble and channel 2i+1 in the high nibble, each 4-bit two's
+ *    complement.  Code buffers are 8-byte (b = 8) or 4-byte (b = 4) aligned.
  *  - Query head h belongs to KV head h / (H_q / H_kv) (contiguous groups).
  *  - Every call takes a cudaStream_t (passed as void*; NULL = legacy default
  *    stream), enqueues its kernels and returns without synchronising.
@@ -78,7 +82,7 @@ extern "C" {
  *                           offsets, doc_offsets[0] = 0; document b owns
  *                           tokens [doc_offsets[b], doc_offsets[b+1]).
  *   pool_kernel           : K of Eq. 1's average pooling; odd, 1..33 (default 5)
- *   quant_bits            : b of Eq. 2; only 8 is supported
+ *   quant_bits            : b of Eq. 2: 8 or 4
  *   softmax_scale         : logit scale; <= 0 means 1/sqrt(d)
  *   flags                 : 0 (Eq. 3 product), or one of TP_SCORE_KEY_ONLY,
  *                           TP_SCORE_NORM_ADD, TP_SCORE_HARMONIC
@@ -120,11 +124,12 @@ int64_t tp_kept_capacity(const tp_problem* p, double keep_ratio, int64_t budget)
 size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget);
 
 /*
- * Eq. 2 (Sec. 3.3) for every token of V: gamma_i = max_c |v_ic| / 127 (fp32,
- * IEEE round-to-nearest division) and int8 codes q_ic = clamp(rint(v_ic /
- * gamma_i), -127, 127) (IEEE fp32 quotient, round-half-even; gamma_i = 0
- * gives q_i = 0).  v: [H_kv, N, d] bf16 in; vq: [H_kv, N, d] int8 out (may be
- * NULL to compute gamma only); gamma: [H_kv, N] fp32 out.
+ * Eq. 2 (Sec. 3.3) for every token of V: gamma_i = max_c |v_ic| / qmax with
+ * qmax = 2^(b-1) - 1 (127 or 7; fp32, IEEE round-to-nearest division) and
+ * codes q_ic = clamp(rint(v_ic / gamma_i), -qmax, qmax) (IEEE fp32 quotient,
+ * round-half-even; gamma_i = 0 gives q_i = 0).  v: [H_kv, N, d] bf16 in;
+ * vq: [H_kv, N, d*b/8] codes out, stored as described above (may be NULL to
+ * compute gamma only); gamma: [H_kv, N] fp32 out.
  */
 int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, void* stream);
 

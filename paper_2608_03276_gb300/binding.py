@@ -164,6 +164,19 @@ def _ptr(t, dtype=None, numel=None, name="tensor", nullable=False):
     return c_void_p(t.data_ptr())
 
 
+def _codes(p: Problem, t, rows: int, name: str):
+    """Eq. 2 code buffer of `rows` rows: int8 [rows, d] at b = 8, uint8
+    [rows, d / 2] (two codes per byte) at b = 4; None allowed."""
+    import torch
+    bits, d = p.c.quant_bits, p.c.head_dim
+    return _ptr(t, torch.int8 if bits == 8 else torch.uint8, rows * d * bits // 8, name, nullable=True)
+
+
+def code_dtype(p: Problem):
+    import torch
+    return torch.int8 if p.c.quant_bits == 8 else torch.uint8
+
+
 def _stream(stream):
     import torch
     s = stream if stream is not None else torch.cuda.current_stream()
@@ -192,7 +205,7 @@ def tp_quantize_v(p: Problem, v, vq, gamma, stream=None):
     hkv, d, n = p.c.n_heads_kv, p.c.head_dim, p.n_total
     _check("tp_quantize_v", load().tp_quantize_v(
         p.ref(), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
-        _ptr(vq, torch.int8, hkv * n * d, "vq", nullable=True),
+        _codes(p, vq, hkv * n, "vq"),
         _ptr(gamma, torch.float32, hkv * n, "gamma"), _stream(stream)))
 
 
@@ -277,7 +290,7 @@ def tp_compact(p: Problem, k, v, gamma, idx, keep_ratio: float, budget: int, kc,
         keep_ratio, budget,
         _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
         _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
-        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _codes(p, vqc, m, "vqc"),
         _ptr(gammac, torch.float32, m, "gammac", nullable=True), _stream(stream)))
 
 
@@ -294,7 +307,7 @@ def tp_compress_layer(p: Problem, q, k, v, keep_ratio: float, budget: int, idx, 
         _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
         _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
         _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
-        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _codes(p, vqc, m, "vqc"),
         _ptr(gammac, torch.float32, m, "gammac", nullable=True),
         _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
@@ -316,7 +329,7 @@ def tp_compress_layer_lse(p: Problem, q, k, v, lse, keep_ratio: float, budget: i
         _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
         _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
         _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
-        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _codes(p, vqc, m, "vqc"),
         _ptr(gammac, torch.float32, m, "gammac", nullable=True),
         _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
@@ -337,7 +350,7 @@ def tp_compress_layer_guide(p: Problem, q, k, v, k_guide, keep_ratio: float, bud
         _ptr(idx, torch.int32, m, "idx", nullable=cap == 0),
         _ptr(kc, torch.bfloat16, m * d, "kc", nullable=True),
         _ptr(vc, torch.bfloat16, m * d, "vc", nullable=True),
-        _ptr(vqc, torch.int8, m * d, "vqc", nullable=True),
+        _codes(p, vqc, m, "vqc"),
         _ptr(gammac, torch.float32, m, "gammac", nullable=True),
         _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
@@ -365,7 +378,7 @@ class CompressOutputs:
         self.idx = torch.empty(shp, dtype=torch.int32, device=device)
         self.kc = torch.empty(shp + (d,), dtype=torch.bfloat16, device=device)
         self.vc = torch.empty(shp + (d,), dtype=torch.bfloat16, device=device)
-        self.vqc = torch.empty(shp + (d,), dtype=torch.int8, device=device)
+        self.vqc = torch.empty(shp + (d * p.c.quant_bits // 8,), dtype=code_dtype(p), device=device)
         self.gammac = torch.empty(shp, dtype=torch.float32, device=device)
         self.scores = torch.empty((hkv, n), dtype=torch.float32, device=device) if with_scores else None
         self.gamma = torch.empty((hkv, n), dtype=torch.float32, device=device) if with_scores else None

@@ -27,6 +27,8 @@ struct Plan {
   int stages1, stages2;
   size_t smem1, smem2;
   float c2, inv_group, sigma;
+  int bits;     // Eq. 2 code width: 8 or 4
+  float qmax;   // 2^(bits-1) - 1
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
@@ -56,7 +58,7 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   if (p->head_dim != 64 && p->head_dim != 128) return TP_ERR_UNSUPPORTED_SHAPE;
   if (p->pool_kernel < 1 || p->pool_kernel % 2 == 0 || p->pool_kernel > 33)
     return TP_ERR_UNSUPPORTED_SHAPE;
-  if (p->quant_bits != 8) return TP_ERR_UNSUPPORTED_SHAPE;
+  if (p->quant_bits != 8 && p->quant_bits != 4) return TP_ERR_UNSUPPORTED_SHAPE;
   const uint32_t score_flags = TP_SCORE_KEY_ONLY | TP_SCORE_NORM_ADD | TP_SCORE_HARMONIC;
   if (p->flags & ~score_flags) return TP_ERR_INVALID_ARG;
   const uint32_t f = p->flags;
@@ -86,6 +88,8 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   const double sigma = p->softmax_scale > 0 ? double(p->softmax_scale) : 1.0 / sqrt(double(P->d));
   P->c2 = static_cast<float>(sigma * 1.4426950408889634);
   P->sigma = static_cast<float>(sigma);
+  P->bits = p->quant_bits;
+  P->qmax = static_cast<float>((1 << (p->quant_bits - 1)) - 1);
   P->inv_group = 1.0f / static_cast<float>(P->g);
 
   // Key tiles per CTA: the smallest T whose CTA count fits one wave.
@@ -198,6 +202,10 @@ bool encode_maps(const Plan& P, const void* q, const void* k, CUtensorMap* tmk, 
                    P.rows_pad < 256 ? P.rows_pad : 256);
 }
 
+// Alignment mask of a code buffer: a thread stores 8 codes at once (8 bytes,
+// or 4 at b = 4).
+uintptr_t code_align(const Plan& P) { return P.bits == 8 ? 7 : 3; }
+
 DocTable doc_table(const Plan& P) {
   DocTable docs;
   memset(&docs, 0, sizeof(docs));
@@ -222,7 +230,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
   lp.docs = doc_table(P);
   lp.q = static_cast<const uint16_t*>(q);
   lp.gamma = gamma;
-  lp.qmax = 127.0f;
+  lp.qmax = P.qmax;
   lp.n_total = P.n_total;
   lp.n_heads_kv = P.hkv;
   lp.rows = P.rows;
@@ -327,7 +335,8 @@ void fill_gather(const Plan& P, GatherParams* gp) {
   gp->head_dim = P.d;
   gp->n_total = P.n_total;
   gp->cap = P.cap;
-  gp->qmax = 127.0f;
+  gp->qmax = P.qmax;
+  gp->bits = P.bits;
 }
 
 // The fused layer.  Without `lse`: two scoring passes (the first also forms
@@ -344,7 +353,7 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   if (!q || !k || !v || (!idx && P.cap > 0) || !aligned16(q) || !aligned16(k) || !aligned16(v))
     return TP_ERR_INVALID_ARG;
   if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
-      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
+      (vqc && (reinterpret_cast<uintptr_t>(vqc) & code_align(P))))
     return TP_ERR_INVALID_ARG;
   if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
     return TP_ERR_WORKSPACE;
@@ -356,7 +365,7 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
     if ((st = run_scoring(P, q, k, v, g, w, s, k_guide)) != TP_OK) return st;
   } else if (P.n_total > 0 && P.grid_x > 0) {
     if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
-                      127.0f, num_sms(), s) != cudaSuccess)
+                      P.qmax, P.bits, num_sms(), s) != cudaSuccess)
       return TP_ERR_CUDA;
     CUtensorMap tmk, tmq;
     if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
@@ -471,10 +480,10 @@ int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, 
   Plan P;
   int st = make_plan(p, 0.0, 0, false, &P);
   if (st != TP_OK) return st;
-  if (!v || !gamma || !aligned16(v) || (vq && (reinterpret_cast<uintptr_t>(vq) & 7)))
+  if (!v || !gamma || !aligned16(v) || (vq && (reinterpret_cast<uintptr_t>(vq) & code_align(P))))
     return TP_ERR_INVALID_ARG;
   return cuda_status(launch_vquant(static_cast<const uint16_t*>(v), vq, gamma,
-                                   int64_t(P.hkv) * P.n_total, P.d, 127.0f, num_sms(),
+                                   int64_t(P.hkv) * P.n_total, P.d, P.qmax, P.bits, num_sms(),
                                    static_cast<cudaStream_t>(stream)));
 }
 
@@ -581,7 +590,7 @@ int tp_compact(const tp_problem* p, const void* k, const void* v, const float* g
   if (P.cap == 0) return TP_OK;
   if (!k || !v || !gamma || !idx || !aligned16(k) || !aligned16(v)) return TP_ERR_INVALID_ARG;
   if ((kc && !aligned16(kc)) || (vc && !aligned16(vc)) ||
-      (vqc && (reinterpret_cast<uintptr_t>(vqc) & 7)))
+      (vqc && (reinterpret_cast<uintptr_t>(vqc) & code_align(P))))
     return TP_ERR_INVALID_ARG;
   GatherParams gp;
   fill_gather(P, &gp);

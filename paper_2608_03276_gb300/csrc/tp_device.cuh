@@ -534,6 +534,17 @@ __device__ __forceinline__ uint2 quant8_packed(const uint4& u, float gamma, floa
   return make_uint2(lo, hi);
 }
 
+// The eight codes of quant8_packed (qmax <= 7) stored as 4-bit two's
+// complement, two per byte: code 2i in the low nibble of byte i, code 2i+1 in
+// its high nibble.
+__device__ __forceinline__ uint32_t quant4_packed(const uint4& u, float gamma, float qmax) {
+  const uint2 c = quant8_packed(u, gamma, qmax);
+  // bytes b0..b3 of a word -> nibbles: (b0 | b1 << 4) in byte 0, (b2 | b3 << 4) in byte 2
+  const uint32_t x = c.x & 0x0F0F0F0Fu, y = c.y & 0x0F0F0F0Fu;
+  const uint32_t xs = x | (x >> 4), ys = y | (y >> 4);
+  return __byte_perm(xs, ys, 0x6420);
+}
+
 __device__ __forceinline__ uint2 quant8_bf16(const uint4& u, float gamma, float qmax) {
   float f[8];
   bf16x8_to_f32(u, f);

@@ -104,6 +104,7 @@ struct GatherParams {
   int64_t n_total;
   int64_t cap;
   float qmax;
+  int bits;           // 8: int8 codes; 4: two codes per byte
   const uint16_t* k;
   const uint16_t* v;
   const float* gamma;
@@ -130,8 +131,8 @@ struct PrefixParams {
 };
 
 // Launchers (return cudaError_t of the launch).
-cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
-                          float qmax, int num_sms, cudaStream_t s);
+cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
+                          float qmax, int bits, int num_sms, cudaStream_t s);
 cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                        const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s);
 // `dependent`: launch as a programmatic dependent of the previous kernel in

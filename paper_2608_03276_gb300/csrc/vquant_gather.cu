@@ -1,5 +1,6 @@
-// Eq. 2 (Sec. 3.3) per-token V scale and int8 codes, and the order-preserving
-// compaction of kept rows into the compressed cache (Sec. 3.1).
+// Eq. 2 (Sec. 3.3) per-token V scale and codes (b = 8: int8; b = 4: two per
+// byte), and the order-preserving compaction of kept rows into the compressed
+// cache (Sec. 3.1).
 //
 // Both kernels move 16-byte vectors: a row of d bf16 is d/8 lanes wide, so a
 // warp covers 32/(d/8) rows per instruction.  The quantisation rule is the
@@ -19,9 +20,9 @@ namespace {
 // lane group so that several 16-byte loads are in flight per thread.
 template <int LPR, int UNROLL>
 __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict__ v,
-                                                      uint2* __restrict__ vq,
+                                                      void* __restrict__ vq,
                                                       float* __restrict__ gamma, int64_t rows,
-                                                      float qmax) {
+                                                      float qmax, int bits) {
   constexpr int RPW = 32 / LPR;  // rows per warp instruction
   const int lane = threadIdx.x & 31;
   const int sub = lane / LPR, part = lane % LPR;
@@ -46,7 +47,12 @@ __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict_
       for (int o = LPR / 2; o >= 1; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
       const float g = __fdiv_rn(a, qmax);
       if (row < rows) {
-        if (vq) vq[row * LPR + part] = quant8_packed(u[k], g, qmax);
+        if (vq) {
+          if (bits == 8)
+            static_cast<uint2*>(vq)[row * LPR + part] = quant8_packed(u[k], g, qmax);
+          else
+            static_cast<uint32_t*>(vq)[row * LPR + part] = quant4_packed(u[k], g, qmax);
+        }
         if (part == 0) gamma[row] = g;
       }
     }
@@ -98,16 +104,20 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
     const int64_t dst = slot * LPR + part;
     if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = kv[u];
     if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = vv[u];
-    if (p.vqc)
-      reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_packed(vv[u], g[u], p.qmax) : make_uint2(0, 0);
+    if (p.vqc) {
+      if (p.bits == 8)
+        reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_packed(vv[u], g[u], p.qmax) : make_uint2(0, 0);
+      else
+        reinterpret_cast<uint32_t*>(p.vqc)[dst] = j[u] >= 0 ? quant4_packed(vv[u], g[u], p.qmax) : 0u;
+    }
     if (p.gammac && part == 0) p.gammac[slot] = g[u];
   }
 }
 
 }  // namespace
 
-cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t rows, int head_dim,
-                          float qmax, int num_sms, cudaStream_t s) {
+cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
+                          float qmax, int bits, int num_sms, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
   constexpr int kUnroll = 4;
   const int threads = 256;
@@ -117,11 +127,10 @@ cudaError_t launch_vquant(const uint16_t* v, int8_t* vq, float* gamma, int64_t r
   const int64_t cap = static_cast<int64_t>(num_sms) * 8;
   if (blocks > cap) blocks = cap;
   const uint4* vv = reinterpret_cast<const uint4*>(v);
-  uint2* qq = reinterpret_cast<uint2*>(vq);
   if (head_dim == 128)
-    tp_vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+    tp_vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits);
   else
-    tp_vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, qq, gamma, rows, qmax);
+    tp_vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits);
   return cudaGetLastError();
 }
 

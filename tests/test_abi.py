@@ -63,7 +63,7 @@ def test_capacity_and_workspace(lib):
 
 @pytest.mark.parametrize("kw", [
     dict(head_dim=96), dict(head_dim=256), dict(pool_kernel=4), dict(pool_kernel=0), dict(pool_kernel=35),
-    dict(quant_bits=4), dict(n_heads_q=7), dict(guide_len=0), dict(guide_len=65, n_heads_q=16),
+    dict(quant_bits=2), dict(quant_bits=16), dict(n_heads_q=7), dict(guide_len=0), dict(guide_len=65, n_heads_q=16),
 ])
 def test_rejects_unsupported(lib, kw):
     p = _prob(lib, [0, 100], **kw)

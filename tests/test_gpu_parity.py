@@ -38,7 +38,7 @@ def _run_compress(binding, w, x, keep_ratio=None, budget=None, **kw):
     return out
 
 
-def _check_layer(w, x, out, ref, heads=None, docs=None, key_only=False):
+def _check_layer(w, x, out, ref, heads=None, docs=None, key_only=False, bits=8):
     scores = out.scores.cpu().numpy()
     gamma = out.gamma.cpu().numpy()
     idx = out.idx.cpu().numpy()
@@ -54,6 +54,7 @@ def _check_layer(w, x, out, ref, heads=None, docs=None, key_only=False):
             parity.assert_kept(idx[b, h], ref["k"][b], ref["scores"][(b, h)], scores[h, lo:hi], tag)
             k_b = ref["k"][b]
             rk, rv, rq, rg = O.gather_rows(x.k, x.v, ref["gamma"], ref["vq"], lo, h, idx[b, h, :k_b])
+            rq = O.pack_codes(rq, bits)
             assert np.array_equal(kc[b, h, :k_b], rk), f"{tag}: Kc"
             assert np.array_equal(vc[b, h, :k_b], rv), f"{tag}: Vc"
             assert np.array_equal(vqc[b, h, :k_b], rq), f"{tag}: Vqc"

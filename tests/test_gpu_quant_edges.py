@@ -1,4 +1,4 @@
-"""Eq. 2 int8 codes next to rounding boundaries, through the C ABI.
+"""Eq. 2 codes (b = 8 and b = 4) next to rounding boundaries, through the C ABI.
 
 The kernels form t = v * fl(1/gamma) and round it with an adder; they take
 the exact division only when t lies within 4e-5 of a half-integer (or a
@@ -23,8 +23,8 @@ def _bf16_values():
     return (bits << 16).view(np.float32)
 
 
-def _edge_rows(d, nrows, seed=3):
-    """Rows whose absmax a fixes an ordinary scale gamma = fl32(a / 127) (not a
+def _edge_rows(d, nrows, seed=3, qmax=127):
+    """Rows whose absmax a fixes an ordinary scale gamma = fl32(a / qmax) (not a
     power of two).  The other values are the bf16 values v < a with
     |v / gamma - (k + 1/2)| < 4e-5 (each scale has one or two; they are
     repeated), and values 4e-5 .. 2e-3 from a boundary (just outside the
@@ -35,7 +35,7 @@ def _edge_rows(d, nrows, seed=3):
     while len(rows) < nrows:
         a = np.float32(rng.uniform(0.5, 300.0))
         a = np.float32((np.array([a]).view(np.uint32) & 0xFFFF0000).view(np.float32)[0])  # a bf16 value
-        gamma = np.float32(a / np.float32(127.0))
+        gamma = np.float32(a / np.float32(qmax))
         if np.frexp(gamma)[0] == 0.5:
             continue
         cand = vals[(vals > 0) & (vals < a)]
@@ -54,26 +54,30 @@ def _edge_rows(d, nrows, seed=3):
     return (r.view(np.uint32) >> 16).astype(np.uint16)
 
 
+@pytest.mark.parametrize("bits", [8, 4])
 @pytest.mark.parametrize("d", [64, 128])
-def test_codes_at_rounding_boundaries(cuda_lib, d):
+def test_codes_at_rounding_boundaries(cuda_lib, d, bits):
     import torch
     from paper_2608_03276_gb300 import binding
     n, hkv = 384, 2
-    v = np.stack([_edge_rows(d, n, seed=10 + h) for h in range(hkv)])  # [H_kv, n, d]
-    p = binding.Problem(2 * hkv, hkv, d, 4, [0, n])
-    vq = torch.empty((hkv, n, d), dtype=torch.int8, device="cuda")
+    qmax = (1 << (bits - 1)) - 1
+    v = np.stack([_edge_rows(d, n, seed=10 + h, qmax=qmax) for h in range(hkv)])  # [H_kv, n, d]
+    p = binding.Problem(2 * hkv, hkv, d, 4, [0, n], quant_bits=bits)
+    vq = torch.empty((hkv, n, d * bits // 8), dtype=binding.code_dtype(p), device="cuda")
     g = torch.empty((hkv, n), dtype=torch.float32, device="cuda")
     binding.tp_quantize_v(p, parity.to_device_bf16(v), vq, g)
-    rg, rq = O.quantize_v(v)
+    rg, rq = O.quantize_v(v, bits)
+    rq = O.pack_codes(rq, bits)
     assert np.array_equal(g.cpu().numpy().view(np.uint32), rg.view(np.uint32))
     got = vq.cpu().numpy()
-    assert np.array_equal(got, rq), f"{int((got != rq).sum())} codes differ"
+    assert np.array_equal(got, rq), f"{int((got != rq).sum())} code bytes differ"
 
     # the same rows through the compaction kernel (every token kept, in order)
     k = np.zeros_like(v)
     idx = np.tile(np.arange(n, dtype=np.int32), (1, hkv, 1))
     kc = torch.empty((1, hkv, n, d), dtype=torch.bfloat16, device="cuda")
-    vc, vqc = torch.empty_like(kc), torch.empty(kc.shape, dtype=torch.int8, device="cuda")
+    vc = torch.empty_like(kc)
+    vqc = torch.empty((1, hkv, n, d * bits // 8), dtype=binding.code_dtype(p), device="cuda")
     gc = torch.empty((1, hkv, n), dtype=torch.float32, device="cuda")
     binding.tp_compact(p, parity.to_device_bf16(k), parity.to_device_bf16(v),
                        torch.tensor(rg, device="cuda"), torch.tensor(idx, device="cuda"), 0.0, n,

@@ -176,3 +176,52 @@ def test_literal_normaliser_layer(cuda_lib, name):
     assert binding.tp_check_status(out.ws) == 0
     ref = _oracle(w, x, k_guide_bits=kg)
     _check_layer(w, x, out, ref)
+
+
+# ---------------------------------------------------------------------------
+# b = 4: scales absmax / 7, codes two per byte (Sec. 4 "Quantization")
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["c1-tiny-2k", "c2-llama-4133", "c5-ragged"])
+def test_int4_fused_layer(cuda_lib, name):
+    """The fused layer at b = 4: pass 1 forms gamma = absmax / 7, the scores use
+    it (Eq. 3), and the compacted codes are packed two per byte."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    out = _run_compress(binding, w, x, quant_bits=4)
+    ref = _oracle(w, x, quant_bits=4)
+    _check_layer(w, x, out, ref, bits=4)
+    assert out.vqc.dtype.itemsize == 1 and out.vqc.shape[-1] == w.head_dim // 2
+
+
+def test_int4_caller_lse_layer(cuda_lib):
+    """b = 4 through tp_compress_layer_lse, whose scales come from the
+    standalone quantiser kernel."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL["c4-gqa7-3001"]
+    x = synth.make_layer(w)
+    lse = _context_lse(w, x)
+    import torch
+    p = _problem(binding, w, x.doc_offsets, quant_bits=4)
+    out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+    binding.compress(p, parity.to_device_bf16(x.q), parity.to_device_bf16(x.k),
+                     parity.to_device_bf16(x.v), w.keep_ratio, w.budget, out,
+                     lse=torch.tensor(lse, device="cuda"))
+    assert binding.tp_check_status(out.ws) == 0
+    ref = _oracle(w, x, quant_bits=4, lse=lse.astype(np.float64))
+    _check_layer(w, x, out, ref, bits=4)
+
+
+@pytest.mark.parametrize("name", ["c1-tiny-2k", "c3-guide128-2053"])
+def test_int4_quantize_v(cuda_lib, name):
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    x = synth.make_layer(w)
+    p = _problem(binding, w, x.doc_offsets, quant_bits=4)
+    vq = torch.empty((w.n_heads_kv, p.n_total, w.head_dim // 2), dtype=torch.uint8, device="cuda")
+    g = torch.empty((w.n_heads_kv, p.n_total), dtype=torch.float32, device="cuda")
+    binding.tp_quantize_v(p, parity.to_device_bf16(x.v), vq, g)
+    rg, rq = O.quantize_v(x.v, 4)
+    assert np.array_equal(g.cpu().numpy().view(np.uint32), rg.view(np.uint32))
+    assert np.array_equal(vq.cpu().numpy(), O.pack_codes(rq, 4))
