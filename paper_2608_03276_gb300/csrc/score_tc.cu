@@ -54,9 +54,9 @@ __host__ __device__ inline ScoreSmem score_layout(int head_dim, int rows_pad, in
 
 // Pass 2 extras after its barriers: up to 1 KB of alignment, the row-offset
 // operands of the extra K step (key side 128 x 32 B, guide side rows x 32 B),
-// the warpgroup partials [2][4][128].
+// the epilogue partials [4 tiles][4][128 keys].
 __host__ __device__ inline uint32_t keyscore_extra_bytes(int rows_pad) {
-  return 1024u + 128u * 32u + static_cast<uint32_t>(rows_pad) * 32u + 2u * 4u * 128u * 4u;
+  return 1024u + 128u * 32u + static_cast<uint32_t>(rows_pad) * 32u + 4u * 4u * 128u * 4u;
 }
 
 __device__ __forceinline__ uint8_t* aligned_smem(uint8_t* raw) {
@@ -581,6 +581,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tfull = q_full + 1;   // [2 TMEM buffers]
   uint64_t* tempty = tfull + 2;   // [2 TMEM buffers], one arrival per epilogue warp
   uint64_t* drain = tempty + 2;
+  uint64_t* pdone = drain + 1;    // [4] partial slots complete, one arrival per warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   // Row offsets as an extra K step of the contraction (32-byte swizzled,
@@ -588,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // hi + mid + lo = -lse[row] / sigma (three bf16 parts, exact to ~2^-24).
   uint8_t* a_aug = smem + ((L.extra + 1023u) & ~1023u);               // [128 keys][32 B]
   uint8_t* b_aug = a_aug + 128 * 32;                                  // [rows_pad][32 B]
-  float* part = reinterpret_cast<float*>(b_aug + rows_pad * 32);      // [2][4][128]
+  float* part = reinterpret_cast<float*>(b_aug + rows_pad * 32);      // [4][4][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -608,9 +609,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull[i], 1);
-      mbar_init(&tempty[i], kEpiWarps);
+      mbar_init(&tempty[i], kEpiWarps / 2);  // one group of eight warps drains a buffer
     }
     mbar_init(drain, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(&pdone[i], 8 * nh);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -722,44 +724,64 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    const int g = (warp - kEpiWarp0) >> 2, quad = warp & 3;
+    // Two groups of eight warps take alternate jobs: job j = lt * nh + hh goes
+    // to group j & 1, which drains TMEM buffer j & 1, so one group's TMEM loads
+    // overlap the other group's arithmetic.  In a group, warp (cg, quad)
+    // reduces TMEM lanes 32 quad .. 32 quad + 31 (keys) over the column chunks
+    // 4 cg .. 4 cg + 3; the second pair of chunks loads while the first pair is
+    // reduced, and the buffer is released once all four are in registers.
+    const int e = warp - kEpiWarp0, grp = e >> 3, cg = (e >> 2) & 1, quad = warp & 3;
     const float c2 = p.c2;
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     bool ok = true;
     for (int lt = 0; lt < nt; ++lt) {
-      float acc = 0.f;
+      float* slot = part + (lt & 3) * 4 * 128;  // partials (hh, cg) of this tile's keys
+      uint64_t* done = &pdone[lt & 3];
       for (int hh = 0; hh < nh; ++hh) {
         const int j = lt * nh + hh, buf = j & 1;
+        if (buf != grp) continue;
         if (ok && !mbar_wait(&tfull[buf], (j >> 1) & 1, abort_flag)) ok = false;
-        if (!ok) break;
+        if (!ok) continue;
         tc_fence_after();
         const int nch = min(256, rows_mma - 256 * hh) / 32;
         const uint32_t tb = tlane + buf * 256;
-        const int c0 = g, c1 = g + 4;
+        const int ch = 4 * cg;
+        float acc = 0.f;
         uint32_t ra[32], rb[32];
-        if (c0 < nch) tmem_ld32_async(tb + c0 * 32, ra);
-        if (c1 < nch) tmem_ld32_async(tb + c1 * 32, rb);
-        if (c0 < nch) tmem_wait(ra);
-        if (c1 < nch) tmem_wait(rb);
+        if (ch < nch) tmem_ld32_async(tb + ch * 32, ra);
+        if (ch + 1 < nch) tmem_ld32_async(tb + (ch + 1) * 32, rb);
+        if (ch < nch) tmem_wait(ra);
+        if (ch + 1 < nch) tmem_wait(rb);
+        if (ch < nch) acc += key_chunk(ra, c2);
+        if (ch + 2 < nch) tmem_ld32_async(tb + (ch + 2) * 32, ra);
+        if (ch + 1 < nch) acc += key_chunk(rb, c2);
+        if (ch + 3 < nch) tmem_ld32_async(tb + (ch + 3) * 32, rb);
+        if (ch + 2 < nch) tmem_wait(ra);
+        if (ch + 3 < nch) tmem_wait(rb);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[buf]);
-        if (c0 < nch) acc += key_chunk(ra, c2);
-        if (c1 < nch) acc += key_chunk(rb, c2);
+        if (ch + 2 < nch) acc += key_chunk(ra, c2);
+        if (ch + 3 < nch) acc += key_chunk(rb, c2);
+        slot[(hh * 2 + cg) * 128 + quad * 32 + lane] = acc;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(done);
       }
-      // fixed-order sum of the four warpgroups' partials for this tile's keys
-      float* slot = part + (lt & 1) * 4 * 128;
-      if (ok) slot[g * 128 + quad * 32 + lane] = acc;
-      asm volatile("bar.sync 1, %0;" ::"r"(kEpiWarps * 32) : "memory");
-      if (!ok || *abort_flag) {
-        ok = false;
-        continue;
-      }
-      if (g == 0) {
-        const int kl = quad * 32 + lane;
-        const float s4 = ((slot[kl] + slot[128 + kl]) + slot[256 + kl]) + slot[384 + kl];
-        const int key = (t0 + lt) * kKeyTile + kl;
-        if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = s4 * p.inv_group;
+      // The cg = 0 warps of the group that ran the tile's last job sum the
+      // partials in a fixed order once every warp of the tile's jobs has
+      // arrived on the slot's barrier (phase lt / 4).  No warp reaches the same
+      // slot four tiles on before this read: that job needs a TMEM buffer that
+      // this group releases only after it.
+      const int fin = (lt * nh + nh - 1) & 1;
+      if (grp == fin && cg == 0) {
+        if (ok && !mbar_wait(done, (lt >> 2) & 1, abort_flag)) ok = false;
+        if (ok) {
+          const int kl = quad * 32 + lane;
+          float s4 = slot[kl] + slot[128 + kl];
+          if (nh == 2) s4 = (s4 + slot[256 + kl]) + slot[384 + kl];
+          const int key = (t0 + lt) * kKeyTile + kl;
+          if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = s4 * p.inv_group;
+        }
       }
     }
   }
