@@ -1,9 +1,9 @@
 #!/usr/bin/env python3
 """Benchmark of the TaskPress compression path on GB300.
 
-One step = the fused per-layer compression (tp_compress_layer: V scales,
-guide scores, per-head top-budget selection, compaction) over every layer of
-the workload, with K/V already resident in HBM.  The metric is context tokens
+One step = the fused compression (V scales, guide scores, per-head
+top-budget selection, compaction) of every layer of the workload in one
+tp_compress_layers call, with K/V already resident in HBM.  The metric is context tokens
 compressed per second per layer (all heads): value = n_tokens * layers / t_step.
 
 Default workload: the Llama-3-8B-shaped 32-layer stack at 128K context with a
@@ -20,6 +20,8 @@ Also reported on the same JSON line:
                 pinned host memory, H2D and D2H copies inside the timed region;
   cpu_baseline  the CPU oracle on a bounded sample of one layer;
   clocks        nvidia-smi samples taken during the timed region;
+  per_layer_calls  the same stack as one tp_compress_layer call per layer;
+  graph_replay  the step's call captured as a CUDA graph and replayed;
   lse_given     the same stack through tp_compress_layer_lse, the row
                 normalisers supplied by the caller (one pass over K);
   literal_normaliser  the same stack through tp_compress_layer_guide (the
@@ -299,6 +301,11 @@ def run_ours(args, w):
                       for n in w.doc_lens) * w.n_heads_kv
 
     def step():
+        # the whole stack in one call: one workspace reset, each layer's first
+        # kernel a programmatic dependent of the previous layer's last
+        binding.tp_compress_layers(p, layers, w.keep_ratio, w.budget, outs, ws, stream)
+
+    def step_layers():
         for (q, k, v), o in zip(layers, outs):
             binding.compress(p, q, k, v, w.keep_ratio, w.budget, o, stream)
 
@@ -363,6 +370,33 @@ def run_ours(args, w):
                 stage_ms[name] += evs[i].elapsed_time(evs[i + 1])
     nstage = reps * nlayer_stage
     stage_ms = {s: v / nstage for s, v in stage_ms.items()}
+
+    # ---- the same stack as one tp_compress_layer call per layer, and the
+    # one-call stack captured into a CUDA graph and replayed
+    for _ in range(args.warmup):
+        step_layers()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step_layers()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms_layers = ev0.elapsed_time(ev1) / args.steps
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        binding.tp_compress_layers(p, layers, w.keep_ratio, w.budget, outs, ws)
+    for _ in range(args.warmup):
+        graph.replay()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        graph.replay()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms_graph = ev0.elapsed_time(ev1) / args.steps
+    del graph
+    per_layer_calls = {"value": w.n_total * L * world / (ms_layers / 1e3), "unit": UNIT,
+                       "ms_per_step": ms_layers, "path": "one tp_compress_layer call per layer"}
+    graph_replay = {"value": w.n_total * L * world / (ms_graph / 1e3), "unit": UNIT,
+                    "ms_per_step": ms_graph, "path": "the tp_compress_layers call captured as a CUDA graph"}
 
     # ---- the single-pass variant: row normalisers supplied by the caller
     # (tp_compress_layer_lse), computed once per layer outside the timed region
@@ -518,7 +552,8 @@ def run_ours(args, w):
                        "l2": "inputs larger than L2 (each layer's K+V exceeds 129 MB; layers use distinct buffers)",
                        "parallelism": f"replicas{world}"},
             "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms,
-            "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk, "lse_given": lse_given,
+            "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk, "per_layer_calls": per_layer_calls,
+            "graph_replay": graph_replay, "lse_given": lse_given,
             "literal_normaliser": literal,
             "cpu_baseline": cpu,
         }

@@ -274,6 +274,23 @@ int tp_compress_layer_guide(const tp_problem* p, const void* q, const void* k, c
                             float* gamma, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * A stack of n_layers layers of one problem in one call (the per-layer path of
+ * tp_compress_layer, layer after layer, on `stream`).  q, k, v, idx, kc, vc,
+ * vqc and gammac are HOST arrays of n_layers device pointers, each laid out as
+ * in tp_compress_layer; kc, vc, vqc and gammac (the arrays, or entries of
+ * them) may be NULL to skip that output.  The workspace is reset once for the
+ * whole stack and layer l's first kernel is launched as a programmatic
+ * dependent of layer l - 1's last one, so consecutive layers overlap at their
+ * boundary.  Results equal n_layers calls of tp_compress_layer.  ws_bytes as
+ * for tp_compress_layer (one layer's workspace serves the whole stack).
+ */
+int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
+                       const void* const* k, const void* const* v, double keep_ratio,
+                       int64_t budget, int32_t* const* idx, void* const* kc, void* const* vc,
+                       int8_t* const* vqc, float* const* gammac, void* ws, size_t ws_bytes,
+                       void* stream);
+
+/*
  * Synchronises `stream`, then reads the device status word that the kernels of
  * the last call on this workspace left.  Every device-side wait in the
  * kernels is bounded; one that gives up records TP_ERR_TIMEOUT there and the

@@ -36,7 +36,7 @@ EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
            "tp_select", "tp_compact",
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
-           "tp_compress_layer_guide", "tp_check_status", "tp_status_string")
+           "tp_compress_layer_guide", "tp_compress_layers", "tp_check_status", "tp_status_string")
 
 
 class TpProblem(ctypes.Structure):
@@ -110,6 +110,10 @@ def load(path: Optional[str] = None):
     lib.tp_guide_prefix_lse.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p]
     lib.tp_compress_layer_guide.restype = c_int
     lib.tp_compress_layer_guide.argtypes = lib.tp_compress_layer_lse.argtypes
+    lib.tp_compress_layers.restype = c_int
+    lib.tp_compress_layers.argtypes = [POINTER(TpProblem), c_int, c_void_p, c_void_p, c_void_p, c_double,
+                                       c_int64, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_void_p, c_size_t, c_void_p]
     lib.tp_check_status.restype = c_int
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
@@ -354,6 +358,37 @@ def tp_compress_layer_guide(p: Problem, q, k, v, k_guide, keep_ratio: float, bud
         _ptr(gammac, torch.float32, m, "gammac", nullable=True),
         _ptr(scores, torch.float32, hkv * n, "scores", nullable=True),
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True),
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_compress_layers(p: Problem, layers, keep_ratio: float, budget: int, outs, ws, stream=None):
+    """A stack of layers in one call.  `layers`: a sequence of (q, k, v) device
+    tensors; `outs`: one CompressOutputs per layer (its idx, kc, vc, vqc and
+    gammac are written; scores and gamma are not)."""
+    import torch
+    n = len(layers)
+    if len(outs) != n:
+        raise ValueError("one CompressOutputs per layer")
+    hq, hkv, d, lt, nt = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+
+    def arr(ptrs):
+        a = (c_void_p * max(1, n))()
+        for i, x in enumerate(ptrs):
+            a[i] = x
+        return a
+
+    q = arr(_ptr(x[0], torch.bfloat16, p.batch * hq * lt * d, "q") for x in layers)
+    k = arr(_ptr(x[1], torch.bfloat16, hkv * nt * d, "k") for x in layers)
+    v = arr(_ptr(x[2], torch.bfloat16, hkv * nt * d, "v") for x in layers)
+    idx = arr(_ptr(o.idx, torch.int32, m, "idx", nullable=cap == 0) for o in outs)
+    kc = arr(_ptr(o.kc, torch.bfloat16, m * d, "kc", nullable=True) for o in outs)
+    vc = arr(_ptr(o.vc, torch.bfloat16, m * d, "vc", nullable=True) for o in outs)
+    vqc = arr(_codes(p, o.vqc, m, "vqc") for o in outs)
+    gc = arr(_ptr(o.gammac, torch.float32, m, "gammac", nullable=True) for o in outs)
+    _check("tp_compress_layers", load().tp_compress_layers(
+        p.ref(), n, q, k, v, keep_ratio, budget, idx, kc, vc, vqc, gc,
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 

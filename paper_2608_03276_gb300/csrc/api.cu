@@ -221,7 +221,7 @@ DocTable doc_table(const Plan& P) {
 // scales of every token into `gamma` when v/gamma are given.  The counters and
 // the status word at the head of the workspace must be zero.
 int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const void* q,
-            const void* v, float* gamma, float* lse, char* ws, cudaStream_t s) {
+            const void* v, float* gamma, float* lse, char* ws, cudaStream_t s, bool dependent = false) {
   CUtensorMap tmv = tmk;
   if (gamma && !encode_3d(&tmv, v, P.d, P.n_total, P.hkv, 128)) return TP_ERR_CUDA;
   int* status = reinterpret_cast<int*>(ws + P.ws_status);
@@ -243,7 +243,8 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
   lp.lse = lse;
   lp.counters = status + 1;
   lp.status = status;
-  return cuda_status(launch_lse(tmk, tmv, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, s));
+  return cuda_status(
+      launch_lse(tmk, tmv, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, dependent, s));
 }
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
@@ -290,12 +291,12 @@ int run_prefix(const Plan& P, const void* q, const void* k_guide, float* lse, bo
 // is given, and the guide prefix folded into the normalisers between them when
 // k_guide is given); leaves the unpooled key scores in the workspace.
 int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
-                cudaStream_t s, const void* k_guide = nullptr) {
+                cudaStream_t s, const void* k_guide = nullptr, bool dependent = false) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
-  int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s);
+  int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s, dependent);
   if (st != TP_OK) return st;
   if (k_guide && (st = run_prefix(P, q, k_guide, lse, true, s)) != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
@@ -629,6 +630,61 @@ int tp_compress_layer_guide(const tp_problem* p, const void* q, const void* k, c
   if (!k_guide || !aligned16(k_guide)) return TP_ERR_INVALID_ARG;
   return compress_layer(p, q, k, v, nullptr, k_guide, keep_ratio, budget, idx, kc, vc, vqc, gammac,
                         scores, gamma, ws, ws_bytes, stream);
+}
+
+int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
+                       const void* const* k, const void* const* v, double keep_ratio,
+                       int64_t budget, int32_t* const* idx, void* const* kc, void* const* vc,
+                       int8_t* const* vqc, float* const* gammac, void* ws, size_t ws_bytes,
+                       void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (n_layers < 0 || (n_layers > 0 && (!q || !k || !v || (!idx && P.cap > 0))))
+    return TP_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!q[l] || !k[l] || !v[l] || !aligned16(q[l]) || !aligned16(k[l]) || !aligned16(v[l]))
+      return TP_ERR_INVALID_ARG;
+    if (P.cap > 0 && !idx[l]) return TP_ERR_INVALID_ARG;
+    if ((kc && kc[l] && !aligned16(kc[l])) || (vc && vc[l] && !aligned16(vc[l])) ||
+        (vqc && vqc[l] && (reinterpret_cast<uintptr_t>(vqc[l]) & code_align(P))))
+      return TP_ERR_INVALID_ARG;
+  }
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  if (n_layers == 0) return TP_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  float* g = reinterpret_cast<float*>(w + P.ws_gamma);
+  // one reset for the whole stack: pass 1 leaves its counters zero again
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
+  for (int l = 0; l < n_layers; ++l) {
+    // layer l's pass 1 is a dependent of layer l - 1's compaction (or of its
+    // selection when nothing is kept): its prologue overlaps that kernel's tail
+    if ((st = run_scoring(P, q[l], k[l], v[l], g, w, s, nullptr, l > 0)) != TP_OK) return st;
+    SelectParams sp;
+    fill_select(P, w, &sp);
+    sp.pool_kernel = p->pool_kernel;
+    sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
+    sp.blend = blend_of(p->flags);
+    sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
+    sp.gamma = g;
+    sp.idx = idx ? idx[l] : nullptr;
+    if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
+    if (P.cap == 0) continue;
+    GatherParams gp;
+    fill_gather(P, &gp);
+    gp.k = static_cast<const uint16_t*>(k[l]);
+    gp.v = static_cast<const uint16_t*>(v[l]);
+    gp.gamma = g;
+    gp.idx = idx[l];
+    gp.kc = kc ? static_cast<uint16_t*>(kc[l]) : nullptr;
+    gp.vc = vc ? static_cast<uint16_t*>(vc[l]) : nullptr;
+    gp.vqc = vqc ? vqc[l] : nullptr;
+    gp.gammac = gammac ? gammac[l] : nullptr;
+    if ((st = cuda_status(launch_gather(gp, true, s))) != TP_OK) return st;
+  }
+  return TP_OK;
 }
 
 int tp_guide_prefix_lse(const tp_problem* p, const void* q, const void* k_guide, float* lse,

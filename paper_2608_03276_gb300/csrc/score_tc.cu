@@ -400,6 +400,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     // cc ^ (row & 7), so eight consecutive rows cover all banks at every step.
     if (with_v) {
       const int vw = warp - kVWarp0;
+      // launched as a dependent of the previous layer's compaction, which may
+      // still read the scale buffer: no store before it has finished
+      grid_dep_wait();
       for (int lt = 0; lt < nt; ++lt) {
         const int vs = lt % kVStages;
         if (!mbar_wait(&full_v[vs], (lt / kVStages) & 1, abort_flag)) break;
@@ -493,6 +496,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   }
   // Every stream has landed and every MMA has finished: the K ring is free.
   __syncthreads();
+  // The workspace partials, normalisers and counters may still be in use by
+  // the previous layer's kernels when this one runs as their dependent.
+  grid_dep_wait();
 
   const bool aborted = *abort_flag != 0;
   if (aborted) {
@@ -522,6 +528,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     if (threadIdx.x == 0) {
       const int prev = atomicAdd(&p.counters[h * p.docs.batch + b], 1);
       *last_flag = (prev == ncta_doc - 1) ? 1 : 0;
+      // every CTA of this (document, head) has counted: the last one leaves the
+      // counter zero again, so the next layer of a stack needs no reset
+      if (prev == ncta_doc - 1) p.counters[h * p.docs.batch + b] = 0;
     }
     __syncthreads();
     if (*last_flag) {
@@ -806,24 +815,34 @@ size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
 
 template <int D, int NRB>
 cudaError_t launch_lse_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
-                         const LseParams& p, dim3 grid, size_t smem, cudaStream_t s) {
+                         const LseParams& p, dim3 grid, size_t smem, bool dependent, cudaStream_t s) {
   cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_lse_kernel<D, NRB>),
                                 1 + (D == 128 ? 3 : 0) + (NRB == 1 ? 0 : NRB == 2 ? 1 : 2));
   if (e != cudaSuccess) return e;
-  tp_lse_kernel<D, NRB><<<grid, kLseThreads, smem, s>>>(tmk, tmv, tmq, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kLseThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, tp_lse_kernel<D, NRB>, tmk, tmv, tmq, p);
 }
 
 cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
-                       const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s) {
+                       const LseParams& p, int head_dim, dim3 grid, size_t smem, bool dependent,
+                       cudaStream_t s) {
   if (head_dim == 128) {
-    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, tmv, tmq, p, grid, smem, s);
-    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, tmv, tmq, p, grid, smem, s);
-    return launch_lse_t<128, 4>(tmk, tmv, tmq, p, grid, smem, s);
+    if (p.nrb == 1) return launch_lse_t<128, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+    if (p.nrb == 2) return launch_lse_t<128, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+    return launch_lse_t<128, 4>(tmk, tmv, tmq, p, grid, smem, dependent, s);
   }
-  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, tmv, tmq, p, grid, smem, s);
-  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, tmv, tmq, p, grid, smem, s);
-  return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, s);
+  if (p.nrb == 1) return launch_lse_t<64, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  if (p.nrb == 2) return launch_lse_t<64, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,

@@ -133,8 +133,12 @@ struct PrefixParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int bits, int num_sms, cudaStream_t s);
+// Pass 1.  `dependent`: launched as a programmatic dependent of the previous
+// layer's last kernel (a stack of layers in one call); it then waits for that
+// kernel before its first store.
 cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
-                       const LseParams& p, int head_dim, dim3 grid, size_t smem, cudaStream_t s);
+                       const LseParams& p, int head_dim, dim3 grid, size_t smem, bool dependent,
+                       cudaStream_t s);
 // `dependent`: launch as a programmatic dependent of the previous kernel in
 // the stream (only where that kernel and this one belong to one layer's
 // sequence, whose inputs were written before its first kernel started).

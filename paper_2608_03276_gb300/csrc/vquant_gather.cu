@@ -77,7 +77,8 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
   const uint4* kin = reinterpret_cast<const uint4*>(p.k);
   const uint4* vin = reinterpret_cast<const uint4*>(p.v);
   const int64_t tok0 = static_cast<int64_t>(h) * p.n_total + p.off[b];
-  grid_dep_wait();  // idx comes from the selection kernel
+  grid_dep_launch();  // the next layer's pass 1 may be scheduled now (it waits before storing)
+  grid_dep_wait();    // idx comes from the selection kernel
   int32_t j[UNR];
   uint4 kv[UNR], vv[UNR];
   float g[UNR];

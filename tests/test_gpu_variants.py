@@ -225,3 +225,68 @@ def test_int4_quantize_v(cuda_lib, name):
     rg, rq = O.quantize_v(x.v, 4)
     assert np.array_equal(g.cpu().numpy().view(np.uint32), rg.view(np.uint32))
     assert np.array_equal(vq.cpu().numpy(), O.pack_codes(rq, 4))
+
+
+# ---------------------------------------------------------------------------
+# A stack of layers in one call (tp_compress_layers) and CUDA-graph capture
+# ---------------------------------------------------------------------------
+def _stack(w, nl):
+    return [synth.make_layer(w, l) for l in range(nl)]
+
+
+def _outputs_equal(a, b, tag):
+    import torch
+    for name in ("idx", "kc", "vc", "vqc", "gammac"):
+        assert torch.equal(getattr(a, name), getattr(b, name)), f"{tag}: {name}"
+
+
+@pytest.mark.parametrize("name,bits", [("c2-llama-4133", 8), ("c5-ragged", 8), ("c1-tiny-2k", 4)])
+def test_layer_stack_matches_single_layers(cuda_lib, name, bits):
+    """tp_compress_layers over three layers (one workspace reset, each layer's
+    pass 1 a dependent of the previous layer's last kernel) equals three
+    tp_compress_layer calls bit for bit, and the oracle on every layer."""
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    xs = _stack(w, 3)
+    p = _problem(binding, w, xs[0].doc_offsets, quant_bits=bits)
+    dev = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in xs]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+    binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, outs[0].ws)
+    assert binding.tp_check_status(outs[0].ws) == 0
+    for l, x in enumerate(xs):
+        single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *dev[l], w.keep_ratio, w.budget, single)
+        _outputs_equal(outs[l], single, f"layer {l}")
+        _check_layer(w, x, single, _oracle(w, x, quant_bits=bits), bits=bits)
+
+
+def test_layer_stack_graph_replay(cuda_lib):
+    """The stack captured into a CUDA graph (its memset and dependent launches
+    become graph nodes) and replayed on new contents of the same input
+    buffers gives the eager results."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL["c3-guide128-2053"]
+    xs = _stack(w, 4)
+    p = _problem(binding, w, xs[0].doc_offsets)
+    bufs = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in xs]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda", with_scores=False) for _ in xs]
+    for o in outs[1:]:
+        o.ws = outs[0].ws
+    binding.tp_compress_layers(p, bufs, w.keep_ratio, w.budget, outs, outs[0].ws)  # eager warm-up
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        binding.tp_compress_layers(p, bufs, w.keep_ratio, w.budget, outs, outs[0].ws)
+    # new contents: the layers in reverse order
+    src = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in reversed(xs)]
+    for dst, s_ in zip(bufs, src):
+        for a, b in zip(dst, s_):
+            a.copy_(b)
+    g.replay()
+    torch.cuda.synchronize()
+    assert binding.tp_check_status(outs[0].ws) == 0
+    for l in range(len(xs)):
+        eager = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *src[l], w.keep_ratio, w.budget, eager)
+        _outputs_equal(outs[l], eager, f"replayed layer {l}")
