@@ -67,10 +67,8 @@ def parse():
 
 
 def dist_env():
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return rank, world, local
+    from paper_2608_03276_gb300 import replicas
+    return replicas.dist_env()
 
 
 def measured_peaks():
@@ -282,14 +280,14 @@ def run_ours(args, w):
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2608_03276_gb300 import binding, synth
+    from paper_2608_03276_gb300 import binding, replicas, synth
 
     hbm_peak, tf_burst, tf_sust, peak_src = measured_peaks()
     stream = torch.cuda.current_stream()
     L = w.layers
     p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, w.doc_offsets())
     # each rank compresses its own stack (weak scaling; no data-path collective)
-    wr = w.with_(seed=w.seed + 7919 * rank)
+    wr = w.with_(seed=replicas.rank_seed(w.seed, rank))
     layers = [synth.make_layer_torch(wr, l, dev) for l in range(L)]
     outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, dev, with_scores=False)
             for _ in range(L)]
@@ -317,8 +315,7 @@ def run_ours(args, w):
         raise RuntimeError(f"device status after warm-up: {binding.tp_status_string(st)}")
 
     # ---- timed region (fused path)
-    if world > 1:
-        dist.barrier()
+    replicas.barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clocks:
@@ -329,14 +326,9 @@ def run_ours(args, w):
         ev1.record(stream)
         torch.cuda.synchronize()
         clocks.mark_end()
-    if world > 1:
-        dist.barrier()
-    ms = ev0.elapsed_time(ev1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = w.n_total * L * world / (ms / 1e3)
+    replicas.barrier()
+    ms = replicas.max_over_ranks(ev0.elapsed_time(ev1) / args.steps, dev)
+    value = replicas.whole_job_value(w.n_total, L, world, ms)
     kernels_per_call = binding.KERNELS_PER_COMPRESS
     gpu_launches = kernels_per_call * L * args.steps
 
@@ -505,8 +497,7 @@ def run_ours(args, w):
     for _ in range(2):
         e2e_step()
     torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
+    replicas.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     s_up.wait_event(e0)
@@ -518,12 +509,8 @@ def run_ours(args, w):
         stream.wait_event(ev_down[l])
     e1.record(stream)
     torch.cuda.synchronize()
-    ems = e0.elapsed_time(e1) / esteps
-    if world > 1:
-        t = torch.tensor([ems], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ems = float(t.item())
-    e2e = {"value": w.n_total * Le * world / (ems / 1e3), "unit": UNIT,
+    ems = replicas.max_over_ranks(e0.elapsed_time(e1) / esteps, dev)
+    e2e = {"value": replicas.whole_job_value(w.n_total, Le, world, ems), "unit": UNIT,
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "layers_per_step": Le,
            "ms_per_step": ems}
 
