@@ -290,3 +290,59 @@ def test_layer_stack_graph_replay(cuda_lib):
         eager = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
         binding.compress(p, *src[l], w.keep_ratio, w.budget, eager)
         _outputs_equal(outs[l], eager, f"replayed layer {l}")
+
+
+# ---------------------------------------------------------------------------
+# Edge shapes for the variants: empty and one-token documents, a 7-token one
+# ---------------------------------------------------------------------------
+EDGE = PREFIX_CASES["ragged-empty"]
+
+
+@pytest.mark.parametrize("variant", ["normadd", "harmonic", "literal", "int4", "stack"])
+def test_variants_on_ragged_edges(cuda_lib, variant):
+    from paper_2608_03276_gb300 import binding
+    w, x = EDGE, synth.make_layer(EDGE)
+    if variant in BLENDS:
+        out = _run_compress(binding, w, x, flags=getattr(binding, BLENDS[variant]))
+        _check_layer(w, x, out, _oracle(w, x, combine_mode=variant))
+    elif variant == "literal":
+        kg = synth.make_guide_keys(w)
+        p = _problem(binding, w, x.doc_offsets)
+        out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, parity.to_device_bf16(x.q), parity.to_device_bf16(x.k),
+                         parity.to_device_bf16(x.v), w.keep_ratio, w.budget, out,
+                         k_guide=parity.to_device_bf16(kg))
+        assert binding.tp_check_status(out.ws) == 0
+        _check_layer(w, x, out, _oracle(w, x, k_guide_bits=kg))
+    elif variant == "int4":
+        out = _run_compress(binding, w, x, quant_bits=4)
+        _check_layer(w, x, out, _oracle(w, x, quant_bits=4), bits=4)
+    else:
+        xs = _stack(w, 2)
+        p = _problem(binding, w, x.doc_offsets)
+        dev = [tuple(parity.to_device_bf16(t) for t in (y.q, y.k, y.v)) for y in xs]
+        outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+        binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, outs[0].ws)
+        assert binding.tp_check_status(outs[0].ws) == 0
+        for l in range(2):
+            single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+            binding.compress(p, *dev[l], w.keep_ratio, w.budget, single)
+            _outputs_equal(outs[l], single, f"layer {l}")
+
+
+def test_full_size_stack(cuda_lib):
+    """Two layers of the 128K Llama-8B-shaped workload through
+    tp_compress_layers, the benchmark's call: layer 0 equals a single-layer call
+    bit for bit, and a sampled head of layer 1 matches the oracle."""
+    from paper_2608_03276_gb300 import binding
+    w = synth.WORKLOADS[3]
+    xs = _stack(w, 2)
+    p = _problem(binding, w, xs[0].doc_offsets)
+    dev = [tuple(parity.to_device_bf16(t) for t in (y.q, y.k, y.v)) for y in xs]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+    binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, outs[0].ws)
+    assert binding.tp_check_status(outs[0].ws) == 0
+    single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+    binding.compress(p, *dev[1], w.keep_ratio, w.budget, single)
+    _outputs_equal(outs[1], single, "layer 1")
+    _check_layer(w, xs[1], single, _oracle(w, xs[1], heads=[6]), heads=[6])
