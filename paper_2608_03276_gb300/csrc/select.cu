@@ -22,6 +22,8 @@
 #include <cooperative_groups.h>
 
 
+#include <cstddef>
+
 #include "tp_device.cuh"
 
 namespace cg = cooperative_groups;
@@ -44,8 +46,12 @@ constexpr int kSliceKeys = 16384;  // keys of a CTA's slice kept in shared memor
 constexpr int kMaxHalf = 16;       // largest pooling half-window of the staging strip
 
 struct SelectSmem {
-  uint32_t keys[kSliceKeys];
-  float strip[kSliceKeys + 2 * kMaxHalf];  // unpooled key scores of a sub-slice + halo
+  uint32_t keys[kSliceKeys + kSliceKeys / 16];  // one padding word after every 16 keys
+  // unpooled key scores of a sub-slice with its halo, and its scales (or given
+  // scores); element g of the global array sits at [g - g_ref] with g_ref a
+  // multiple of 4, so 16-byte groups of the two line up (4 floats of slack)
+  float strip[kSliceKeys + 2 * kMaxHalf + 4];
+  float vals[kSliceKeys + 4];
   int hist1[kBins1];
   int hist2[kBins2];
   int hist3[kBins3];
@@ -57,6 +63,8 @@ struct SelectSmem {
   float norm2[2];  // this CTA's sums of squares of pooled key scores and scales
   float inv_norm[2];
 };
+static_assert(offsetof(SelectSmem, strip) % 16 == 0 && offsetof(SelectSmem, vals) % 16 == 0,
+              "16-byte cp.async destinations must be 16-byte aligned");
 
 // Sum of v over the block in a fixed order (warp trees, then warp totals).
 __device__ __forceinline__ float block_sum_f(float v, float* warp_part) {
@@ -155,12 +163,39 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   return d;
 }
 
+// Stages global floats src[ga, gb) into dst[g - g_ref] (g_ref a multiple of 4,
+// dst 16-byte aligned): 16-byte cp.async over the aligned middle, 4-byte ones
+// at the two ragged ends.  Called by every thread of the block.
+__device__ __forceinline__ void stage_floats(float* dst, const float* src, int64_t ga, int64_t gb,
+                                             int64_t g_ref) {
+  if (gb <= ga) return;
+  const int64_t a4 = (ga + 3) & ~int64_t(3), b4 = gb & ~int64_t(3);
+  // a caller's array need only be 4-byte aligned: then every copy is 4 bytes
+  if (a4 >= b4 || (reinterpret_cast<uintptr_t>(src) & 15) != 0) {
+    for (int64_t g = ga + threadIdx.x; g < gb; g += blockDim.x) cp_async4(dst + (g - g_ref), src + g, true);
+    return;
+  }
+  const int64_t groups = (b4 - a4) >> 2;
+  for (int64_t q = threadIdx.x; q < groups; q += blockDim.x) {
+    const int64_t g = a4 + 4 * q;
+    cp_async16(dst + (g - g_ref), src + g);
+  }
+  const int head = static_cast<int>(a4 - ga), tail = static_cast<int>(gb - b4);
+  if (static_cast<int>(threadIdx.x) < head) {
+    const int64_t g = ga + threadIdx.x;
+    cp_async4(dst + (g - g_ref), src + g, true);
+  } else if (static_cast<int>(threadIdx.x) >= 32 && static_cast<int>(threadIdx.x) < 32 + tail) {
+    const int64_t g = b4 + (threadIdx.x - 32);
+    cp_async4(dst + (g - g_ref), src + g, true);
+  }
+}
+
 // CL: CTAs per (document, head) cluster.  BLEND: how the fused path combines
 // the pooled key score with the scale (a compile-time choice, so the product
 // kernel's per-token loop carries nothing for the other blends).
 template <int CL, int BLEND>
 __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_constant__ SelectParams p) {
-  extern __shared__ uint8_t smem_raw[];
+  extern __shared__ __align__(128) uint8_t smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -176,7 +211,13 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   // the slice's keys: in shared memory when they fit, else in the global scratch
   const bool in_smem = (s1 - s0 <= kSliceKeys);
   uint32_t* const keys_base = in_smem ? sm.keys : p.keys + row;
-  const int kofs = in_smem ? s0 : 0;  // keys of token i live at keys_base[i - kofs]
+  // key of token i: keys_base[kpos(i)].  In shared memory every 16 keys are
+  // followed by a padding word, so the compaction's runs of 16 consecutive
+  // keys per thread start 17 words apart and its reads hit distinct banks.
+  auto kpos = [&](int i) {
+    const int r = in_smem ? i - s0 : i;
+    return in_smem ? r + (r >> 4) : r;
+  };
 
   grid_dep_launch();
   for (int i = threadIdx.x; i < kBins1; i += kThreads) {
@@ -199,71 +240,59 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
     float sa = 0.f, sb = 0.f;
     for (int c0 = s0; c0 < s1; c0 += kSliceKeys) {
       const int c1 = min(c0 + kSliceKeys, s1);
-      // this thread's first round of scale (or score) loads go out before the
-      // key-score strip is staged, so the two global round trips overlap
-      float sv[8];
-      auto load_round = [&](int base) {
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int i = base + u * kThreads + threadIdx.x;
-          sv[u] = 0.f;
-          if (i < c1) sv[u] = p.scores_in ? __ldg(p.scores_in + row + i)
-                                          : (p.key_only ? 1.f : __ldg(p.gamma + row + i));
-        }
-      };
-      load_round(c0);
+      // Every load of the sub-slice goes out at once, straight into shared
+      // memory (cp.async, 16-byte groups where aligned): the key scores with
+      // their halo and the scales (or given scores).  Halo positions outside
+      // the document are zero.  One global round trip per sub-slice.
+      const float* vsrc = p.scores_in ? p.scores_in : (p.key_only ? nullptr : p.gamma);
+      const int64_t g0 = static_cast<int64_t>(row);  // global index of token 0
+      const int64_t sref = (g0 + c0 - half) & ~int64_t(3), vref = (g0 + c0) & ~int64_t(3);
       if (fused) {
-        const float* sk = p.skey + row;
-        const int len = c1 - c0 + 2 * half;
-        for (int j0 = threadIdx.x; j0 < len; j0 += 8 * kThreads) {
-          float v[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {  // eight independent loads in flight
-            const int j = j0 + u * kThreads, i = c0 - half + j;
-            v[u] = (j < len && i >= 0 && i < n) ? __ldg(sk + i) : 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            if (j0 + u * kThreads < len) sm.strip[j0 + u * kThreads] = v[u];
-        }
-        __syncthreads();
+        const int ia = max(c0 - half, 0), ib = min(c1 + half, n);  // halo inside the document
+        stage_floats(sm.strip, p.skey, g0 + ia, g0 + ib, sref);
+        for (int i = c0 - half + static_cast<int>(threadIdx.x); i < c1 + half; i += kThreads)
+          if (i < ia || i >= ib) sm.strip[g0 + i - sref] = 0.f;
       }
-      for (int base = c0; base < c1; base += 8 * kThreads) {
-        if (base != c0) load_round(base);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int i = base + u * kThreads + threadIdx.x;
-          const bool live = i < c1;
-          uint32_t key = 0;
-          if (live) {
-            float sc = sv[u];
-            if (fused) {
-              float acc = 0.f;
-              const float* w = sm.strip + (i - c0);
-              for (int o = 0; o <= 2 * half; ++o) acc += w[o];
-              const float a = acc * inv_k, g = sv[u];
-              if (norms_only) {
-                sa += a * a;
-                sb += g * g;
-                continue;
-              }
-              if (p.key_only) {
-                sc = a;
-              } else if constexpr (BLEND == kBlendNormAdd) {
-                sc = a * inv_na + g * inv_nb;
-              } else if constexpr (BLEND == kBlendHarmonic) {
-                const float den = a + g;
-                sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
-              } else {
-                sc = a * g;
-              }
-              if (p.scores_out) p.scores_out[row + i] = sc;
-            }
-            key = score_key(sc);
-            keys_base[i - kofs] = key;
+      if (vsrc) stage_floats(sm.vals, vsrc, g0 + c0, g0 + c1, vref);
+      cp_async_wait_all();
+      __syncthreads();
+      // four independent keys per trip, so their shared-memory loads overlap
+      const float* vrow = sm.vals + (g0 + c0 - vref);             // token c0 at vrow[0]
+      const float* srow = sm.strip + (g0 + c0 - half - sref);      // token c0's window at srow[0]
+#pragma unroll 4
+      for (int i = c0 + threadIdx.x; i < c1; i += kThreads) {
+        const int r = i - c0;
+        float sc = vsrc ? vrow[r] : 1.f;
+        if (fused) {
+          const float* w = srow + r;
+          float acc;
+          if (half == 2) {  // the default window of five, summed in the same order
+            acc = (((w[0] + w[1]) + w[2]) + w[3]) + w[4];
+          } else {
+            acc = 0.f;
+            for (int o = 0; o <= 2 * half; ++o) acc += w[o];
           }
-          if (!p.scores_only && live) atomicAdd(&sm.hist1[key >> 21], 1);
+          const float a = acc * inv_k, g = sc;
+          if (norms_only) {
+            sa += a * a;
+            sb += g * g;
+            continue;
+          }
+          if (p.key_only) {
+            sc = a;
+          } else if constexpr (BLEND == kBlendNormAdd) {
+            sc = a * inv_na + g * inv_nb;
+          } else if constexpr (BLEND == kBlendHarmonic) {
+            const float den = a + g;
+            sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
+          } else {
+            sc = a * g;
+          }
+          if (p.scores_out) p.scores_out[row + i] = sc;
         }
+        const uint32_t key = score_key(sc);
+        keys_base[kpos(i)] = key;
+        if (!p.scores_only) atomicAdd(&sm.hist1[key >> 21], 1);
       }
       __syncthreads();
     }
@@ -307,19 +336,19 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
     int above;
     const int d1 = cluster_digit<CL>(cluster, sm, sm.hist1, kBins1, kk, &above);
     int need = kk - above;
-    for (int base = s0; base < s1; base += kThreads) {
-      const int i = base + threadIdx.x;
-      const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
-      if (i < s1 && (key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
+#pragma unroll 4
+    for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
+      const uint32_t key = keys_base[kpos(i)];
+      if ((key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
     }
     cluster.sync();
     const int d2 = cluster_digit<CL>(cluster, sm, sm.hist2, kBins2, need, &above);
     need -= above;
     const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
-    for (int base = s0; base < s1; base += kThreads) {
-      const int i = base + threadIdx.x;
-      const uint32_t key = i < s1 ? keys_base[i - kofs] : 0u;
-      if (i < s1 && (key >> 10) == pre) atomicAdd(&sm.hist3[key & 0x3FF], 1);
+#pragma unroll 4
+    for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
+      const uint32_t key = keys_base[kpos(i)];
+      if ((key >> 10) == pre) atomicAdd(&sm.hist3[key & 0x3FF], 1);
     }
     cluster.sync();
     const int d3 = cluster_digit<CL>(cluster, sm, sm.hist3, kBins3, need, &above);
@@ -336,8 +365,9 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   {
     int gt = 0, eq = 0;
     if (kk > 0) {
+#pragma unroll 4
       for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
-        const uint32_t key = keys_base[i - kofs];
+        const uint32_t key = keys_base[kpos(i)];
         if (need_eq < 0 || key > thr) ++gt;
         else if (key == thr) ++eq;
       }
@@ -368,7 +398,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 #pragma unroll
     for (int e = 0; e < kPer; ++e) {
       const int j = j0 + e;
-      kv[e] = j < s1 ? keys_base[j - kofs] : 0u;
+      kv[e] = j < s1 ? keys_base[kpos(j)] : 0u;
       if (j < s1) {
         if (need_eq < 0 || kv[e] > thr) ++ngt;
         else if (kv[e] == thr) ++neq;
