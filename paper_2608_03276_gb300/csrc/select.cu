@@ -55,8 +55,11 @@ struct SelectSmem {
   int hist1[kBins1];
   int hist2[kBins2];
   int hist3[kBins3];
-  int red[kBins1 / 4];  // this CTA's slice of the cluster-summed histogram
-  int red_total;
+  // this CTA's slice of the cluster-summed histogram and its total, one
+  // buffer per digit so that no search overwrites what another CTA may still
+  // be reading from the previous one
+  int red[3][kBins1 / 4];
+  int red_total[3];
   int counts[2];  // (> T, == T) in this CTA's slice
   int scratch[33];
   int result[2];
@@ -108,7 +111,9 @@ __device__ __forceinline__ int ld_dsmem(uint32_t addr) {
 //      (highest bins first), and scans that slice's bins from its owner.
 template <int CL>
 __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const int* local_hist,
-                             int nbins, int need, int* above) {
+                             int nbins, int need, int* above, int level) {
+  int* const red = sm.red[level];
+  int* const red_total = &sm.red_total[level];
   const int rank = static_cast<int>(cluster.block_rank());
   const int slice = nbins / CL;  // at most 512 bins (CL >= 4): one per thread
   if (threadIdx.x < slice) {
@@ -119,22 +124,22 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
     int t = 0;
 #pragma unroll
     for (int r = 0; r < CL; ++r) t += v[r];
-    sm.red[threadIdx.x] = t;
+    red[threadIdx.x] = t;
   }
   __syncthreads();
   if (threadIdx.x < 32) {
     int t = 0;
-    for (int i = threadIdx.x; i < slice; i += 32) t += sm.red[i];
+    for (int i = threadIdx.x; i < slice; i += 32) t += red[i];
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (threadIdx.x == 0) sm.red_total = t;
+    if (threadIdx.x == 0) *red_total = t;
   }
   cluster.sync();  // every slice reduced
   // slice totals, highest slice first, and the slice that holds the target
   if (threadIdx.x == 0) {
     int before = 0, s_hit = 0, s_before = 0;
     for (int r = CL - 1; r >= 0; --r) {
-      const int t = ld_dsmem(dsmem(&sm.red_total, r));
+      const int t = ld_dsmem(dsmem(red_total, r));
       if (before < need && before + t >= need) {
         s_hit = r;
         s_before = before;
@@ -149,7 +154,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   __syncthreads();
   // scan the hit slice's bins, highest first (one bin per thread)
   int cnt = 0;
-  if (threadIdx.x < slice) cnt = ld_dsmem(dsmem(&sm.red[slice - 1 - threadIdx.x], s_hit));
+  if (threadIdx.x < slice) cnt = ld_dsmem(dsmem(&red[slice - 1 - threadIdx.x], s_hit));
   int total;
   const int before = s_before + block_excl_scan(cnt, sm.scratch, &total);
   if (threadIdx.x < slice && before < need && before + cnt >= need) {
@@ -159,7 +164,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   __syncthreads();
   *above = sm.result[1];
   const int d = sm.result[0];
-  cluster.sync();  // no CTA overwrites red / red_total while others still read them
+  __syncthreads();  // sm.result is reused by the next search
   return d;
 }
 
@@ -334,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   int need_eq = -1;  // -1: keep every token of the document
   if (kk > 0 && kk < n) {
     int above;
-    const int d1 = cluster_digit<CL>(cluster, sm, sm.hist1, kBins1, kk, &above);
+    const int d1 = cluster_digit<CL>(cluster, sm, sm.hist1, kBins1, kk, &above, 0);
     int need = kk - above;
 #pragma unroll 4
     for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
@@ -342,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
       if ((key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
     }
     cluster.sync();
-    const int d2 = cluster_digit<CL>(cluster, sm, sm.hist2, kBins2, need, &above);
+    const int d2 = cluster_digit<CL>(cluster, sm, sm.hist2, kBins2, need, &above, 1);
     need -= above;
     const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
 #pragma unroll 4
@@ -351,14 +356,14 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
       if ((key >> 10) == pre) atomicAdd(&sm.hist3[key & 0x3FF], 1);
     }
     cluster.sync();
-    const int d3 = cluster_digit<CL>(cluster, sm, sm.hist3, kBins3, need, &above);
+    const int d3 = cluster_digit<CL>(cluster, sm, sm.hist3, kBins3, need, &above, 2);
     need_eq = need - above;
     thr = (pre << 10) | static_cast<uint32_t>(d3);
   } else {
-    // the cluster-wide barriers must match on every CTA: two per digit search
-    // (three searches) and one after each of the two later histograms
+    // the same cluster-wide barriers as the other branch: one per digit
+    // search (three searches) and one after each of the two later histograms
 #pragma unroll 1
-    for (int i = 0; i < 8; ++i) cluster.sync();
+    for (int i = 0; i < 5; ++i) cluster.sync();
   }
 
   // D: counts of this slice, then prefix over the slices before it
