@@ -77,32 +77,6 @@ __device__ __forceinline__ float2 lse_merge(float2 a, float2 b) {
   return make_float2(m, a.y * ex2(a.x - m) + b.y * ex2(b.x - m));
 }
 
-// Max of 32 values (three-input max, 16 instructions).
-__device__ __forceinline__ float max32(const float (&x)[32]) {
-  float t[11];
-#pragma unroll
-  for (int i = 0; i < 10; ++i) t[i] = fmax3(x[3 * i], x[3 * i + 1], x[3 * i + 2]);
-  t[10] = fmaxf(x[30], x[31]);
-  const float a = fmax3(t[0], t[1], t[2]), b = fmax3(t[3], t[4], t[5]);
-  const float c = fmax3(t[6], t[7], t[8]), d = fmaxf(t[9], t[10]);
-  return fmaxf(fmax3(a, b, c), d);
-}
-
-// sum_i 2^(x_i * c2 + off) for 32 values with packed fma/add into four
-// partial sums (keeps few registers live while the next chunk is in flight).
-__device__ __forceinline__ float sum_exp2(const float (&x)[32], float c2, float off) {
-  float2 a[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                 make_float2(0.f, 0.f)};
-  const float2 cc = make_float2(c2, c2), oo = make_float2(off, off);
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const float2 y = ffma2(make_float2(x[2 * i], x[2 * i + 1]), cc, oo);
-    a[i & 3] = fadd2(a[i & 3], make_float2(ex2(y.x), ex2(y.y)));
-  }
-  const float2 t = fadd2(fadd2(a[0], a[1]), fadd2(a[2], a[3]));
-  return t.x + t.y;
-}
-
 // Value i of a 64-column span held as two 32-register chunks.
 #define TP_X64(i) __uint_as_float((i) < 32 ? ra[(i) & 31] : rb[(i) & 31])
 
@@ -134,8 +108,11 @@ __device__ __forceinline__ float sum_exp2_64(const uint32_t (&ra)[32], const uin
 }
 #undef TP_X64
 
-// lse_chunk (below) for a 64-column span given as two 32-column chunks: one
-// offset decision for all 64 values; columns >= `valid` are masked in place.
+// A 64-column span of a guide row's logits (two 32-column chunks) into the
+// running (offset m, sum z) of pass 1, both in log2 units:
+// z = sum 2^(x*c2 - m).  The offset is refreshed from the exact maximum of the
+// span only when it is unset or the span's sum would leave the safe range
+// (2^64); otherwise no max is computed.  Columns >= `valid` are masked in place.
 __device__ __forceinline__ void lse_chunk64(uint32_t (&ra)[32], uint32_t (&rb)[32], int col0,
                                             int valid, float c2, float& m, float& z) {
   if (valid < col0 + 64) {
@@ -165,39 +142,6 @@ __device__ __forceinline__ void lse_chunk64(uint32_t (&ra)[32], uint32_t (&rb)[3
   }
 }
 
-// One 32-column chunk of a guide row's logits into the running (offset m,
-// sum z) of pass 1, both in log2 units: z = sum 2^(x*c2 - m).  The offset is
-// refreshed from the exact chunk maximum only when it is unset or the chunk
-// sum would leave the safe range (2^64); otherwise no max is computed.
-__device__ __forceinline__ void lse_chunk(const uint32_t (&r)[32], int col0, int valid, float c2,
-                                          float& m, float& z) {
-  float x[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(r[i]);
-  if (valid < col0 + 32) {
-#pragma unroll
-    for (int i = 0; i < 32; ++i)
-      if (col0 + i >= valid) x[i] = -INFINITY;
-  }
-  float s = 0.f;
-  bool exact = (m == -INFINITY);
-  if (!exact) {
-    s = sum_exp2(x, c2, -m);
-    exact = !(s <= 0x1p64f);
-  }
-  if (exact) {
-    const float mn = fmaxf(m, max32(x) * c2);
-    if (mn == -INFINITY) return;
-    s = sum_exp2(x, c2, -mn);
-    z *= ex2(m - mn);
-    m = mn;
-  }
-  z += s;
-  if (z > 0x1p64f) {
-    z *= 0x1p-64f;
-    m += 64.f;
-  }
-}
 
 // One 32-column chunk of a key's logits in pass 2: sum_r 2^(D_r * c2), where
 // the accumulator D already holds logit_r - lse_r / sigma (the row offset
