@@ -98,3 +98,39 @@ def test_null_pointers_rejected_before_any_launch(lib):
     assert cdll.tp_guide_prefix_lse(p.ref(), None, None, None, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_select(p.ref(), None, 0.5, -1, None, None, 0, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_status_string(-5) == b"device-side wait timed out"
+
+
+def test_layer_stack_arguments_rejected_before_any_launch(lib):
+    """tp_compress_layers checks every layer's pointers (present, 16-byte
+    aligned) and the workspace before it enqueues anything.  The addresses
+    below are never dereferenced."""
+    from ctypes import c_void_p
+    cdll = lib.load()
+    p = _prob(lib, [0, 100])
+
+    def arr(*xs):
+        a = (c_void_p * len(xs))()
+        for i, x in enumerate(xs):
+            a[i] = x
+        return a
+
+    good = 0x10000
+    q, k, v, idx = arr(good, good), arr(good, good), arr(good, good), arr(good, good)
+    call = lambda n, q_, k_, v_, idx_, ws, ws_bytes: cdll.tp_compress_layers(
+        p.ref(), n, q_, k_, v_, 0.5, -1, idx_, None, None, None, None, ws, ws_bytes, None)
+    assert call(-1, q, k, v, idx, good, 1 << 30) == lib.TP_ERR_INVALID_ARG
+    assert call(2, None, k, v, idx, good, 1 << 30) == lib.TP_ERR_INVALID_ARG
+    assert call(2, arr(good, None), k, v, idx, good, 1 << 30) == lib.TP_ERR_INVALID_ARG
+    assert call(2, q, arr(good, good + 8), v, idx, good, 1 << 30) == lib.TP_ERR_INVALID_ARG
+    assert call(2, q, k, v, arr(good, None), good, 1 << 30) == lib.TP_ERR_INVALID_ARG
+    assert call(2, q, k, v, idx, None, 1 << 30) == lib.TP_ERR_WORKSPACE
+    assert call(2, q, k, v, idx, good, 16) == lib.TP_ERR_WORKSPACE
+    assert call(0, None, None, None, None, good, 1 << 30) == 0  # an empty stack is a no-op
+
+
+def test_code_buffer_alignment(lib):
+    """b = 4 code buffers need 4-byte alignment, b = 8 ones 8-byte."""
+    cdll = lib.load()
+    for bits, bad in ((8, 0x10004), (4, 0x10002)):
+        p = _prob(lib, [0, 100], quant_bits=bits)
+        assert cdll.tp_quantize_v(p.ref(), 0x10000, bad, 0x10000, None) == lib.TP_ERR_INVALID_ARG
