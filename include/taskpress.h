@@ -134,6 +134,18 @@ size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget
 int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, void* stream);
 
 /*
+ * The Eq. 2 rule for any rows of d bf16 values (for example the compacted K,
+ * which makes the compressed cache fully quantised; the paper's experiments
+ * store both K and V in 4 bits, Sec. 4): scale[r] = max_c |x_rc| / qmax and
+ * codes clamp(rint(x_rc / scale[r]), -qmax, qmax) exactly as tp_quantize_v,
+ * qmax = 2^(quant_bits-1) - 1.  x: [rows, d] bf16, 16-byte aligned;
+ * xq: [rows, d*quant_bits/8] codes out (may be NULL); scale: [rows] fp32 out.
+ * head_dim: 64 or 128; quant_bits: 8 or 4.  No problem description needed.
+ */
+int tp_quantize_rows(const void* x, int64_t rows, int head_dim, int quant_bits, void* xq,
+                     float* scale, void* stream);
+
+/*
  * Combined importance s_i of every context token (Sec. 3.2-3.4):
  *   A = softmax over the context of sigma * Q_guide K^T, per guide row
  *       (the guide-to-context block of the prefill attention map, Sec. 3.2),

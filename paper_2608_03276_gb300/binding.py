@@ -36,7 +36,8 @@ EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
            "tp_select", "tp_compact",
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
-           "tp_compress_layer_guide", "tp_compress_layers", "tp_check_status", "tp_status_string")
+           "tp_compress_layer_guide", "tp_compress_layers", "tp_quantize_rows", "tp_check_status",
+           "tp_status_string")
 
 
 class TpProblem(ctypes.Structure):
@@ -114,6 +115,8 @@ def load(path: Optional[str] = None):
     lib.tp_compress_layers.argtypes = [POINTER(TpProblem), c_int, c_void_p, c_void_p, c_void_p, c_double,
                                        c_int64, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                        c_void_p, c_size_t, c_void_p]
+    lib.tp_quantize_rows.restype = c_int
+    lib.tp_quantize_rows.argtypes = [c_void_p, c_int64, c_int, c_int, c_void_p, c_void_p, c_void_p]
     lib.tp_check_status.restype = c_int
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
@@ -211,6 +214,20 @@ def tp_quantize_v(p: Problem, v, vq, gamma, stream=None):
         p.ref(), _ptr(v, torch.bfloat16, hkv * n * d, "v"),
         _codes(p, vq, hkv * n, "vq"),
         _ptr(gamma, torch.float32, hkv * n, "gamma"), _stream(stream)))
+
+
+def tp_quantize_rows(x, quant_bits: int, xq, scale, stream=None):
+    """Eq. 2 for every row of `x` ([..., d] bf16): per-row scales `scale`
+    ([...] fp32) and codes `xq` ([..., d*quant_bits/8], int8 at 8 bits, uint8
+    two per byte at 4 bits; None to skip)."""
+    import torch
+    d = x.shape[-1]
+    rows = x.numel() // d
+    _check("tp_quantize_rows", load().tp_quantize_rows(
+        _ptr(x, torch.bfloat16, None, "x"), rows, d, quant_bits,
+        _ptr(xq, torch.int8 if quant_bits == 8 else torch.uint8, rows * d * quant_bits // 8, "xq",
+             nullable=True),
+        _ptr(scale, torch.float32, rows, "scale"), _stream(stream)))
 
 
 def tp_guide_scores(p: Problem, q, k, gamma, scores, ws, stream=None):

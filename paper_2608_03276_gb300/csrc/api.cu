@@ -488,6 +488,19 @@ int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, 
                                    static_cast<cudaStream_t>(stream)));
 }
 
+int tp_quantize_rows(const void* x, int64_t rows, int head_dim, int quant_bits, void* xq,
+                     float* scale, void* stream) {
+  if (rows < 0 || (head_dim != 64 && head_dim != 128) || (quant_bits != 8 && quant_bits != 4))
+    return rows < 0 ? TP_ERR_INVALID_ARG : TP_ERR_UNSUPPORTED_SHAPE;
+  if (rows == 0) return TP_OK;
+  if (!x || !scale || !aligned16(x) ||
+      (xq && (reinterpret_cast<uintptr_t>(xq) & (quant_bits == 8 ? 7u : 3u))))
+    return TP_ERR_INVALID_ARG;
+  const float qmax = static_cast<float>((1 << (quant_bits - 1)) - 1);
+  return cuda_status(launch_vquant(static_cast<const uint16_t*>(x), xq, scale, rows, head_dim, qmax,
+                                   quant_bits, num_sms(), static_cast<cudaStream_t>(stream)));
+}
+
 int tp_guide_scores(const tp_problem* p, const void* q, const void* k, const float* gamma,
                     float* scores, void* ws, size_t ws_bytes, void* stream) {
   Plan P;

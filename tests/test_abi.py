@@ -29,7 +29,7 @@ def declared_symbols():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_symbols()
-    assert len(names) == 17, names
+    assert len(names) == 18, names
     assert sorted(lib.EXPORTS) == names
     cdll = lib.load()
     for n in names:
@@ -134,3 +134,15 @@ def test_code_buffer_alignment(lib):
     for bits, bad in ((8, 0x10004), (4, 0x10002)):
         p = _prob(lib, [0, 100], quant_bits=bits)
         assert cdll.tp_quantize_v(p.ref(), 0x10000, bad, 0x10000, None) == lib.TP_ERR_INVALID_ARG
+
+
+def test_quantize_rows_arguments(lib):
+    cdll = lib.load()
+    ok = 0x10000
+    assert cdll.tp_quantize_rows(ok, -1, 128, 8, ok, ok, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_quantize_rows(ok, 10, 96, 8, ok, ok, None) == lib.TP_ERR_UNSUPPORTED_SHAPE
+    assert cdll.tp_quantize_rows(ok, 10, 128, 6, ok, ok, None) == lib.TP_ERR_UNSUPPORTED_SHAPE
+    assert cdll.tp_quantize_rows(ok + 8, 10, 128, 8, ok, ok, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_quantize_rows(ok, 10, 128, 8, ok + 4, ok, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_quantize_rows(ok, 10, 128, 4, ok, None, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_quantize_rows(None, 0, 128, 4, None, None, None) == 0  # nothing to do

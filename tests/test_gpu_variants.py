@@ -346,3 +346,27 @@ def test_full_size_stack(cuda_lib):
     binding.compress(p, *dev[1], w.keep_ratio, w.budget, single)
     _outputs_equal(outs[1], single, "layer 1")
     _check_layer(w, xs[1], single, _oracle(w, xs[1], heads=[6]), heads=[6])
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_fully_quantised_cache(cuda_lib, bits):
+    """The compacted K quantised by tp_quantize_rows (K and V both in b bits,
+    as the paper's experiments store the cache): scales and codes equal the
+    oracle's Eq. 2 on the kept K rows, and unused slots (zero rows) get zero
+    scales and codes."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL["c5-ragged"]
+    x = synth.make_layer(w)
+    out = _run_compress(binding, w, x, quant_bits=bits)
+    shp = tuple(out.kc.shape[:-1])
+    kq = torch.empty(shp + (w.head_dim * bits // 8,), dtype=binding.code_dtype(
+        _problem(binding, w, x.doc_offsets, quant_bits=bits)), device="cuda")
+    ks = torch.empty(shp, dtype=torch.float32, device="cuda")
+    binding.tp_quantize_rows(out.kc, bits, kq, ks)
+    torch.cuda.synchronize()
+    rg, rq = O.quantize_v(parity.bf16_bits(out.kc), bits)
+    assert np.array_equal(ks.cpu().numpy().view(np.uint32), rg.view(np.uint32))
+    assert np.array_equal(kq.cpu().numpy(), O.pack_codes(rq, bits))
+    idx = out.idx.cpu().numpy()
+    assert not ks.cpu().numpy()[idx < 0].any()
