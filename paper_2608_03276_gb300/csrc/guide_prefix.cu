@@ -20,16 +20,30 @@ constexpr int kPrefixThreads = 256;
 constexpr int kRowsPerCta = 32;   // 8 warps x 4 rows
 constexpr int kKeyBlock = 128;    // 32 lanes x 4 keys
 constexpr int kMaxD = 128;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.69314718055994531f;
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// Merge of two (max, sum) pairs of exp terms; an empty pair is (-inf, 0).
-__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
+// Merge of two (max, sum) pairs of base-2 exp terms; an empty pair is (-inf, 0).
+__device__ __forceinline__ void merge_ms2(float& m, float& s, float m2, float s2) {
   const float mm = fmaxf(m, m2);
   if (mm == -INFINITY) return;
-  s = s * expf(m - mm) + s2 * expf(m2 - mm);
+  s = s * ex2(m - mm) + s2 * ex2(m2 - mm);
   m = mm;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
 }
 
 // Stages `count` bf16 rows of d elements (row stride d) into a transposed fp32
@@ -73,7 +87,8 @@ __device__ __forceinline__ void stage_transposed(float* t, int ld, const uint16_
 // lane l keys kb + 4l .. 4l+3 of each key block: per feature c it reads one
 // broadcast float4 of queries and one float4 of keys and does 16 FMAs.  Each
 // lane keeps a running (max, sum) per row over its keys; the lanes merge at
-// the end, and lane 0 folds the result into the row's normaliser.
+// the end, and lane 0 folds the result into the row's normaliser.  All sums
+// are kept in base-2 units (logits times sigma * log2(e)).
 __global__ void __launch_bounds__(kPrefixThreads) tp_prefix_kernel(const __grid_constant__ PrefixParams p) {
   extern __shared__ float4 prefix_smem[];
   float* qs = reinterpret_cast<float*>(prefix_smem);     // [kMaxD][kRowsPerCta]
@@ -93,6 +108,7 @@ __global__ void __launch_bounds__(kPrefixThreads) tp_prefix_kernel(const __grid_
   for (int rr = 0; rr < nrows; ++rr) jmax = max(jmax, (r0 + rr) % lt);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float c2 = p.sigma * kLog2e;
   float m[4], s[4];
   int jrow[4];
 #pragma unroll
@@ -123,33 +139,29 @@ __global__ void __launch_bounds__(kPrefixThreads) tp_prefix_kernel(const __grid_
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[i][e] = fmaf(qa[i], ka[e], acc[i][e]);
     }
+    // This block's terms per row, branch-free: the row's maximum over the
+    // warp, then the sum of 2^(x - max); merged into the running pair.
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
+      float x[4], lm = -INFINITY;
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int key = kb + 4 * lane + e;
-        if (key > jrow[i]) continue;  // causal: guide token j sees keys 0..j
-        const float x = acc[i][e] * p.sigma;
-        if (x > m[i]) {
-          s[i] = s[i] * expf(m[i] - x) + 1.f;
-          m[i] = x;
-        } else {
-          s[i] += expf(x - m[i]);
-        }
+        x[e] = key <= jrow[i] ? acc[i][e] * c2 : -INFINITY;  // causal: keys 0..j
+        lm = fmaxf(lm, x[e]);
       }
-    }
-  }
+      const float bm = warp_max(lm);
+      float ls = 0.f;
+      if (bm != -INFINITY) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, m[i], o);
-      const float s2 = __shfl_xor_sync(0xffffffffu, s[i], o);
-      merge_ms(m[i], s[i], m2, s2);
+        for (int e = 0; e < 4; ++e) ls += ex2(x[e] - bm);
+      }
+      merge_ms2(m[i], s[i], bm, warp_sum(ls));
     }
   }
   grid_dep_wait();  // the context normalisers come from scoring pass 1
   if (lane < 4) {
+    // every lane holds the warp's totals; lane i writes row i
     float mi = m[0], si = s[0];
     int ji = jrow[0];
 #pragma unroll
@@ -161,15 +173,15 @@ __global__ void __launch_bounds__(kPrefixThreads) tp_prefix_kernel(const __grid_
       }
     if (ji >= 0) {
       const size_t at = unit_row0 + r0 + 4 * warp + lane;
-      const float pre = mi + logf(si);  // every row sees at least its own key
+      const float pre = mi + lg2(si);  // every row sees at least its own key
       // an empty document has no context terms (pass 1 writes no normaliser for it)
-      const float ctx = p.off[b + 1] == p.off[b] ? -INFINITY : p.lse[at];
+      const float ctx = p.off[b + 1] == p.off[b] ? -INFINITY : p.lse[at] * kLog2e;
       float out = pre;
       if (ctx != -INFINITY) {
         const float mm = fmaxf(ctx, pre);
-        out = mm + logf(expf(ctx - mm) + expf(pre - mm));
+        out = mm + lg2(ex2(ctx - mm) + ex2(pre - mm));
       }
-      p.lse[at] = out;
+      p.lse[at] = out * kLn2;
     }
   }
 }
