@@ -16,6 +16,8 @@ Also reported on the same JSON line:
                 staged pass of the same workload (the fused call's kernels
                 launched one entry point at a time);
   hbm_fused     algorithmic bytes of the fused layer / its time / HBM peak;
+  kernels       every kernel of the layer against its own bound (CUDA events,
+                staged pass);
   e2e           the same metric through the public API with the inputs in
                 pinned host memory, H2D and D2H copies inside the timed region;
   cpu_baseline  the CPU oracle on a bounded sample of one layer;
@@ -446,6 +448,21 @@ def run_ours(args, w):
                 "per_launch_ms": dom_ms,
                 "flops_per_launch": flops1}
     t_layer_s = ms / L / 1e3
+    # every kernel of the layer against its own bound: the scoring passes
+    # against the tensor peak (one QK^T each; pass 1 also streams V), the
+    # compaction against HBM (kept rows of K and V read, the cache written)
+    d = w.head_dim
+    gather_bytes = kept_tokens * (2 * 2 * d + 2 * 2 * d + d + 4 + 4)
+    kernels = {
+        "tp_lse_kernel": {"ms": stage_ms["lse+vscale"], "bound": "tensor",
+                          "frac": flops1 / (stage_ms["lse+vscale"] / 1e3) / 1e12 / tf_sust,
+                          "hbm_frac": 4 * d * w.n_total * w.n_heads_kv / (stage_ms["lse+vscale"] / 1e3) / 1e9 / hbm_peak},
+        "tp_keyscore_kernel": {"ms": stage_ms["keyscore"], "bound": "tensor",
+                               "frac": flops1 / (stage_ms["keyscore"] / 1e3) / 1e12 / tf_sust},
+        "tp_select_kernel": {"ms": stage_ms["select"], "bound": "latency"},
+        "tp_gather_kernel": {"ms": stage_ms["gather"], "bound": "hbm", "bytes": gather_bytes,
+                             "frac": gather_bytes / (stage_ms["gather"] / 1e3) / 1e9 / hbm_peak},
+    }
     hbm_fused = {"algorithmic_bytes": read_b + write_b, "achieved_gbs": (read_b + write_b) / t_layer_s / 1e9,
                  "peak_gbs": hbm_peak, "frac": (read_b + write_b) / t_layer_s / 1e9 / hbm_peak,
                  "frac_of_nominal_8tbs": (read_b + write_b) / t_layer_s / 8e12,
@@ -538,7 +555,7 @@ def run_ours(args, w):
                        "budget": w.budget if w.budget >= 0 else None,
                        "l2": "inputs larger than L2 (each layer's K+V exceeds 129 MB; layers use distinct buffers)",
                        "parallelism": f"replicas{world}"},
-            "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms,
+            "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms, "kernels": kernels,
             "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk, "per_layer_calls": per_layer_calls,
             "graph_replay": graph_replay, "lse_given": lse_given,
             "literal_normaliser": literal,
