@@ -370,3 +370,34 @@ def test_fully_quantised_cache(cuda_lib, bits):
     assert np.array_equal(kq.cpu().numpy(), O.pack_codes(rq, bits))
     idx = out.idx.cpu().numpy()
     assert not ks.cpu().numpy()[idx < 0].any()
+
+
+@pytest.mark.parametrize("variant", ["caller_lse", "literal", "int4"])
+def test_full_size_variants(cuda_lib, variant):
+    """One 128K layer of the Llama-8B-shaped workload (8 KV heads, guide 128 x
+    GQA 4) through each variant path in the benchmark's configuration; one
+    sampled head against the oracle."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = synth.WORKLOADS[3]
+    x = synth.make_layer(w)
+    heads = [5]
+    dev = tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v))
+    if variant == "int4":
+        out = _run_compress(binding, w, x, quant_bits=4)
+        _check_layer(w, x, out, _oracle(w, x, heads=heads, quant_bits=4), heads=heads, bits=4)
+        return
+    p = _problem(binding, w, x.doc_offsets)
+    out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+    if variant == "caller_lse":
+        lse = torch.empty((w.batch, w.n_heads_kv, w.rows), dtype=torch.float32, device="cuda")
+        ws = torch.empty(binding.tp_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+        binding.tp_guide_lse(p, dev[0], dev[1], lse, ws)
+        binding.compress(p, *dev, w.keep_ratio, w.budget, out, lse=lse)
+        ref = _oracle(w, x, heads=heads, lse=lse.cpu().numpy().astype(np.float64))
+    else:
+        kg = synth.make_guide_keys(w)
+        binding.compress(p, *dev, w.keep_ratio, w.budget, out, k_guide=parity.to_device_bf16(kg))
+        ref = _oracle(w, x, heads=heads, k_guide_bits=kg)
+    assert binding.tp_check_status(out.ws) == 0
+    _check_layer(w, x, out, ref, heads=heads)
