@@ -317,10 +317,19 @@ def run_ours(args, w):
         raise RuntimeError(f"device status after warm-up: {binding.tp_status_string(st)}")
 
     # ---- timed region (fused path)
-    replicas.barrier()
-    torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clocks:
+        # the sampler's start-up pause lets the GPU idle: warm it up again, at
+        # least W steps and 50 ms of work, so a short timed region does not
+        # start on lowered clocks
+        t_warm = time.perf_counter() + 0.05
+        n_warm = 0
+        while n_warm < args.warmup or time.perf_counter() < t_warm:
+            step()
+            torch.cuda.synchronize()
+            n_warm += 1
+        replicas.barrier()
+        torch.cuda.synchronize()
         clocks.mark_start()
         ev0.record(stream)
         for _ in range(args.steps):
