@@ -311,6 +311,16 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
  */
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * Self-test of the failure path: one thread waits, through the same bounded
+ * mbarrier wait every kernel uses, on a barrier that nothing arrives at.
+ * After limit_ns (0 < limit_ns <= 1e9) it gives up, records TP_ERR_TIMEOUT in
+ * the workspace status word (which this call first zeroes) and the kernel
+ * returns normally; tp_check_status(ws, ...) then reports TP_ERR_TIMEOUT and
+ * the context stays usable.  Nothing faults, traps or hangs.
+ */
+int tp_selftest_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream);
+
 /* Human-readable name of a status code (static storage). */
 const char* tp_status_string(int status);
 

@@ -37,7 +37,7 @@ EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v
            "tp_select", "tp_compact",
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
            "tp_compress_layer_guide", "tp_compress_layers", "tp_quantize_rows", "tp_check_status",
-           "tp_status_string")
+           "tp_selftest_wait_timeout", "tp_status_string")
 
 
 class TpProblem(ctypes.Structure):
@@ -117,6 +117,8 @@ def load(path: Optional[str] = None):
                                        c_void_p, c_size_t, c_void_p]
     lib.tp_quantize_rows.restype = c_int
     lib.tp_quantize_rows.argtypes = [c_void_p, c_int64, c_int, c_int, c_void_p, c_void_p, c_void_p]
+    lib.tp_selftest_wait_timeout.restype = c_int
+    lib.tp_selftest_wait_timeout.argtypes = [c_void_p, c_size_t, c_int64, c_void_p]
     lib.tp_check_status.restype = c_int
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
@@ -407,6 +409,14 @@ def tp_compress_layers(p: Problem, layers, keep_ratio: float, budget: int, outs,
     _check("tp_compress_layers", load().tp_compress_layers(
         p.ref(), n, q, k, v, keep_ratio, budget, idx, kc, vc, vqc, gc,
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_selftest_wait_timeout(ws, limit_ns: int, stream=None):
+    """Runs the bounded-wait self-test: the status word of `ws` then reads
+    TP_ERR_TIMEOUT (see tp_check_status)."""
+    import torch
+    _check("tp_selftest_wait_timeout", load().tp_selftest_wait_timeout(
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), int(limit_ns), _stream(stream)))
 
 
 def tp_check_status(ws, stream=None) -> int:

@@ -709,6 +709,14 @@ int tp_guide_prefix_lse(const tp_problem* p, const void* q, const void* k_guide,
   return run_prefix(P, q, k_guide, lse, false, static_cast<cudaStream_t>(stream));
 }
 
+int tp_selftest_wait_timeout(void* ws, size_t ws_bytes, int64_t limit_ns, void* stream) {
+  if (!ws || ws_bytes < sizeof(int) || (reinterpret_cast<uintptr_t>(ws) & 3)) return TP_ERR_WORKSPACE;
+  if (limit_ns <= 0 || limit_ns > 1000000000) return TP_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, sizeof(int), s) != cudaSuccess) return TP_ERR_CUDA;
+  return cuda_status(launch_wait_selftest(static_cast<int*>(ws), static_cast<uint64_t>(limit_ns), s));
+}
+
 int tp_check_status(const void* ws, size_t ws_bytes, void* stream) {
   if (!ws || ws_bytes < sizeof(int)) return TP_ERR_WORKSPACE;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return TP_ERR_CUDA;

@@ -148,6 +148,7 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
+cudaError_t launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once per
 // (kernel slot, device); `slot` names the kernel in a small registry.

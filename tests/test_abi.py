@@ -29,7 +29,7 @@ def declared_symbols():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_symbols()
-    assert len(names) == 18, names
+    assert len(names) == 19, names
     assert sorted(lib.EXPORTS) == names
     cdll = lib.load()
     for n in names:
@@ -146,3 +146,11 @@ def test_quantize_rows_arguments(lib):
     assert cdll.tp_quantize_rows(ok, 10, 128, 8, ok + 4, ok, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_quantize_rows(ok, 10, 128, 4, ok, None, None) == lib.TP_ERR_INVALID_ARG
     assert cdll.tp_quantize_rows(None, 0, 128, 4, None, None, None) == 0  # nothing to do
+
+
+def test_selftest_arguments(lib):
+    cdll = lib.load()
+    assert cdll.tp_selftest_wait_timeout(None, 256, 1000, None) == lib.TP_ERR_WORKSPACE
+    assert cdll.tp_selftest_wait_timeout(0x10000, 2, 1000, None) == lib.TP_ERR_WORKSPACE
+    assert cdll.tp_selftest_wait_timeout(0x10000, 256, 0, None) == lib.TP_ERR_INVALID_ARG
+    assert cdll.tp_selftest_wait_timeout(0x10000, 256, 2_000_000_000, None) == lib.TP_ERR_INVALID_ARG
