@@ -272,9 +272,11 @@ def run_ours(args, w):
     import torch
     import torch.distributed as dist
 
+    from paper_2608_03276_gb300 import replicas
+
     rank, world, local = dist_env()
     if world > 1:
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+        replicas.init("nccl" if torch.cuda.is_available() else "gloo")
     if not torch.cuda.is_available():
         raise SystemExit("bench.py needs a CUDA GPU")
     torch.cuda.set_device(local)
@@ -282,7 +284,7 @@ def run_ours(args, w):
 
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2608_03276_gb300 import binding, replicas, synth
+    from paper_2608_03276_gb300 import binding, synth
 
     hbm_peak, tf_burst, tf_sust, peak_src = measured_peaks()
     stream = torch.cuda.current_stream()

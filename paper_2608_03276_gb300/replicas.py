@@ -20,6 +20,15 @@ def dist_env():
     return rank, world, local
 
 
+def init(backend: str, timeout_s: float = 600.0) -> None:
+    """Joins the replica group.  The timeout bounds every barrier and
+    reduction: a rank that died or hung makes the others' next collective
+    fail within it instead of blocking them."""
+    import datetime
+    import torch.distributed as dist
+    dist.init_process_group(backend, timeout=datetime.timedelta(seconds=timeout_s))
+
+
 def rank_seed(seed: int, rank: int) -> int:
     """Seed of rank `rank`'s replica: every rank compresses different data."""
     return seed + 7919 * rank

@@ -9,6 +9,7 @@ one another.
 """
 import os
 import socket
+import time
 
 import pytest
 
@@ -73,3 +74,42 @@ def test_single_process_defaults(monkeypatch):
     assert replicas.max_over_ranks(12.5) == 12.5
     assert replicas.rank_seed(7, 0) == 7 and replicas.rank_seed(7, 1) != 7
     replicas.barrier()
+
+
+def _dying_worker(rank, world, port, queue):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    from paper_2608_03276_gb300 import replicas
+    replicas.init("gloo", timeout_s=10.0)
+    replicas.barrier()  # step 1: both ranks present
+    if rank == 1:
+        os._exit(3)  # rank 1 dies between steps, with nothing in flight
+    t0 = time.perf_counter()
+    try:
+        replicas.barrier()  # step 2: the survivor must get an error, not block
+        queue.put(("no error", time.perf_counter() - t0))
+    except Exception as e:  # noqa: BLE001 - any collective error is the detection
+        queue.put((type(e).__name__, time.perf_counter() - t0))
+
+
+def test_dead_rank_is_detected():
+    """A rank that exits between steps makes the survivor's next barrier fail
+    within the replica group's timeout instead of blocking it."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_dying_worker, args=(r, 2, port, queue)) for r in range(2)]
+    for p in procs:
+        p.start()
+    try:
+        what, waited = queue.get(timeout=120)
+    finally:
+        for p in procs:
+            p.join(timeout=60)
+            if p.is_alive():
+                p.kill()
+    assert what != "no error"
+    assert waited < 60.0
+    assert procs[1].exitcode == 3
