@@ -71,6 +71,9 @@ extern "C" {
 /* Limits. */
 #define TP_MAX_BATCH 256   /* documents per call                              */
 #define TP_MAX_ROWS 512    /* G * L_t stacked guide rows per KV head          */
+/* TP_MAX_ROWS bounds the guide: at most 512 / G tokens (128 at G = 4, 64 at
+ * G = 8).  Longer guides, such as the 256- and 1024-token guides of the
+ * paper's TTFT study (Sec. 4.2.3), return TP_ERR_UNSUPPORTED_SHAPE. */
 
 /*
  * One layer's compression problem.
@@ -187,9 +190,12 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
  *  - Problems whose pass-1 scratch exceeds 2 MiB are rejected with
  *    TP_ERR_WORKSPACE (typical shapes need well under 1 MiB: about
  *    8 bytes x number of SMs x guide rows, plus 4 bytes per document and head).
- *  - The first call on each device looks up that array's device address
- *    (cudaGetSymbolAddress) with the device current; make that first call
- *    before any stream capture.
+ *  - The first call in each CUDA context looks up that array's device address
+ *    (cudaGetSymbolAddress) with the context current; make that first call
+ *    before any stream capture.  The address is cached by the context's ID
+ *    (cuCtxGetId), checked on every call: cudaDeviceReset or a second
+ *    context on the same device gets its own copy of the array and its own
+ *    lookup, and a reset context's address is never reused.
  *  - All calls share the one array: calls that may overlap on the GPU (other
  *    streams, other threads) race and must be serialised by the caller.
  *  - Nothing is allocated: no cudaMalloc, cudaFree or allocating library call.

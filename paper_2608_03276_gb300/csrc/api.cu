@@ -427,22 +427,77 @@ static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBy
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_static_mu;
-void* g_static_ptr[kMaxDevices];
+// The array's device address belongs to one CUDA context: a context created
+// after cudaDeviceReset, or a second context on the same device, holds its
+// own copy at another address.  Addresses are therefore cached by the
+// context's process-unique ID (cuCtxGetId), never by device number.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
 
-// Device address of g_static_scratch on the current device (host code cannot
-// use the symbol itself as an address), looked up once per device.
-int static_scratch(char** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TP_ERR_CUDA;
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_ptr[dev]) {
-    void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) return TP_ERR_CUDA;
-    g_static_ptr[dev] = ptr;
+struct CtxFns {
+  CtxGetCurrentFn get_current = nullptr;
+  CtxGetIdFn get_id = nullptr;
+};
+
+const CtxFns& ctx_fns() {
+  static std::once_flag once;
+  static CtxFns fns;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      fns.get_current = reinterpret_cast<CtxGetCurrentFn>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      fns.get_id = reinterpret_cast<CtxGetIdFn>(f);
+  });
+  return fns;
+}
+
+constexpr int kStaticCacheSlots = 64;
+std::mutex g_static_mu;
+struct StaticSlot {
+  unsigned long long ctx_id;
+  void* ptr;
+};
+StaticSlot g_static_cache[kStaticCacheSlots];
+int g_static_used = 0;
+
+// ID of the calling thread's current context; when the thread has none yet,
+// the runtime's primary context of the current device is made current first.
+int current_ctx_id(unsigned long long* id) {
+  const CtxFns& fns = ctx_fns();
+  if (!fns.get_current || !fns.get_id) return TP_ERR_CUDA;
+  CUcontext ctx = nullptr;
+  if (fns.get_current(&ctx) != CUDA_SUCCESS) return TP_ERR_CUDA;
+  if (!ctx) {
+    void* ptr = nullptr;  // any runtime call that needs a context binds the primary one
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess) return TP_ERR_CUDA;
+    if (fns.get_current(&ctx) != CUDA_SUCCESS || !ctx) return TP_ERR_CUDA;
   }
-  *out = static_cast<char*>(g_static_ptr[dev]);
+  return fns.get_id(ctx, id) == CUDA_SUCCESS ? TP_OK : TP_ERR_CUDA;
+}
+
+// Device address of g_static_scratch in the current context (host code cannot
+// use the symbol itself as an address): looked up on the first call in each
+// context and cached by context ID.  The ID check runs on every call; it is a
+// query of the driver's context state and needs no device work.
+int static_scratch(char** out) {
+  unsigned long long id = 0;
+  int st = current_ctx_id(&id);
+  if (st != TP_OK) return st;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  for (int i = 0; i < g_static_used; ++i)
+    if (g_static_cache[i].ctx_id == id) {
+      *out = static_cast<char*>(g_static_cache[i].ptr);
+      return TP_OK;
+    }
+  void* ptr = nullptr;
+  if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) return TP_ERR_CUDA;
+  if (g_static_used < kStaticCacheSlots) g_static_cache[g_static_used++] = {id, ptr};
+  *out = static_cast<char*>(ptr);
   return TP_OK;
 }
 

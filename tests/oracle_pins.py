@@ -294,6 +294,57 @@ def pin_key_scores_given_lse(O):
     assert np.allclose(b, a * math.exp(-0.75), rtol=1e-12, atol=0)
 
 
+def pin_layer_given_lse_indexing(O):
+    """compress_layer with caller normalisers: Q = 0 makes every logit 0, so
+    the unpooled key score of document b, head h is (1/G) sum_r exp(-lse[b, h, r]).
+    Two documents x two heads with distinct normalisers: a layer that reads
+    another document's or head's row of lse gives another constant."""
+    hq, hkv, lt, d = 4, 2, 3, 8
+    g = hq // hkv
+    lens = [5, 9]
+    offs = [0, 5, 14]
+    rng = np.random.Generator(np.random.PCG64(21))
+    def b16(x):
+        return (x.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    q = np.zeros((2, hq, lt, d), np.uint16)
+    k = b16(rng.standard_normal((hkv, 14, d)))
+    v = b16(rng.standard_normal((hkv, 14, d)))
+    lse = np.empty((2, hkv, g * lt))
+    for b in range(2):
+        for h in range(hkv):
+            lse[b, h] = np.log(3.0 + 10.0 * b + 4.0 * h + np.arange(g * lt))
+    out = O.compress_layer(q, k, v, offs, n_heads_q=hq, n_heads_kv=hkv, keep_ratio=0.5,
+                           pool_kernel=1, lse=lse)
+    for b in range(2):
+        for h in range(hkv):
+            want = sum(1.0 / (3.0 + 10.0 * b + 4.0 * h + r) for r in range(g * lt)) / g
+            got = out["key"][(b, h)]
+            assert got.shape == (lens[b],)
+            assert np.allclose(got, want, rtol=1e-13, atol=0), (b, h, got[0], want)
+
+
+def pin_kept_count_fixed_budget(O):
+    """A fixed per-(document, head) budget keeps min(budget, n) tokens (Sec. 4
+    "Eviction"); budget -1 falls back to the ratio rule.  A document shorter
+    than the budget keeps all of its tokens."""
+    assert O.kept_count(10, 0.5, 3) == 3
+    assert O.kept_count(10, 0.5, 10) == 10
+    assert O.kept_count(10, 0.5, 25) == 10
+    assert O.kept_count(0, 0.5, 4) == 0
+    assert O.kept_count(10, 0.5, 0) == 0
+    assert O.kept_count(10, 0.3, -1) == 3
+    rng = np.random.Generator(np.random.PCG64(22))
+    def b16(x):
+        return (x.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    q = b16(rng.standard_normal((2, 2, 2, 8)))
+    k = b16(rng.standard_normal((1, 11, 8)))
+    v = b16(rng.standard_normal((1, 11, 8)))
+    out = O.compress_layer(q, k, v, [0, 4, 11], n_heads_q=2, n_heads_kv=1, fixed_budget=6)
+    assert out["k"] == {0: 4, 1: 6}
+    assert list(out["idx"][(0, 0)]) == [0, 1, 2, 3]
+    assert len(out["idx"][(1, 0)]) == 6
+
+
 def pin_literal_lse_closed_form(O):
     """Q = 0: every logit is 0, so row r = (g, j) of the causal prefill map has
     n context terms and j + 1 guide terms: lse_r = log(n + j + 1), rows ordered

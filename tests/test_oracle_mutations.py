@@ -39,6 +39,9 @@ MUTATIONS = {
     "gather ignores the document offset": ("tok = doc_lo + np.asarray(idx, dtype=np.int64)", "tok = np.asarray(idx, dtype=np.int64)"),
     "documents not offset": ("s_key = key_scores(qg, k_all[h, lo:hi], sigma)\n", "s_key = key_scores(qg, k_all[h, 0:n], sigma)\n"),
     "given normaliser added": ("np.exp(x - np.asarray(lse_rows", "np.exp(x + np.asarray(lse_rows"),
+    "given normalisers of document 0": ("key_scores_given_lse(qg, k_all[h, lo:hi], sigma, np.asarray(lse)[b, h])", "key_scores_given_lse(qg, k_all[h, lo:hi], sigma, np.asarray(lse)[0, h])"),
+    "given normalisers of head 0": ("key_scores_given_lse(qg, k_all[h, lo:hi], sigma, np.asarray(lse)[b, h])", "key_scores_given_lse(qg, k_all[h, lo:hi], sigma, np.asarray(lse)[b, 0])"),
+    "fixed budget not clamped to n": ("return int(min(fixed_budget, n))", "return int(fixed_budget)"),
     "given-normaliser scores not averaged over G": ("[:, None]).sum(axis=0) / g", "[:, None]).sum(axis=0)"),
     "guide prefix excludes the token itself": ("x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma", "x = np.concatenate([k_ctx @ qr, k_guide[:j] @ qr]) * sigma"),
     "whole guide, no causal mask": ("x = np.concatenate([k_ctx @ qr, k_guide[: j + 1] @ qr]) * sigma", "x = np.concatenate([k_ctx @ qr, k_guide @ qr]) * sigma"),

@@ -35,10 +35,11 @@ def test_static_scratch_matches_workspace_entry(cuda_lib):
             got_g = torch.full_like(ref_g, float("nan"))
             binding.tp_guide_lse_static(p, q, k, got, v=v, gamma=got_g)
             torch.cuda.synchronize()
+            # the same kernel on the same inputs, its partials merged in a fixed
+            # CTA order: the normalisers must agree bit for bit
             a, b = got.cpu().numpy(), ref.cpu().numpy()
-            live = np.isfinite(b)
-            assert np.all(np.isfinite(a[live]))
-            assert np.abs(a[live] - b[live]).max() <= parity.RTOL
+            assert np.all(np.isfinite(a))
+            assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
             assert np.array_equal(got_g.cpu().numpy().view(np.uint32),
                                   ref_g.cpu().numpy().view(np.uint32))
 
