@@ -342,7 +342,7 @@ def run_ours(args, w):
     replicas.barrier()
     ms = replicas.max_over_ranks(ev0.elapsed_time(ev1) / args.steps, dev)
     value = replicas.whole_job_value(w.n_total, L, world, ms)
-    kernels_per_call = binding.KERNELS_PER_COMPRESS
+    kernels_per_call = binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget, binding.MODE_TWO_PASS)
     gpu_launches = kernels_per_call * L * args.steps
 
     # ---- staged pass: per-kernel CUDA-event times of the same launches

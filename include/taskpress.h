@@ -242,6 +242,12 @@ int tp_compact(const tp_problem* p, const void* k, const void* v, const float* g
  * top-budget selection and compaction, all on `stream` with no host
  * synchronisation.  Outputs as in tp_select and tp_compact; `scores` and
  * `gamma` ([H_kv, N] fp32) are optional outputs (NULL to skip).
+ * Kernels: the normalising pass (which also forms the Eq. 2 scales), then the
+ * key-score pass, which for most problems goes on to select and compact the
+ * kept rows itself; otherwise (a CTA's key range beyond 16384 keys, more
+ * scoring CTAs than SMs, or TP_SCORE_NORM_ADD) a selection kernel and a
+ * compaction kernel follow.  Results are the same either way.
+ * tp_compress_kernel_count says how many kernels a call launches.
  */
 int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,
                       double keep_ratio, int64_t budget, int32_t* idx, void* kc, void* vc,
@@ -307,6 +313,14 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
                        int64_t budget, int32_t* const* idx, void* const* kc, void* const* vc,
                        int8_t* const* vqc, float* const* gammac, void* ws, size_t ws_bytes,
                        void* stream);
+
+/*
+ * How many kernels one fused call launches for this problem (mode 0:
+ * tp_compress_layer, 1: tp_compress_layer_lse, 2: tp_compress_layer_guide;
+ * tp_compress_layers launches mode 0's count per layer); -1 on invalid
+ * arguments.  A planning query: it launches nothing.
+ */
+int tp_compress_kernel_count(const tp_problem* p, double keep_ratio, int64_t budget, int mode);
 
 /*
  * Synchronises `stream`, then reads the device status word that the kernels of

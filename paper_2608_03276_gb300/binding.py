@@ -27,17 +27,13 @@ TP_SCORE_NORM_ADD = 0x2
 TP_SCORE_HARMONIC = 0x4
 TP_MAX_BATCH = 256
 TP_MAX_ROWS = 512
-#: kernels one tp_compress_layer call launches (scoring pass 1 with the V
-#: scales, scoring pass 2, selection, compaction)
-KERNELS_PER_COMPRESS = 4
-
 #: every symbol include/taskpress.h declares
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",
            "tp_select", "tp_compact",
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
            "tp_compress_layer_guide", "tp_compress_layers", "tp_quantize_rows", "tp_check_status",
-           "tp_selftest_wait_timeout", "tp_status_string")
+           "tp_selftest_wait_timeout", "tp_status_string", "tp_compress_kernel_count")
 
 
 class TpProblem(ctypes.Structure):
@@ -123,6 +119,8 @@ def load(path: Optional[str] = None):
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
     lib.tp_status_string.argtypes = [c_int]
+    lib.tp_compress_kernel_count.restype = c_int
+    lib.tp_compress_kernel_count.argtypes = [POINTER(TpProblem), c_double, c_int64, c_int]
     _lib = lib
     return lib
 
@@ -425,6 +423,18 @@ def tp_check_status(ws, stream=None) -> int:
 
 def tp_status_string(status: int) -> str:
     return _status_string(status)
+
+
+#: tp_compress_kernel_count modes
+MODE_TWO_PASS, MODE_CALLER_LSE, MODE_LITERAL = 0, 1, 2
+
+
+def tp_compress_kernel_count(p: Problem, keep_ratio: float, budget: int, mode: int = MODE_TWO_PASS) -> int:
+    """Kernels one fused call launches for this problem (a planning query)."""
+    n = int(load().tp_compress_kernel_count(p.ref(), keep_ratio, budget, mode))
+    if n < 0:
+        raise TaskPressError("tp_compress_kernel_count", TP_ERR_INVALID_ARG)
+    return n
 
 
 class CompressOutputs:

@@ -15,11 +15,14 @@
 //
 // Both passes stream 128-key tiles of K with TMA (128-byte swizzle) through a
 // ring of shared-memory stages; one thread issues the MMAs; four epilogue
-// warpgroups drain TMEM.  Warp roles per CTA (18 warps):
+// warpgroups drain TMEM.  Warp roles per CTA (18 warps; pass 1 has 20):
 //   warp 0  TMEM owner + TMA producer      warp 1  MMA issuer
 //   warps 2-17  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
+//   warps 18-19 (pass 1) Eq. 2 scales of the CTA's V rows from a TMA ring
+// Pass 2 may go on to select and compact the layer's kept rows (tail.cuh).
 #include <math.h>
 
+#include "tail.cuh"
 #include "tp_device.cuh"
 
 namespace tp {
@@ -744,9 +747,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  if (p.tail)
+    keyscore_tail<D>(p, smem, b, h, c, p.docs.cta[b + 1] - p.docs.cta[b], t0, nt, n, doc_lo,
+                     abort_flag);
 }
 
 }  // namespace
+
+size_t tail_smem_bytes() { return sizeof(TailSmem) + 1024; }
 
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
   (void)rows_pad;  // the guide rows live in tensor memory; V has its own ring

@@ -38,10 +38,6 @@ constexpr int kBins1 = 2048;             // bits 31..21
 constexpr int kBins2 = 2048;             // bits 20..10
 constexpr int kBins3 = 1024;             // bits 9..0
 
-__device__ __forceinline__ uint32_t score_key(float s) {
-  return (s > 0.f) ? __float_as_uint(s) : 0u;  // -0, +0, NaN and negatives -> 0
-}
-
 constexpr int kSliceKeys = 16384;  // keys of a CTA's slice kept in shared memory
 constexpr int kMaxHalf = 16;       // largest pooling half-window of the staging strip
 
@@ -166,33 +162,6 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   const int d = sm.result[0];
   __syncthreads();  // sm.result is reused by the next search
   return d;
-}
-
-// Stages global floats src[ga, gb) into dst[g - g_ref] (g_ref a multiple of 4,
-// dst 16-byte aligned): 16-byte cp.async over the aligned middle, 4-byte ones
-// at the two ragged ends.  Called by every thread of the block.
-__device__ __forceinline__ void stage_floats(float* dst, const float* src, int64_t ga, int64_t gb,
-                                             int64_t g_ref) {
-  if (gb <= ga) return;
-  const int64_t a4 = (ga + 3) & ~int64_t(3), b4 = gb & ~int64_t(3);
-  // a caller's array need only be 4-byte aligned: then every copy is 4 bytes
-  if (a4 >= b4 || (reinterpret_cast<uintptr_t>(src) & 15) != 0) {
-    for (int64_t g = ga + threadIdx.x; g < gb; g += blockDim.x) cp_async4(dst + (g - g_ref), src + g, true);
-    return;
-  }
-  const int64_t groups = (b4 - a4) >> 2;
-  for (int64_t q = threadIdx.x; q < groups; q += blockDim.x) {
-    const int64_t g = a4 + 4 * q;
-    cp_async16(dst + (g - g_ref), src + g);
-  }
-  const int head = static_cast<int>(a4 - ga), tail = static_cast<int>(gb - b4);
-  if (static_cast<int>(threadIdx.x) < head) {
-    const int64_t g = ga + threadIdx.x;
-    cp_async4(dst + (g - g_ref), src + g, true);
-  } else if (static_cast<int>(threadIdx.x) >= 32 && static_cast<int>(threadIdx.x) < 32 + tail) {
-    const int64_t g = b4 + (threadIdx.x - 32);
-    cp_async4(dst + (g - g_ref), src + g, true);
-  }
 }
 
 // CL: CTAs per (document, head) cluster.  BLEND: how the fused path combines
