@@ -14,18 +14,23 @@ and consecutive layers use different buffers, so no L2 flush is needed.
 Also reported on the same JSON line:
   roofline      the dominant kernel, timed per launch with CUDA events over a
                 staged pass of the same workload (the fused call's kernels
-                launched one entry point at a time);
+                launched one entry point at a time), against the burst tensor
+                peak (a kernel timed alone);
   hbm_fused     algorithmic bytes of the fused layer / its time / HBM peak;
   kernels       every kernel of the layer against its own bound (CUDA events,
                 staged pass);
+  workload_legs the other workloads of the metric, each through the same
+                call: the 32K Llama layer, the 64K wide-GQA layer at its four
+                keep ratios and the ragged 8-document batch (value, hbm_fused,
+                staged kernel times);
   e2e           the same metric through the public API with the inputs in
                 pinned host memory, H2D and D2H copies inside the timed region;
-  cpu_baseline  the CPU oracle on a bounded sample of one layer;
+  cpu_baseline  the CPU oracle on every host core (a bounded sample of layer 0);
   clocks        nvidia-smi samples taken during the timed region;
   per_layer_calls  the same stack as one tp_compress_layer call per layer;
   graph_replay  the step's call captured as a CUDA graph and replayed;
   lse_given     the same stack through tp_compress_layer_lse, the row
-                normalisers supplied by the caller (one pass over K);
+                normalisers supplied by the caller (one scoring pass over K);
   literal_normaliser  the same stack through tp_compress_layer_guide (the
                 guide's causal prefix folded into the normalisers).
 
@@ -64,7 +69,7 @@ def parse():
     ap.add_argument("--layers", type=int, default=0, help="override the workload's layer count")
     ap.add_argument("--e2e-layers", type=int, default=4)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-sample-heads", type=int, default=0, help="0: every KV head of one layer")
+    ap.add_argument("--no-legs", action="store_true", help="skip the 32K / 64K / ragged workload legs")
     return ap.parse_args()
 
 
@@ -198,68 +203,122 @@ def traffic_record(kernel: str, workload: str):
 # ---------------------------------------------------------------------------
 # CPU oracle sample (the cpu_baseline leg and the reference arm)
 # ---------------------------------------------------------------------------
+def cpu_model() -> str:
+    """The host CPU's model name (x86 'model name', Arm 'CPU part' or lscpu)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu part")):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def _oracle_worker_init():
+    os.environ["OPENBLAS_NUM_THREADS"] = "1"
+    os.environ["OMP_NUM_THREADS"] = "1"
+    import numpy  # noqa: F401  (import cost outside the timed map)
+    from oracle import taskpress_oracle  # noqa: F401
+
+
 def _oracle_unit(args):
-    q, k, v, g, n_heads_q, keep_ratio, budget = args
+    """One (document 0, KV head) unit of the oracle: the whole per-head path
+    (Eq. 2 scales, both scoring passes in fp64, pooling, full sort, gather)."""
+    qf, kf, vf, g, keep_ratio, budget = args
+    import numpy as np
     from oracle import taskpress_oracle as O
+    q, k, v = np.load(qf), np.load(kf, mmap_mode="r"), np.load(vf, mmap_mode="r")
     t0 = time.perf_counter()
-    O.compress_layer(q, k, v, [0, k.shape[1]], n_heads_q=g, n_heads_kv=1,
-                     keep_ratio=keep_ratio, fixed_budget=budget)
+    out = O.compress_layer(q, k, v, [0, k.shape[1]], n_heads_q=g, n_heads_kv=1,
+                           keep_ratio=keep_ratio, fixed_budget=budget)
+    O.gather_rows(k, v, out["gamma"], out["vq"], 0, 0, out["idx"][(0, 0)])
     return time.perf_counter() - t0
 
 
-def oracle_inputs(w):
-    """Host inputs of layer 0, document 0 of the workload (what the oracle sample sees)."""
-    from paper_2608_03276_gb300 import synth
-    one_doc = w.with_(doc_lens=(w.doc_lens[0],))
-    return one_doc, synth.make_layer(one_doc)
+class OracleSample:
+    """The CPU oracle on every host core: document 0 of layer 0 of the workload
+    is split into its KV heads, and each of the nproc worker processes (spawned
+    before any timing, BLAS single-threaded) compresses one head; with more
+    cores than heads, heads are repeated.  value = tokens x (units / H_kv) /
+    wall, i.e. context tokens compressed per second per layer."""
+
+    def __init__(self, w, cores=None):
+        import multiprocessing as mp
+        import numpy as np
+        from paper_2608_03276_gb300 import synth
+        self.w = w
+        self.cores = cores or os.cpu_count() or 1
+        one_doc = w.with_(doc_lens=(w.doc_lens[0],))
+        x = synth.make_layer(one_doc)
+        self.n = one_doc.n_total
+        self.tmp = tempfile.mkdtemp(prefix="tp_oracle_")
+        g = w.group
+        files = []
+        for h in range(w.n_heads_kv):
+            fq, fk, fv = (os.path.join(self.tmp, f"{t}{h}.npy") for t in "qkv")
+            np.save(fq, np.ascontiguousarray(x.q[:, h * g:(h + 1) * g]))
+            np.save(fk, np.ascontiguousarray(x.k[h:h + 1]))
+            np.save(fv, np.ascontiguousarray(x.v[h:h + 1]))
+            files.append((fq, fk, fv))
+        self.units = [files[i % w.n_heads_kv] + (g, w.keep_ratio, w.budget)
+                      for i in range(self.cores)]
+        self.pool = mp.get_context("spawn").Pool(processes=self.cores, initializer=_oracle_worker_init)
+        self.pool.map(_oracle_worker_init_probe, range(self.cores))  # every worker is up
+
+    def run(self):
+        t0 = time.perf_counter()
+        per_unit = self.pool.map(_oracle_unit, self.units, chunksize=1)
+        wall = time.perf_counter() - t0
+        layers = len(self.units) / self.w.n_heads_kv
+        value = self.n * layers / wall
+        detail = (f"{self.w.name}: document 0 of layer 0 (n={self.n}), {len(self.units)} (KV head) "
+                  f"units = {layers:g} layer(s) of {self.w.n_heads_kv} heads on {self.cores} "
+                  f"processes (one unit each, heads repeated when cores > heads), fp64 numpy; "
+                  f"wall {wall:.1f}s, CPU {sum(per_unit):.1f}s")
+        return value, detail
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+        import shutil
+        shutil.rmtree(self.tmp, ignore_errors=True)
 
 
-def oracle_sample(w, sample, heads, workers):
-    """Times the oracle on `heads` KV heads of layer 0 of document 0 (one
-    process per head, BLAS single-threaded).  Returns (tokens/s/layer, detail, cores)."""
-    import multiprocessing as mp
-    one_doc, x = sample
-    n = one_doc.n_total
-    g = w.group
-    units = [(x.q[:, h * g:(h + 1) * g].copy(), x.k[h:h + 1].copy(), x.v[h:h + 1].copy(), g, g,
-              w.keep_ratio, w.budget) for h in heads]
-    os.environ["OPENBLAS_NUM_THREADS"] = "1"
-    os.environ["OMP_NUM_THREADS"] = "1"
-    ctx = mp.get_context("spawn")
-    t0 = time.perf_counter()
-    with ctx.Pool(processes=min(workers, len(units))) as pool:
-        per_unit = pool.map(_oracle_unit, units)
-    wall = time.perf_counter() - t0
-    # heads of one layer are independent: the sample covers len(heads)/H_kv of a layer
-    frac = len(heads) / w.n_heads_kv
-    value = n * frac / wall
-    detail = (f"layer 0 of {w.name}: {len(heads)} of {w.n_heads_kv} KV heads of document 0 "
-              f"(n={n}), one process per head, fp64 numpy; wall {wall:.1f}s, "
-              f"CPU {sum(per_unit):.1f}s")
-    return value, detail, min(workers, len(units))
+def _oracle_worker_init_probe(_):
+    return os.getpid()
 
 
 def run_reference(args, w):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    cores = os.cpu_count() or 1
+    sample = OracleSample(w)
     times = []
-    heads = list(range(min(w.n_heads_kv, cores)))
-    sample = oracle_inputs(w)
-    for i in range(args.warmup + args.steps):
-        v, detail, used = oracle_sample(w, sample, heads, cores)
-        if i >= args.warmup:
-            times.append(v)
+    detail = ""
+    try:
+        for i in range(args.warmup + args.steps):
+            v, detail = sample.run()
+            if i >= args.warmup:
+                times.append(v)
+    finally:
+        sample.close()
     value = statistics.median(times)
-    n_units = len(heads)
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "layers_sampled": 1, "heads_sampled": n_units},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": used, "kind": "oracle",
-                         "sample": detail},
+        "config": {"workload": w.name, "layers_sampled": 1, "heads_sampled": w.n_heads_kv},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": sample.cores, "kind": "oracle",
+                         "cpu_model": cpu_model(), "sample": detail},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
@@ -267,6 +326,108 @@ def run_reference(args, w):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+def kept_tokens_of(w, binding, keep_ratio=None):
+    r = w.keep_ratio if keep_ratio is None else keep_ratio
+    return sum(int(min(w.budget, n)) if w.budget >= 0 else binding.tp_budget(int(n), r)
+               for n in w.doc_lens) * w.n_heads_kv
+
+
+def hbm_fused_of(w, kept_tokens, t_layer_s, hbm_peak, peak_src):
+    """Algorithmic bytes of one layer (K + V read once, the compressed cache
+    written once, the guide read once) over the layer's time, against HBM."""
+    read_b, write_b, _ = layer_algorithmic(w, kept_tokens)
+    ach = (read_b + write_b) / t_layer_s / 1e9
+    return {"algorithmic_bytes": read_b + write_b, "achieved_gbs": ach, "peak_gbs": hbm_peak,
+            "frac": ach / hbm_peak, "frac_of_nominal_8tbs": ach * 1e9 / 8e12,
+            "peak_source": f"{peak_src} copy bandwidth"}
+
+
+def staged_times(binding, torch, p, w, layers, outs, ws, stream, reps, keep_ratio=None):
+    """Per-kernel CUDA-event times, one entry point at a time on the launching
+    stream: pass 1 with the Eq. 2 scales (tp_guide_lse), pass 2 (tp_guide_key_scores),
+    the selection (tp_select) and the compaction (tp_compact) as standalone kernels."""
+    dev = outs[0].idx.device
+    r = w.keep_ratio if keep_ratio is None else keep_ratio
+    lse = torch.empty((w.batch, w.n_heads_kv, w.rows), dtype=torch.float32, device=dev)
+    skey = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    gamma = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    scores = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
+    names = ["lse+vscale", "keyscore", "select", "gather"]
+    acc = {s: 0.0 for s in names}
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    nl = min(len(layers), 8)
+    for _ in range(max(1, reps)):
+        for li in range(nl):
+            (q, k, v), o = layers[li], outs[li]
+            binding.tp_guide_scores(p, q, k, gamma, scores, ws, stream)  # scores for select; not timed
+            evs[0].record(stream)
+            binding.tp_guide_lse(p, q, k, lse, ws, stream, v=v, gamma=gamma)
+            evs[1].record(stream)
+            binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
+            evs[2].record(stream)
+            binding.tp_select(p, scores, r, w.budget, o.idx, ws, stream)
+            evs[3].record(stream)
+            binding.tp_compact(p, k, v, gamma, o.idx, r, w.budget, o.kc, o.vc, o.vqc, o.gammac, stream)
+            evs[4].record(stream)
+            torch.cuda.synchronize()
+            for i, name in enumerate(names):
+                acc[name] += evs[i].elapsed_time(evs[i + 1])
+    n = max(1, reps) * nl
+    return {s: v / n for s, v in acc.items()}
+
+
+def time_calls(torch, fn, steps, warmup, stream):
+    for _ in range(warmup):
+        fn()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def workload_leg(binding, torch, synth, w, n_layers, args, dev, stream, hbm_peak, peak_src,
+                 keep_ratios=None):
+    """Another workload of the metric (32K layer, 64K wide-GQA layer, ragged
+    batch): tp_compress_layers over n_layers distinct layers per step (their
+    K + V exceed L2 together), plus the staged per-kernel times."""
+    L = n_layers
+    p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, w.doc_offsets())
+    layers = [synth.make_layer_torch(w, l, dev) for l in range(L)]
+    out = {"workload": w.name, "n_ctx": w.n_total, "layers_per_step": L, "docs": w.batch,
+           "guide_len": w.guide_len, "heads_q": w.n_heads_q, "heads_kv": w.n_heads_kv}
+    legs = {}
+    for r in (keep_ratios or (w.keep_ratio,)):
+        outs = [binding.CompressOutputs(p, r, w.budget, dev, with_scores=False) for _ in range(L)]
+        ws = outs[0].ws
+        for o in outs[1:]:
+            o.ws = ws
+
+        def step():
+            binding.tp_compress_layers(p, layers, r, w.budget, outs, ws, stream)
+
+        steps = max(args.steps, 20)
+        ms = time_calls(torch, step, steps, max(args.warmup, 3), stream)
+        st = binding.tp_check_status(ws)
+        if st != 0:
+            raise RuntimeError(f"{w.name}: device status {binding.tp_status_string(st)}")
+        kept = kept_tokens_of(w, binding, r)
+        t_layer = ms / L / 1e3
+        legs[f"keep_{r:g}" if w.budget < 0 else f"budget_{w.budget}"] = {
+            "value": w.n_total / t_layer, "unit": UNIT, "ms_per_layer": ms / L,
+            "hbm_fused": hbm_fused_of(w, kept, t_layer, hbm_peak, peak_src),
+            "stages_ms": staged_times(binding, torch, p, w, layers, outs, ws, stream, 3, r),
+            "kernels_per_layer": binding.tp_compress_kernel_count(p, r, w.budget, binding.MODE_TWO_PASS)}
+        del outs, ws
+    out["results"] = legs
+    del layers
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args, w):
     import numpy as np
     import torch
@@ -347,34 +508,7 @@ def run_ours(args, w):
 
     # ---- staged pass: per-kernel CUDA-event times of the same launches
     rows = w.rows
-    lse = torch.empty((w.batch, w.n_heads_kv, rows), dtype=torch.float32, device=dev)
-    skey = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
-    gamma = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
-    scores = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
-    stage_names = ["lse+vscale", "keyscore", "select", "gather"]
-    stage_ms = {s: 0.0 for s in stage_names}
-    reps = max(1, args.steps)
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
-    nlayer_stage = min(L, 8)
-    for _ in range(reps):
-        for li in range(nlayer_stage):
-            (q, k, v), o = layers[li], outs[li]
-            binding.tp_guide_scores(p, q, k, gamma, scores, ws, stream)  # scores for select; not timed
-            evs[0].record(stream)
-            binding.tp_guide_lse(p, q, k, lse, ws, stream, v=v, gamma=gamma)
-            evs[1].record(stream)
-            binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
-            evs[2].record(stream)
-            binding.tp_select(p, scores, w.keep_ratio, w.budget, o.idx, ws, stream)
-            evs[3].record(stream)
-            binding.tp_compact(p, k, v, gamma, o.idx, w.keep_ratio, w.budget, o.kc, o.vc, o.vqc,
-                               o.gammac, stream)
-            evs[4].record(stream)
-            torch.cuda.synchronize()
-            for i, name in enumerate(stage_names):
-                stage_ms[name] += evs[i].elapsed_time(evs[i + 1])
-    nstage = reps * nlayer_stage
-    stage_ms = {s: v / nstage for s, v in stage_ms.items()}
+    stage_ms = staged_times(binding, torch, p, w, layers, outs, ws, stream, args.steps)
 
     # ---- the same stack as one tp_compress_layer call per layer, and the
     # one-call stack captured into a CUDA graph and replayed
@@ -425,7 +559,11 @@ def run_ours(args, w):
     ms_lse = ev0.elapsed_time(ev1) / args.steps
     lse_given = {"value": w.n_total * L * world / (ms_lse / 1e3), "unit": UNIT,
                  "ms_per_step": ms_lse,
-                 "path": "tp_compress_layer_lse: caller row normalisers, one pass over K"}
+                 "hbm_fused": hbm_fused_of(w, kept_tokens, ms_lse / L / 1e3, hbm_peak, peak_src),
+                 "kernels_per_layer": binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget,
+                                                                       binding.MODE_CALLER_LSE),
+                 "path": "tp_compress_layer_lse: caller row normalisers, one scoring pass over K, "
+                         "V scales from the quantiser pass"}
     del lses
 
     # ---- the literal normaliser: guide keys given (tp_compress_layer_guide)
@@ -444,6 +582,7 @@ def run_ours(args, w):
     torch.cuda.synchronize()
     ms_lit = ev0.elapsed_time(ev1) / args.steps
     literal = {"value": w.n_total * L * world / (ms_lit / 1e3), "unit": UNIT, "ms_per_step": ms_lit,
+               "hbm_fused": hbm_fused_of(w, kept_tokens, ms_lit / L / 1e3, hbm_peak, peak_src),
                "path": "tp_compress_layer_guide: guide prefix folded into the normalisers"}
     del kgs
 
@@ -452,32 +591,42 @@ def run_ours(args, w):
     dom_ms = stage_ms[dom]
     achieved = flops1 / (dom_ms / 1e3) / 1e12
     kname = {"lse+vscale": "tp_lse_kernel", "keyscore": "tp_keyscore_kernel"}[dom]
+    # the staged times are single launches timed alone: the burst tensor peak applies
     roofline = {"bound": "tensor", "kernel": kname, "achieved": achieved,
-                "peak": tf_sust, "unit": "TFLOP/s", "frac": achieved / tf_sust,
-                "peak_source": f"{peak_src} bf16 sustained",
+                "peak": tf_burst, "unit": "TFLOP/s", "frac": achieved / tf_burst,
+                "peak_source": f"{peak_src} bf16 burst (the kernel is timed alone, per launch)",
+                "frac_of_sustained": achieved / tf_sust,
                 "traffic": traffic_record(kname, w.name),
                 "per_launch_ms": dom_ms,
                 "flops_per_launch": flops1}
     t_layer_s = ms / L / 1e3
     # every kernel of the layer against its own bound: the scoring passes
-    # against the tensor peak (one QK^T each; pass 1 also streams V), the
-    # compaction against HBM (kept rows of K and V read, the cache written)
+    # against the burst tensor peak (one QK^T each; pass 1 also streams V),
+    # the compaction against HBM (kept rows of K and V read, the cache written)
     d = w.head_dim
     gather_bytes = kept_tokens * (2 * 2 * d + 2 * 2 * d + d + 4 + 4)
     kernels = {
         "tp_lse_kernel": {"ms": stage_ms["lse+vscale"], "bound": "tensor",
-                          "frac": flops1 / (stage_ms["lse+vscale"] / 1e3) / 1e12 / tf_sust,
+                          "frac": flops1 / (stage_ms["lse+vscale"] / 1e3) / 1e12 / tf_burst,
                           "hbm_frac": 4 * d * w.n_total * w.n_heads_kv / (stage_ms["lse+vscale"] / 1e3) / 1e9 / hbm_peak},
         "tp_keyscore_kernel": {"ms": stage_ms["keyscore"], "bound": "tensor",
-                               "frac": flops1 / (stage_ms["keyscore"] / 1e3) / 1e12 / tf_sust},
+                               "frac": flops1 / (stage_ms["keyscore"] / 1e3) / 1e12 / tf_burst},
         "tp_select_kernel": {"ms": stage_ms["select"], "bound": "latency"},
-        "tp_gather_kernel": {"ms": stage_ms["gather"], "bound": "hbm", "bytes": gather_bytes,
-                             "frac": gather_bytes / (stage_ms["gather"] / 1e3) / 1e9 / hbm_peak},
+        "tp_gather_kernel": {"ms": stage_ms["gather"], "bound": "hbm", "bytes_touched": gather_bytes,
+                             "touched_frac": gather_bytes / (stage_ms["gather"] / 1e3) / 1e9 / hbm_peak,
+                             "note": "bytes the kernel reads and writes (kept K and V rows, the cache); "
+                                     "part of the writes is absorbed by L2 and reaches DRAM after the "
+                                     "kernel, so this is a throughput of bytes touched, not DRAM bandwidth"},
     }
-    hbm_fused = {"algorithmic_bytes": read_b + write_b, "achieved_gbs": (read_b + write_b) / t_layer_s / 1e9,
-                 "peak_gbs": hbm_peak, "frac": (read_b + write_b) / t_layer_s / 1e9 / hbm_peak,
-                 "frac_of_nominal_8tbs": (read_b + write_b) / t_layer_s / 8e12,
-                 "peak_source": peak_src}
+    fused_tail_ms = ms / L - stage_ms["lse+vscale"] - stage_ms["keyscore"]
+    hbm_fused = hbm_fused_of(w, kept_tokens, t_layer_s, hbm_peak, peak_src)
+
+    legs = {}
+    if rank == 0 and not args.no_legs and args.config == 3:
+        for cfg, nl, ratios in ((2, 4, None), (4, 4, (0.05, 0.10, 0.25, 0.50)), (5, 2, None)):
+            legs[synth.WORKLOADS[cfg].name] = workload_leg(
+                binding, torch, synth, synth.WORKLOADS[cfg].with_(seed=replicas.rank_seed(synth.WORKLOADS[cfg].seed, rank)),
+                nl, args, dev, stream, hbm_peak, peak_src, ratios)
 
     # ---- e2e: host buffers through the public API, copies inside the timed region
     Le = max(1, min(args.e2e_layers, L))
@@ -549,11 +698,13 @@ def run_ours(args, w):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cores = os.cpu_count() or 1
-        nh = args.cpu_sample_heads or w.n_heads_kv
-        heads = list(range(min(nh, w.n_heads_kv)))
-        cv, detail, used = oracle_sample(w, oracle_inputs(w), heads, cores)
-        cpu = {"value": cv, "unit": UNIT, "cores": used, "kind": "oracle", "sample": detail}
+        sample = OracleSample(w)
+        try:
+            cv, detail = sample.run()
+        finally:
+            sample.close()
+        cpu = {"value": cv, "unit": UNIT, "cores": sample.cores, "cpu_model": cpu_model(),
+               "kind": "oracle", "sample": detail}
 
     if rank == 0:
         line = {
@@ -567,6 +718,9 @@ def run_ours(args, w):
                        "l2": "inputs larger than L2 (each layer's K+V exceeds 129 MB; layers use distinct buffers)",
                        "parallelism": f"replicas{world}"},
             "roofline": roofline, "hbm_fused": hbm_fused, "stages_ms": stage_ms, "kernels": kernels,
+            "fused_layer_ms": ms / L, "kernels_per_layer": kernels_per_call,
+            "layer_minus_scoring_passes_ms": fused_tail_ms,
+            "workload_legs": legs,
             "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk, "per_layer_calls": per_layer_calls,
             "graph_replay": graph_replay, "lse_given": lse_given,
             "literal_normaliser": literal,

@@ -20,3 +20,19 @@ def cuda_lib():
         pytest.fail("GPU test run without a CUDA device")
     from paper_2608_03276_gb300 import binding
     return binding.load()
+
+
+def pytest_terminal_summary(terminalreporter):
+    """Worst relative score error and near-tie kept-set differences of every
+    parity test that compared scores with the oracle (tests/parity.py)."""
+    from tests import parity
+    if not parity.STATS:
+        return
+    tr = terminalreporter
+    tr.section("parity margins (bar: rel err <= 2e-3; kept sets equal outside near-ties)")
+    worst = 0.0
+    for test, st in sorted(parity.STATS.items()):
+        worst = max(worst, st["max_rel"])
+        tr.write_line(f"{test}: max rel err {st['max_rel']:.2e} over {st['units']} "
+                      f"(document, head) rows; {st['near_tie_diffs']} near-tie kept-set differences")
+    tr.write_line(f"worst over all tests: {worst:.2e}")

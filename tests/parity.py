@@ -20,6 +20,18 @@ from oracle import taskpress_oracle as O
 RTOL = 2e-3
 TINY = 2.0 ** -100
 
+#: per-test margins, reported at the end of the run (tests/conftest.py):
+#: test id -> {"max_rel": worst relative score error, "units": checked rows,
+#: "near_tie_diffs": kept-set differences at near-ties of the cut-off}
+STATS: dict = {}
+
+
+def _stat(key: str, value, how=max):
+    import os
+    test = os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0]
+    st = STATS.setdefault(test, {"max_rel": 0.0, "units": 0, "near_tie_diffs": 0})
+    st[key] = how(st[key], value) if key == "max_rel" else st[key] + value
+
 
 def to_device_bf16(bits: np.ndarray):
     import torch
@@ -37,8 +49,10 @@ def assert_scores_close(gpu: np.ndarray, ref: np.ndarray, what: str = "scores"):
     assert gpu.shape == ref.shape, (gpu.shape, ref.shape)
     assert np.all(np.isfinite(gpu)), f"{what}: non-finite GPU values"
     big = ref >= TINY
+    _stat("units", 1)
     if big.any():
         rel = np.abs(gpu[big] - ref[big]) / ref[big]
+        _stat("max_rel", float(rel.max()))
         worst = int(np.argmax(rel))
         assert rel.max() <= RTOL, (f"{what}: rel err {rel.max():.3e} at {np.flatnonzero(big)[worst]} "
                                    f"gpu={gpu[big][worst]!r} ref={ref[big][worst]!r}")
@@ -64,6 +78,7 @@ def assert_kept(gpu_idx: np.ndarray, k: int, ref_scores: np.ndarray, gpu_scores:
         assert np.array_equal(kept, ref)
         return
     diff = np.setxor1d(kept, ref)
+    _stat("near_tie_diffs", int(diff.size))
     if diff.size:
         cut = ref_scores[ref].min()
         gap = np.abs(ref_scores[diff] - cut) / max(cut, TINY)

@@ -382,19 +382,23 @@ def test_repeatable(cuda_lib):
 
 
 # ---------------------------------------------------------------------------
-# Full-size workloads in the benchmark's launch configuration (sampled heads)
+# Full-size workloads in the benchmark's launch configuration: every KV head
+# of every document against the oracle (computed unit by unit in a pool of
+# spawned processes, tests/oracle_pool.py)
 # ---------------------------------------------------------------------------
-@pytest.mark.parametrize("cfg,heads,docs,ratios", [
-    (2, [0, 5], None, None),
-    (3, [3], None, None),
-    (4, [1], None, (0.05, 0.10, 0.25, 0.50)),
-    (5, [2], [0, 5], None),
+@pytest.mark.parametrize("cfg,ratios", [
+    (2, None),
+    (3, None),
+    (4, (0.05, 0.10, 0.25, 0.50)),
+    (5, None),
 ])
-def test_full_size_sampled(cuda_lib, cfg, heads, docs, ratios):
+def test_full_size_all_heads(cuda_lib, cfg, ratios):
     from paper_2608_03276_gb300 import binding
+    from tests import oracle_pool
     w = W[cfg]
     x = synth.make_layer(w)
     for r in (ratios or (w.keep_ratio,)):
         out = _run_compress(binding, w, x, keep_ratio=r)
-        ref = _oracle(w, x, keep_ratio=r, heads=heads, docs=docs)
-        _check_layer(w, x, out, ref, heads=heads, docs=docs)
+        ref = oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv, keep_ratio=r,
+                                         fixed_budget=w.budget)
+        _check_layer(w, x, out, ref)

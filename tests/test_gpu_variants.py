@@ -331,21 +331,25 @@ def test_variants_on_ragged_edges(cuda_lib, variant):
 
 
 def test_full_size_stack(cuda_lib):
-    """Two layers of the 128K Llama-8B-shaped workload through
-    tp_compress_layers, the benchmark's call: layer 0 equals a single-layer call
-    bit for bit, and a sampled head of layer 1 matches the oracle."""
+    """Layers 0, 15 and 31 of the 128K Llama-8B-shaped stack through
+    tp_compress_layers, the benchmark's call: every layer equals a
+    single-layer call bit for bit, and every KV head of every layer matches the
+    oracle."""
     from paper_2608_03276_gb300 import binding
+    from tests import oracle_pool
     w = synth.WORKLOADS[3]
-    xs = _stack(w, 2)
+    xs = [synth.make_layer(w, l) for l in (0, 15, 31)]
     p = _problem(binding, w, xs[0].doc_offsets)
     dev = [tuple(parity.to_device_bf16(t) for t in (y.q, y.k, y.v)) for y in xs]
     outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
     binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, outs[0].ws)
     assert binding.tp_check_status(outs[0].ws) == 0
-    single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
-    binding.compress(p, *dev[1], w.keep_ratio, w.budget, single)
-    _outputs_equal(outs[1], single, "layer 1")
-    _check_layer(w, xs[1], single, _oracle(w, xs[1], heads=[6]), heads=[6])
+    for l, x in enumerate(xs):
+        single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *dev[l], w.keep_ratio, w.budget, single)
+        _outputs_equal(outs[l], single, f"stack layer {l}")
+        _check_layer(w, x, single, oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv,
+                                                               keep_ratio=w.keep_ratio))
 
 
 @pytest.mark.parametrize("bits", [4, 8])
@@ -375,17 +379,19 @@ def test_fully_quantised_cache(cuda_lib, bits):
 @pytest.mark.parametrize("variant", ["caller_lse", "literal", "int4"])
 def test_full_size_variants(cuda_lib, variant):
     """One 128K layer of the Llama-8B-shaped workload (8 KV heads, guide 128 x
-    GQA 4) through each variant path in the benchmark's configuration; one
-    sampled head against the oracle."""
+    GQA 4) through each variant path in the benchmark's configuration; every
+    KV head against the oracle."""
     import torch
     from paper_2608_03276_gb300 import binding
+    from tests import oracle_pool
     w = synth.WORKLOADS[3]
     x = synth.make_layer(w)
-    heads = [5]
     dev = tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v))
     if variant == "int4":
         out = _run_compress(binding, w, x, quant_bits=4)
-        _check_layer(w, x, out, _oracle(w, x, heads=heads, quant_bits=4), heads=heads, bits=4)
+        ref = oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv, keep_ratio=w.keep_ratio,
+                                         quant_bits=4)
+        _check_layer(w, x, out, ref, bits=4)
         return
     p = _problem(binding, w, x.doc_offsets)
     out = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
@@ -394,10 +400,12 @@ def test_full_size_variants(cuda_lib, variant):
         ws = torch.empty(binding.tp_workspace_bytes(p), dtype=torch.uint8, device="cuda")
         binding.tp_guide_lse(p, dev[0], dev[1], lse, ws)
         binding.compress(p, *dev, w.keep_ratio, w.budget, out, lse=lse)
-        ref = _oracle(w, x, heads=heads, lse=lse.cpu().numpy().astype(np.float64))
+        ref = oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv, keep_ratio=w.keep_ratio,
+                                         lse=lse.cpu().numpy().astype(np.float64))
     else:
         kg = synth.make_guide_keys(w)
         binding.compress(p, *dev, w.keep_ratio, w.budget, out, k_guide=parity.to_device_bf16(kg))
-        ref = _oracle(w, x, heads=heads, k_guide_bits=kg)
+        ref = oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv, keep_ratio=w.keep_ratio,
+                                         k_guide_bits=kg)
     assert binding.tp_check_status(out.ws) == 0
-    _check_layer(w, x, out, ref, heads=heads)
+    _check_layer(w, x, out, ref)
