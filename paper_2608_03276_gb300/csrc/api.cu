@@ -35,8 +35,8 @@ struct Plan {
   // resident at once and each CTA's key range fits the tail's shared memory.
   bool tail_ok;
   // workspace offsets
-  size_t ws_status, ws_tsync, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_thist, ws_tcount,
-      ws_total;
+  size_t ws_status, ws_tsync, ws_tflag, ws_thist, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys,
+      ws_tcount, ws_total;
 };
 
 int num_sms() {
@@ -130,9 +130,14 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
     return TP_ERR_UNSUPPORTED_SHAPE;
   P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
   if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
-  P->tail_ok = int64_t(P->grid_x) * P->hkv <= sms && P->tiles_per_cta * 128 <= kTailMaxKeys &&
-               tail_smem_bytes() <= size_t(kMaxSmem);
-  if (P->tail_ok) P->smem2 = std::max(P->smem2, tail_smem_bytes());
+  P->tail_ok = int64_t(P->grid_x) * P->hkv <= sms &&
+               int64_t(P->tiles_per_cta) * 128 + kTailSlack <= kTailMaxKeys &&
+               keyscore_tail_smem_bytes(P->d, P->rows_pad, 1) <= size_t(kMaxSmem);
+  if (P->tail_ok) {  // the tail's layout and histogram fit next to the deepest ring that allows
+    while (P->stages2 > 1 && keyscore_tail_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem)
+      --P->stages2;
+    P->smem2 = keyscore_tail_smem_bytes(P->d, P->rows_pad, P->stages2);
+  }
 
   P->cap = 0;
   if (need_select) {
@@ -146,12 +151,17 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
 
   const size_t units = size_t(P->hkv) * P->batch;
 
-  // [status | counters | tail barrier counters] are zeroed at the start of a call.
+  // [status | counters | tail barrier counters, flags and histograms] are
+  // zeroed at the start of a call.
   size_t o = 0;
   P->ws_status = o;
   o = align_up(o + sizeof(int) * (1 + units));
   P->ws_tsync = o;
   if (P->tail_ok) o = align_up(o + sizeof(int) * 2 * units);
+  P->ws_tflag = o;
+  if (P->tail_ok) o = align_up(o + sizeof(int) * size_t(P->hkv) * P->grid_x);
+  P->ws_thist = o;
+  if (P->tail_ok) o = align_up(o + sizeof(int) * kTailHistInts * units);
   P->ws_partials = o;
   o = align_up(o + sizeof(float2) * size_t(P->hkv) * P->grid_x * P->rows_pad);
   P->ws_lse = o;
@@ -162,8 +172,6 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_keys = o;
   o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
-  P->ws_thist = o;
-  if (P->tail_ok) o = align_up(o + sizeof(int) * kTailHistInts * units);
   P->ws_tcount = o;
   if (P->tail_ok) o = align_up(o + sizeof(int) * 2 * size_t(P->hkv) * P->grid_x);
   P->ws_total = o;
@@ -303,7 +311,7 @@ bool use_tail(const Plan& P, const tp_problem* p) {
 // the gather, for pass 2 of one layer.
 KeyScoreParams tail_params(const Plan& P, const tp_problem* p, char* ws, const void* k,
                            const void* v, const float* gamma, float* scores, int32_t* idx,
-                           void* kc, void* vc, int8_t* vqc, float* gammac) {
+                           void* kc, void* vc, int8_t* vqc, float* gammac, int epoch = 1) {
   KeyScoreParams kp;
   memset(&kp, 0, sizeof(kp));
   kp.tail = 1;
@@ -321,9 +329,12 @@ KeyScoreParams tail_params(const Plan& P, const tp_problem* p, char* ws, const v
   kp.vc = static_cast<uint16_t*>(vc);
   kp.vqc = vqc;
   kp.gammac = gammac;
+  kp.keys = reinterpret_cast<uint32_t*>(ws + P.ws_keys);
   kp.tsync = reinterpret_cast<int*>(ws + P.ws_tsync);
   kp.thist = reinterpret_cast<int*>(ws + P.ws_thist);
   kp.tcount = reinterpret_cast<int*>(ws + P.ws_tcount);
+  kp.tflag = reinterpret_cast<int*>(ws + P.ws_tflag);
+  kp.epoch = epoch;
   return kp;
 }
 
@@ -792,9 +803,11 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
     // with the fused tail, its compaction, or its selection when nothing is
     // kept): its prologue overlaps that kernel's end
     if (tail) {
+      // the CTAs' flags of layer l carry the value l + 1 (zero after the reset)
       const KeyScoreParams extra =
           tail_params(P, p, w, k[l], v[l], g, nullptr, idx ? idx[l] : nullptr, kc ? kc[l] : nullptr,
-                      vc ? vc[l] : nullptr, vqc ? vqc[l] : nullptr, gammac ? gammac[l] : nullptr);
+                      vc ? vc[l] : nullptr, vqc ? vqc[l] : nullptr, gammac ? gammac[l] : nullptr,
+                      l + 1);
       if ((st = run_scoring(P, q[l], k[l], v[l], g, w, s, nullptr, l > 0, extra)) != TP_OK)
         return st;
       continue;

@@ -1,23 +1,27 @@
 // The fused tail of scoring pass 2: a layer's top-budget selection (Sec. 3.4;
 // Sec. 4 "Eviction": a uniform budget per KV head, heads selected
 // independently) and the compaction of the kept rows, run by the same CTAs
-// that scored the keys, right after their scoring loop.
+// that scored the keys.
 //
 // The CTAs of one (document, KV head) unit each own a contiguous key range.
 // The selection is the three-digit radix select of the standalone selection
 // kernel (11, 11 and 10 bits of the fp32 score's bit pattern, lowest token
 // index first among equal scores), with the unit's histograms summed in global
-// memory instead of a cluster's shared memory:
-//   B1  every range's unpooled key scores are in global memory (Eq. 1's
-//       pooling reads up to 16 scores of each neighbouring range);
-//       radix keys of the range (pooled score x gamma, Eq. 3) into shared
-//       memory, digit-1 histogram added into the unit's global histogram
-//   B2  digit 1 (every CTA reads the same histogram and takes the same
-//       decision); digit-2 histogram         B3  digit 2; digit-3 histogram
-//   B4  threshold T: each range's (> T, == T) counts
-//   B5  ordered compaction: a range's kept tokens take consecutive slots after
-//       those of the ranges before it
-//   B6  the unit's kept rows copied into the compressed cache, split evenly
+// memory instead of a cluster's shared memory.
+//
+// During the scoring loop two otherwise idle warps of each CTA turn every
+// scored tile into radix keys (Eq. 1 pooling x gamma, Eq. 3) and count their
+// top digit (tail_keys_in_loop).  A key needs the scores up to K/2 tokens to
+// its right, so the keys of the last K/2 tokens of a range wait for the next
+// CTA's first tile, which that CTA announces with a flag as soon as it is
+// scored.  After the loop (keyscore_tail):
+//   B1  the unit's digit-1 histogram is complete and every key is written;
+//       digit 1 (every CTA reads the same histogram and takes the same
+//       decision); digit-2 histogram       B2  digit 2; digit-3 histogram
+//   B3  threshold T: each range's (> T, == T) counts
+//   B4  ordered compaction: a range's kept tokens take consecutive slots after
+//       those of the ranges before it (warp ballots)
+//   B5  the unit's kept rows copied into the compressed cache, split evenly
 //       over the unit's CTAs
 // A barrier is an arrival counter per unit in the workspace (release add,
 // acquire poll), bounded by the same 2 s limit as every other wait.  The host
@@ -30,27 +34,22 @@
 
 namespace tp {
 
-constexpr int kTailChunk = 4096;   // tokens whose inputs are staged at once
-constexpr int kTailHalfMax = 16;   // largest pooling half-window (pool kernel <= 33)
 constexpr int kTailBins1 = 2048;   // key bits 31..21
 constexpr int kTailBins2 = 2048;   // key bits 20..10
 constexpr int kTailBins3 = 1024;   // key bits 9..0
-constexpr int kTailPer = 16;       // tokens per thread in one compaction round
+constexpr int kKeyWarp0 = 18;      // first of the two key warps of pass 2
+constexpr int kKeyThreads = 64;
 static_assert(kTailBins1 + kTailBins2 + kTailBins3 == kTailHistInts, "histogram layout");
 
 struct TailSmem {
-  uint32_t keys[kTailMaxKeys + kTailMaxKeys / 16];  // one padding word after every 16 keys
-  // unpooled key scores of a chunk with its halo, and its scales: element g of
-  // the global array sits at [g - g_ref], g_ref a multiple of 4
-  float strip[kTailChunk + 2 * kTailHalfMax + 4];
-  float vals[kTailChunk + 4];
-  int hist[kTailBins1];  // this range's histogram of the current digit
+  // the range's keys: token i at keys[g0 + i - kref], kref = (g0 + first) & ~3
+  uint32_t keys[kTailMaxKeys + 4];
+  int hist[kTailBins2];   // this range's histogram of digit 2 or 3
   int scratch[33];
   int result[2];
+  int wsum[2][32];        // per-warp (> T, == T) counts, then their exclusive prefix
 };
-static_assert(sizeof(uint32_t) * (kTailMaxKeys + kTailMaxKeys / 16) % 16 == 0 &&
-                  sizeof(float) * (kTailChunk + 2 * kTailHalfMax + 4) % 16 == 0,
-              "16-byte cp.async destinations must be 16-byte aligned");
+static_assert(sizeof(uint32_t) * (kTailMaxKeys + 4) % 16 == 0, "16-byte cp.async destinations");
 
 __device__ __forceinline__ void red_release_add(int* p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
@@ -62,16 +61,19 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
   return v;
 }
 
-// Stages global floats src[ga, gb) into dst[g - g_ref] (g_ref a multiple of 4,
-// dst 16-byte aligned), reading through L2 only: the values were written by
-// other CTAs of this grid.  16-byte cp.async.cg over the aligned middle, plain
-// L2 loads at the two ragged ends.  Called by every thread of the block;
-// complete after cp_async_wait_all() and a barrier.
-__device__ __forceinline__ void stage_floats_l2(float* dst, const float* src, int64_t ga,
-                                                int64_t gb, int64_t g_ref) {
+__device__ __forceinline__ void st_release(int* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Stages 32-bit words src[ga, gb) into dst[g - g_ref] (g_ref a multiple of 4,
+// dst 16-byte aligned), reading through L2 only: 16-byte cp.async.cg over the
+// aligned middle, plain L2 loads at the two ragged ends (or everywhere when
+// src is not 16-byte aligned).  Called by every thread of the block; complete
+// after cp_async_wait_all() and a barrier.
+__device__ __forceinline__ void stage_words_l2(uint32_t* dst, const uint32_t* src, int64_t ga,
+                                               int64_t gb, int64_t g_ref) {
   if (gb <= ga) return;
   const int64_t a4 = (ga + 3) & ~int64_t(3), b4 = gb & ~int64_t(3);
-  // a caller's array need only be 4-byte aligned: then every load is 4 bytes
   if (a4 >= b4 || (reinterpret_cast<uintptr_t>(src) & 15) != 0) {
     for (int64_t g = ga + threadIdx.x; g < gb; g += blockDim.x) dst[g - g_ref] = __ldcg(src + g);
     return;
@@ -88,6 +90,94 @@ __device__ __forceinline__ void stage_floats_l2(float* dst, const float* src, in
   } else if (static_cast<int>(threadIdx.x) >= 32 && static_cast<int>(threadIdx.x) < 32 + tail) {
     const int64_t g = b4 + (threadIdx.x - 32);
     dst[g - g_ref] = __ldcg(src + g);
+  }
+}
+
+// Radix key of token i of the document whose token 0 is global index g0
+// (Eq. 1 pooling of the unpooled key scores, zero outside [0, n), divisor K;
+// then Eq. 3's product with gamma, or the harmonic blend, or the key score
+// alone); the combined score goes to scores_out when asked.  Reads through L2.
+__device__ __forceinline__ uint32_t tail_key(const KeyScoreParams& p, int64_t g0, int i, int n,
+                                             int half, float inv_k) {
+  const float* w = p.skey + g0 + i - half;
+  float acc;
+  if (half == 2 && i >= 2 && i + 2 < n) {  // the default window of five, summed in the same order
+    acc = (((__ldcg(w) + __ldcg(w + 1)) + __ldcg(w + 2)) + __ldcg(w + 3)) + __ldcg(w + 4);
+  } else {
+    acc = 0.f;
+    for (int o = 0; o <= 2 * half; ++o) {
+      const int t = i - half + o;
+      acc += (t >= 0 && t < n) ? __ldcg(w + o) : 0.f;
+    }
+  }
+  const float a = acc * inv_k;
+  float sc;
+  if (p.key_only) {
+    sc = a;
+  } else if (p.blend == kBlendHarmonic) {
+    const float g = __ldcg(p.gamma + g0 + i);
+    const float den = a + g;
+    sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
+  } else {
+    sc = a * __ldcg(p.gamma + g0 + i);
+  }
+  if (p.scores_out) p.scores_out[g0 + i] = sc;
+  return score_key(sc);
+}
+
+// Digit-1 count of a key in the packed 16-bit histogram (bins 2w and 2w + 1
+// share word w; a range holds at most kTailMaxKeys keys, so no count overflows).
+__device__ __forceinline__ void hist16_add(uint32_t* hist16, uint32_t key) {
+  const uint32_t bin = key >> 21;
+  atomicAdd(hist16 + (bin >> 1), 1u << ((bin & 1u) << 4));
+}
+
+// Waits until *count reaches `target` (bounded like every wait).
+__device__ __forceinline__ bool wait_count(volatile int* count, int target, volatile int* abort_flag) {
+  if (*count >= target) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (*count < target) {
+    if (*abort_flag) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      return false;
+    }
+    __nanosleep(64);
+  }
+  return true;
+}
+
+// The two key warps during the scoring loop: keys of tokens [o0, ilim) of the
+// CTA's range, tile by tile, as the epilogue announces scored tiles on
+// `tiles_done` (four arrivals per tile).  ilim stops K/2 tokens short of the
+// range's end unless the range ends the document.  After tile 0 is scored its
+// keys... and the CTA's flag tells the previous CTA of the unit that the
+// scores it needs for its last K/2 keys are in memory.
+__device__ void tail_keys_in_loop(const KeyScoreParams& p, uint32_t* hist16, volatile int* tiles_done,
+                                  int c, int t0, int nt, int n, int64_t doc_lo, int h,
+                                  volatile int* abort_flag) {
+  const int tid = static_cast<int>(threadIdx.x) - kKeyWarp0 * 32;
+  for (int i = tid; i < kTailBins1 / 2; i += kKeyThreads) hist16[i] = 0;
+  asm volatile("bar.sync 1, %0;" ::"n"(kKeyThreads) : "memory");  // the two key warps only
+  const int half = p.pool_kernel / 2;
+  const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
+  const int s0 = t0 * kKeyTile, s1 = min((t0 + nt) * kKeyTile, n);
+  const int o0 = c == 0 ? 0 : min(s0 + half, n);
+  const int ilim = s1 >= n ? n : s1 - half;
+  const int64_t g0 = static_cast<int64_t>(h) * p.n_total + doc_lo;
+  const int cta_lin = blockIdx.y * gridDim.x + blockIdx.x;
+  for (int lt = 0; lt < nt; ++lt) {
+    if (!wait_count(tiles_done, 4 * min(lt + 2, nt), abort_flag)) return;
+    if (lt == 0 && tid == 0) {
+      __threadfence();
+      st_release(p.tflag + cta_lin, p.epoch);
+    }
+    const int a = max(o0, s0 + lt * kKeyTile), e = min(s0 + (lt + 1) * kKeyTile, ilim);
+    for (int i = a + tid; i < e; i += kKeyThreads) {
+      const uint32_t key = tail_key(p, g0, i, n, half, inv_k);
+      p.keys[g0 + i] = key;
+      hist16_add(hist16, key);
+    }
   }
 }
 
@@ -217,12 +307,14 @@ __device__ __forceinline__ void tail_clear(const KeyScoreParams& p, int64_t slot
 }
 
 // The tail of one CTA: document b, head h, this CTA the c-th of the ncta CTAs
-// of the unit, owning key tiles t0 .. t0+nt-1 of the n-token document.  Every
+// of the unit, owning key tiles t0 .. t0+nt-1 of the n-token document; its
+// key range is [o0, o1) (the tiles' tokens shifted right by K/2, see above).
+// `hist16` holds the digit-1 counts of the keys the key warps formed.  Every
 // thread of the block calls it after the scoring loop (the shared memory of
 // the scoring pipeline is free again).
 template <int D>
-__device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int h, int c,
-                              int ncta, int t0, int nt, int n, int64_t doc_lo,
+__device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, uint32_t* hist16, int b,
+                              int h, int c, int ncta, int t0, int nt, int n, int64_t doc_lo,
                               volatile int* abort_flag) {
   TailSmem& sm = *reinterpret_cast<TailSmem*>(smem);
   const int unit = b * p.n_heads_kv + h;
@@ -232,13 +324,19 @@ __device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int
   int* const gh3 = gh2 + kTailBins2;
   const int kk = max(0, min(p.kept[b], n));
   const bool radix = kk > 0 && kk < n;
-  const int phases = 1 + (radix ? 3 : 0) + (kk > 0 ? 2 : 0);
-  const int s0 = t0 * kKeyTile, s1 = min((t0 + nt) * kKeyTile, n);
+  const int phases = 1 + (radix ? 2 : 0) + (kk > 0 ? 2 : 0);
+  const int half = p.pool_kernel / 2;
+  const int s1 = min((t0 + nt) * kKeyTile, n);
+  const int o0 = c == 0 ? 0 : min(t0 * kKeyTile + half, n);
+  const int o1 = c == ncta - 1 ? n : min(s1 + half, n);
   const int64_t g0 = static_cast<int64_t>(h) * p.n_total + doc_lo;  // token 0 of the document
+  const int64_t kref = (g0 + o0) & ~int64_t(3);
   const int64_t slot0 = static_cast<int64_t>(unit) * p.cap;
   const int cta_lin = blockIdx.y * gridDim.x + blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
   int arrived = 0;  // thread 0's arrivals on ctr
   int phase = 0;
+  auto key_at = [&](int i) { return sm.keys[g0 + i - kref]; };
 
   // barrier over the unit's CTAs: every CTA's global writes before it are
   // visible to every CTA after it
@@ -257,10 +355,9 @@ __device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int
             *abort_flag = 1;
             break;
           }
-          __nanosleep(64);
+          __nanosleep(32);
         }
       }
-      __threadfence();
     }
     __syncthreads();
     return *abort_flag == 0;
@@ -286,86 +383,63 @@ __device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int
     bail();
     return;
   }
-  // this CTA's share of the unit's histograms starts at zero (before B1, so
-  // every CTA adds into zeroed bins after it)
-  if (radix) {
-    const int za = kTailHistInts * c / ncta, zb = kTailHistInts * (c + 1) / ncta;
-    for (int i = za + threadIdx.x; i < zb; i += blockDim.x) gh1[i] = 0;
-  }
-  for (int i = threadIdx.x; i < kTailBins1; i += blockDim.x) sm.hist[i] = 0;
-  if (!unit_sync()) {  // B1
-    bail();
-    return;
-  }
-
-  // radix keys of the range: Eq. 1 pooling of the key scores (zero outside the
-  // document, divisor K), times gamma (Eq. 3) or a blend
-  const int half = p.pool_kernel / 2;
-  const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
-  auto kpos = [&](int i) {
-    const int r = i - s0;
-    return r + (r >> 4);
-  };
-  for (int c0 = s0; c0 < s1; c0 += kTailChunk) {
-    const int c1 = min(c0 + kTailChunk, s1);
-    const int64_t sref = (g0 + c0 - half) & ~int64_t(3), vref = (g0 + c0) & ~int64_t(3);
-    const int ia = max(c0 - half, 0), ib = min(c1 + half, n);  // halo inside the document
-    stage_floats_l2(sm.strip, p.skey, g0 + ia, g0 + ib, sref);
-    for (int i = c0 - half + static_cast<int>(threadIdx.x); i < c1 + half; i += blockDim.x)
-      if (i < ia || i >= ib) sm.strip[g0 + i - sref] = 0.f;
-    if (!p.key_only) stage_floats_l2(sm.vals, p.gamma, g0 + c0, g0 + c1, vref);
-    cp_async_wait_all();
-    __syncthreads();
-    const float* vrow = sm.vals + (g0 + c0 - vref);         // token c0 at vrow[0]
-    const float* srow = sm.strip + (g0 + c0 - half - sref);  // token c0's window at srow[0]
-#pragma unroll 4
-    for (int i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-      const int r = i - c0;
-      const float* w = srow + r;
-      float acc;
-      if (half == 2) {  // the default window of five, summed in the same order
-        acc = (((w[0] + w[1]) + w[2]) + w[3]) + w[4];
-      } else {
-        acc = 0.f;
-        for (int o = 0; o <= 2 * half; ++o) acc += w[o];
+  // keys of the last K/2 tokens of the range: their windows reach into the
+  // next CTA's first tile, announced by that CTA's flag
+  if (c < ncta - 1) {
+    if (threadIdx.x == 0) {
+      const int* flag = p.tflag + cta_lin + 1;
+      const uint64_t tw = global_timer_ns();
+      while (ld_acquire(flag) < p.epoch) {
+        if (global_timer_ns() - tw > kWaitLimitNs) {
+          *abort_flag = 1;
+          break;
+        }
+        __nanosleep(32);
       }
-      const float a = acc * inv_k;
-      float sc;
-      if (p.key_only) {
-        sc = a;
-      } else if (p.blend == kBlendHarmonic) {
-        const float g = vrow[r];
-        const float den = a + g;
-        sc = den > 0.f ? __fdiv_rn(2.f * a * g, den) : 0.f;
-      } else {
-        sc = a * vrow[r];
-      }
-      if (p.scores_out) p.scores_out[g0 + i] = sc;
-      const uint32_t key = score_key(sc);
-      sm.keys[kpos(i)] = key;
-      if (radix) atomicAdd(&sm.hist[key >> 21], 1);
     }
     __syncthreads();
+    if (*abort_flag) {
+      bail();
+      return;
+    }
+    const float inv_k = 1.0f / static_cast<float>(p.pool_kernel);
+    for (int i = max(o0, s1 - half) + static_cast<int>(threadIdx.x); i < o1; i += blockDim.x) {
+      const uint32_t key = tail_key(p, g0, i, n, half, inv_k);
+      p.keys[g0 + i] = key;
+      hist16_add(hist16, key);
+    }
+  }
+  __syncthreads();
+  // the range's digit-1 counts into the unit's histogram, and its keys into
+  // shared memory (in flight across the barrier)
+  if (radix) {
+    for (int w = threadIdx.x; w < kTailBins1 / 2; w += blockDim.x) {
+      const uint32_t v = hist16[w];
+      if (v & 0xFFFFu) atomicAdd(gh1 + 2 * w, static_cast<int>(v & 0xFFFFu));
+      if (v >> 16) atomicAdd(gh1 + 2 * w + 1, static_cast<int>(v >> 16));
+    }
+  }
+  if (kk > 0) stage_words_l2(sm.keys, p.keys, g0 + o0, g0 + o1, kref);
+  for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) sm.hist[i] = 0;
+  cp_async_wait_all();
+  if (!unit_sync()) {  // B1: digit-1 histogram complete, every key written
+    bail();
+    return;
   }
 
   uint32_t thr = 0;
   int need_eq = -1;  // -1: every token of the document is kept
   if (radix) {
-    tail_flush_hist(gh1, sm.hist, kTailBins1);
-    if (!unit_sync()) {  // B2
-      bail();
-      return;
-    }
     int above;
     const int d1 = tail_digit(gh1, kTailBins1, kk, &above, sm);
     int need = kk - above;
 #pragma unroll 4
-    for (int i = s0 + threadIdx.x; i < s1; i += blockDim.x) {
-      const uint32_t key = sm.keys[kpos(i)];
+    for (int i = o0 + threadIdx.x; i < o1; i += blockDim.x) {
+      const uint32_t key = key_at(i);
       if ((key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist[(key >> 10) & 0x7FF], 1);
     }
     tail_flush_hist(gh2, sm.hist, kTailBins2);
-    if (!unit_sync()) {  // B3
+    if (!unit_sync()) {  // B2
       bail();
       return;
     }
@@ -373,12 +447,12 @@ __device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int
     need -= above;
     const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
 #pragma unroll 4
-    for (int i = s0 + threadIdx.x; i < s1; i += blockDim.x) {
-      const uint32_t key = sm.keys[kpos(i)];
+    for (int i = o0 + threadIdx.x; i < o1; i += blockDim.x) {
+      const uint32_t key = key_at(i);
       if ((key >> 10) == pre) atomicAdd(&sm.hist[key & 0x3FF], 1);
     }
     tail_flush_hist(gh3, sm.hist, kTailBins3);
-    if (!unit_sync()) {  // B4
+    if (!unit_sync()) {  // B3
       bail();
       return;
     }
@@ -388,83 +462,80 @@ __device__ void keyscore_tail(const KeyScoreParams& p, uint8_t* smem, int b, int
   }
 
   if (kk > 0) {
-    // (> T, == T) counts of this range
+    // warp w owns the chunk [w0, w1) of the range, a multiple of 32 tokens long
+    const int m = o1 - o0;
+    const int chunk = ((m + nwarps - 1) / nwarps + 31) & ~31;
+    const int w0 = min(o0 + warp * chunk, o1), w1 = min(w0 + chunk, o1);
     int gt = 0, eq = 0;
-#pragma unroll 4
-    for (int i = s0 + threadIdx.x; i < s1; i += blockDim.x) {
-      const uint32_t key = sm.keys[kpos(i)];
+    for (int j = w0 + lane; j < w1; j += 32) {
+      const uint32_t key = key_at(j);
       if (need_eq < 0 || key > thr) ++gt;
       else if (key == thr) ++eq;
     }
-    gt = block_sum(gt, sm.scratch);
-    eq = block_sum(eq, sm.scratch);
-    if (threadIdx.x == 0) {
-      p.tcount[2 * cta_lin] = gt;
-      p.tcount[2 * cta_lin + 1] = eq;
+    gt = __reduce_add_sync(0xffffffffu, gt);
+    eq = __reduce_add_sync(0xffffffffu, eq);
+    if (lane == 0) {
+      sm.wsum[0][warp] = gt;
+      sm.wsum[1][warp] = eq;
     }
-    if (!unit_sync()) {  // B5
+    __syncthreads();
+    if (threadIdx.x == 0) {  // the range's counts, and each warp's prefix within it
+      int a = 0, e = 0;
+      for (int w = 0; w < nwarps; ++w) {
+        const int tg = sm.wsum[0][w], te = sm.wsum[1][w];
+        sm.wsum[0][w] = a;
+        sm.wsum[1][w] = e;
+        a += tg;
+        e += te;
+      }
+      p.tcount[2 * cta_lin] = a;
+      p.tcount[2 * cta_lin + 1] = e;
+    }
+    if (!unit_sync()) {  // B3 / B4: every range's counts are in memory
       bail();
       return;
     }
+    // zero this CTA's share of the unit's histograms for the next layer:
+    // every CTA read them before arriving here
+    if (radix) {
+      const int za = kTailHistInts * c / ncta, zb = kTailHistInts * (c + 1) / ncta;
+      for (int i = za + threadIdx.x; i < zb; i += blockDim.x) gh1[i] = 0;
+    }
     // counts of the unit's ranges before this one (CTAs c' < c of this head row)
-    if (threadIdx.x < 32) {
+    if (warp == 0) {
       int a = 0, e = 0;
       const int lin0 = cta_lin - c;
-      for (int j = threadIdx.x; j < c; j += 32) {
+      for (int j = lane; j < c; j += 32) {
         a += __ldcg(p.tcount + 2 * (lin0 + j));
         e += __ldcg(p.tcount + 2 * (lin0 + j) + 1);
       }
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) {
-        a += __shfl_xor_sync(0xffffffffu, a, o);
-        e += __shfl_xor_sync(0xffffffffu, e, o);
-      }
-      if (threadIdx.x == 0) {
+      a = __reduce_add_sync(0xffffffffu, a);
+      e = __reduce_add_sync(0xffffffffu, e);
+      if (lane == 0) {
         sm.result[0] = a;
         sm.result[1] = e;
       }
     }
     __syncthreads();
-    int gt_before = sm.result[0], eq_before = sm.result[1];
-    __syncthreads();
-    // ordered compaction: a kept token's slot is (tokens > T before it) +
-    // min(tokens == T before it, need_eq)
-    const int round = static_cast<int>(blockDim.x) * kTailPer;
-    for (int base = s0; base < s1; base += round) {
-      const int j0 = base + static_cast<int>(threadIdx.x) * kTailPer;
-      int ngt = 0, neq = 0;
-      uint32_t kv[kTailPer];
-#pragma unroll
-      for (int e = 0; e < kTailPer; ++e) {
-        const int j = j0 + e;
-        kv[e] = j < s1 ? sm.keys[kpos(j)] : 0u;
-        if (j < s1) {
-          if (need_eq < 0 || kv[e] > thr) ++ngt;
-          else if (kv[e] == thr) ++neq;
-        }
+    // ordered compaction by warp ballots: a kept token's slot is (tokens > T
+    // before it) + min(tokens == T before it, need_eq)
+    int gbase = sm.result[0] + sm.wsum[0][warp], ebase = sm.result[1] + sm.wsum[1][warp];
+    const uint32_t below = (1u << lane) - 1u;
+    for (int j0 = w0; j0 < w1; j0 += 32) {
+      const int j = j0 + lane;
+      const uint32_t key = j < w1 ? key_at(j) : 0u;
+      const bool is_gt = j < w1 && (need_eq < 0 || key > thr);
+      const bool is_eq = j < w1 && !is_gt && key == thr;
+      const uint32_t mg = __ballot_sync(0xffffffffu, is_gt), me = __ballot_sync(0xffffffffu, is_eq);
+      const int gr = gbase + __popc(mg & below), er = ebase + __popc(me & below);
+      if (is_gt || (is_eq && er < need_eq)) {
+        const int slot = gr + (need_eq < 0 ? 0 : min(er, need_eq));
+        if (slot < kk) p.idx[slot0 + slot] = j;  // always true when the counts agree
       }
-      // one scan of packed counts: (> T) in the high 16 bits, (== T) in the low
-      int tot;
-      const int pre = block_excl_scan((ngt << 16) | neq, sm.scratch, &tot);
-      int gt_rank = gt_before + (pre >> 16);
-      int eq_rank = eq_before + (pre & 0xFFFF);
-#pragma unroll
-      for (int e = 0; e < kTailPer; ++e) {
-        const int j = j0 + e;
-        if (j >= s1) break;
-        const bool is_gt = need_eq < 0 || kv[e] > thr;
-        const bool is_eq = !is_gt && kv[e] == thr;
-        if (is_gt || (is_eq && eq_rank < need_eq)) {
-          const int slot = gt_rank + (need_eq < 0 ? 0 : min(eq_rank, need_eq));
-          if (slot < kk) p.idx[slot0 + slot] = j;  // always true when the counts agree
-        }
-        gt_rank += is_gt;
-        eq_rank += is_eq;
-      }
-      gt_before += tot >> 16;
-      eq_before += tot & 0xFFFF;
+      gbase += __popc(mg);
+      ebase += __popc(me);
     }
-    if (!unit_sync()) {  // B6: every kept index of the unit is written
+    if (!unit_sync()) {  // B4 / B5: every kept index of the unit is written
       bail();
       return;
     }
