@@ -242,11 +242,9 @@ int tp_compact(const tp_problem* p, const void* k, const void* v, const float* g
  * top-budget selection and compaction, all on `stream` with no host
  * synchronisation.  Outputs as in tp_select and tp_compact; `scores` and
  * `gamma` ([H_kv, N] fp32) are optional outputs (NULL to skip).
- * Kernels: the normalising pass (which also forms the Eq. 2 scales), then the
- * key-score pass, which for most problems goes on to select and compact the
- * kept rows itself; otherwise (a CTA's key range beyond 16384 keys, more
- * scoring CTAs than SMs, or TP_SCORE_NORM_ADD) a selection kernel and a
- * compaction kernel follow.  Results are the same either way.
+ * Kernels: the normalising pass (which also forms the Eq. 2 scales), the
+ * key-score pass, the selection and the compaction (none when nothing is
+ * kept), each a programmatic dependent of the one before;
  * tp_compress_kernel_count says how many kernels a call launches.
  */
 int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const void* v,

@@ -31,12 +31,8 @@ struct Plan {
   float qmax;   // 2^(bits-1) - 1
   int32_t kept[kMaxBatch];
   int64_t cap;
-  // Pass 2 can also select and compact (tail.cuh): every CTA of its grid is
-  // resident at once and each CTA's key range fits the tail's shared memory.
-  bool tail_ok;
   // workspace offsets
-  size_t ws_status, ws_tsync, ws_tflag, ws_thist, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys,
-      ws_tcount, ws_total;
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
 };
 
 int num_sms() {
@@ -130,14 +126,6 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
     return TP_ERR_UNSUPPORTED_SHAPE;
   P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
   if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
-  P->tail_ok = int64_t(P->grid_x) * P->hkv <= sms &&
-               int64_t(P->tiles_per_cta) * 128 + kTailSlack <= kTailMaxKeys &&
-               keyscore_tail_smem_bytes(P->d, P->rows_pad, 1) <= size_t(kMaxSmem);
-  if (P->tail_ok) {  // the tail's layout and histogram fit next to the deepest ring that allows
-    while (P->stages2 > 1 && keyscore_tail_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem)
-      --P->stages2;
-    P->smem2 = keyscore_tail_smem_bytes(P->d, P->rows_pad, P->stages2);
-  }
 
   P->cap = 0;
   if (need_select) {
@@ -151,17 +139,10 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
 
   const size_t units = size_t(P->hkv) * P->batch;
 
-  // [status | counters | tail barrier counters, flags and histograms] are
-  // zeroed at the start of a call.
+  // [status | counters] are zeroed at the start of a call.
   size_t o = 0;
   P->ws_status = o;
   o = align_up(o + sizeof(int) * (1 + units));
-  P->ws_tsync = o;
-  if (P->tail_ok) o = align_up(o + sizeof(int) * 2 * units);
-  P->ws_tflag = o;
-  if (P->tail_ok) o = align_up(o + sizeof(int) * size_t(P->hkv) * P->grid_x);
-  P->ws_thist = o;
-  if (P->tail_ok) o = align_up(o + sizeof(int) * kTailHistInts * units);
   P->ws_partials = o;
   o = align_up(o + sizeof(float2) * size_t(P->hkv) * P->grid_x * P->rows_pad);
   P->ws_lse = o;
@@ -172,8 +153,6 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_keys = o;
   o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
-  P->ws_tcount = o;
-  if (P->tail_ok) o = align_up(o + sizeof(int) * 2 * size_t(P->hkv) * P->grid_x);
   P->ws_total = o;
   return TP_OK;
 }
@@ -268,18 +247,11 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
       launch_lse(tmk, tmv, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, dependent, s));
 }
 
-int blend_of(uint32_t flags) {
-  if (flags & TP_SCORE_NORM_ADD) return kBlendNormAdd;
-  if (flags & TP_SCORE_HARMONIC) return kBlendHarmonic;
-  return kBlendProduct;
-}
-
-// Pass 2: unpooled key scores [H_kv, N] from the row normalisers.  `kp`
-// carries what the pass does besides (zero: nothing): the layer's selection
-// and compaction (tail).
+// Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
 int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const float* lse,
-                 float* skey, int* status, bool dependent, cudaStream_t s,
-                 KeyScoreParams kp = KeyScoreParams{}) {
+                 float* skey, int* status, bool dependent, cudaStream_t s) {
+  KeyScoreParams kp;
+  memset(&kp, 0, sizeof(kp));
   kp.docs = doc_table(P);
   kp.n_heads_kv = P.hkv;
   kp.rows = P.rows;
@@ -293,49 +265,8 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
   kp.lse = lse;
   kp.skey = skey;
   kp.status = status;
-  kp.qmax = P.qmax;
-  kp.bits = P.bits;
   return cuda_status(
       launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
-}
-
-// Whether a fused call selects and compacts in pass 2's tail (tail.cuh)
-// rather than in the selection and gather kernels: the plan allows it, some
-// document has tokens (pass 2 runs), and the blend needs no norms over the
-// whole (document, head).
-bool use_tail(const Plan& P, const tp_problem* p) {
-  return P.tail_ok && P.grid_x > 0 && P.n_total > 0 && blend_of(p->flags) != kBlendNormAdd;
-}
-
-// The tail's arguments: the selection of fill_select and the compaction of
-// the gather, for pass 2 of one layer.
-KeyScoreParams tail_params(const Plan& P, const tp_problem* p, char* ws, const void* k,
-                           const void* v, const float* gamma, float* scores, int32_t* idx,
-                           void* kc, void* vc, int8_t* vqc, float* gammac, int epoch = 1) {
-  KeyScoreParams kp;
-  memset(&kp, 0, sizeof(kp));
-  kp.tail = 1;
-  kp.pool_kernel = p->pool_kernel;
-  kp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
-  kp.blend = blend_of(p->flags);
-  kp.cap = P.cap;
-  for (int b = 0; b < P.batch; ++b) kp.kept[b] = P.kept[b];
-  kp.gamma = gamma;
-  kp.scores_out = scores;
-  kp.idx = idx;
-  kp.k = static_cast<const uint16_t*>(k);
-  kp.v = static_cast<const uint16_t*>(v);
-  kp.kc = static_cast<uint16_t*>(kc);
-  kp.vc = static_cast<uint16_t*>(vc);
-  kp.vqc = vqc;
-  kp.gammac = gammac;
-  kp.keys = reinterpret_cast<uint32_t*>(ws + P.ws_keys);
-  kp.tsync = reinterpret_cast<int*>(ws + P.ws_tsync);
-  kp.thist = reinterpret_cast<int*>(ws + P.ws_thist);
-  kp.tcount = reinterpret_cast<int*>(ws + P.ws_tcount);
-  kp.tflag = reinterpret_cast<int*>(ws + P.ws_tflag);
-  kp.epoch = epoch;
-  return kp;
 }
 
 // The guide-prefix fold of the literal normaliser (`lse` in place).
@@ -360,8 +291,7 @@ int run_prefix(const Plan& P, const void* q, const void* k_guide, float* lse, bo
 // is given, and the guide prefix folded into the normalisers between them when
 // k_guide is given); leaves the unpooled key scores in the workspace.
 int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
-                cudaStream_t s, const void* k_guide = nullptr, bool dependent = false,
-                const KeyScoreParams& extra = KeyScoreParams{}) {
+                cudaStream_t s, const void* k_guide = nullptr, bool dependent = false) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
@@ -370,7 +300,13 @@ int run_scoring(const Plan& P, const void* q, const void* k, const void* v, floa
   if (st != TP_OK) return st;
   if (k_guide && (st = run_prefix(P, q, k_guide, lse, true, s)) != TP_OK) return st;
   return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
-                      reinterpret_cast<int*>(ws + P.ws_status), true, s, extra);
+                      reinterpret_cast<int*>(ws + P.ws_status), true, s);
+}
+
+int blend_of(uint32_t flags) {
+  if (flags & TP_SCORE_NORM_ADD) return kBlendNormAdd;
+  if (flags & TP_SCORE_HARMONIC) return kBlendHarmonic;
+  return kBlendProduct;
 }
 
 void fill_select(const Plan& P, char* ws, SelectParams* sp) {
@@ -426,24 +362,18 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   char* w = static_cast<char*>(ws);
   float* g = gamma ? gamma : reinterpret_cast<float*>(w + P.ws_gamma);
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  const bool tail = use_tail(P, p);
-  KeyScoreParams extra;
-  memset(&extra, 0, sizeof(extra));
-  if (tail) extra = tail_params(P, p, w, k, v, g, scores, idx, kc, vc, vqc, gammac);
   if (!lse_in) {
-    if ((st = run_scoring(P, q, k, v, g, w, s, k_guide, false, extra)) != TP_OK) return st;
+    if ((st = run_scoring(P, q, k, v, g, w, s, k_guide)) != TP_OK) return st;
   } else if (P.n_total > 0 && P.grid_x > 0) {
-    // one scoring pass over K; the Eq. 2 scales from a pass over V
     if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
                       P.qmax, P.bits, num_sms(), s) != cudaSuccess)
       return TP_ERR_CUDA;
     CUtensorMap tmk, tmq;
     if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
     if ((st = run_keyscore(P, tmk, tmq, lse_in, reinterpret_cast<float*>(w + P.ws_skey),
-                           reinterpret_cast<int*>(w + P.ws_status), false, s, extra)) != TP_OK)
+                           reinterpret_cast<int*>(w + P.ws_status), false, s)) != TP_OK)
       return st;
   }
-  if (tail) return TP_OK;
   SelectParams sp;
   fill_select(P, w, &sp);
   sp.pool_kernel = p->pool_kernel;
@@ -794,24 +724,11 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
   float* g = reinterpret_cast<float*>(w + P.ws_gamma);
-  // one reset for the whole stack: pass 1 leaves its counters zero again, and
-  // so does pass 2's tail with its barrier counters
+  // one reset for the whole stack: pass 1 leaves its counters zero again
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  const bool tail = use_tail(P, p);
   for (int l = 0; l < n_layers; ++l) {
-    // layer l's pass 1 is a dependent of layer l - 1's last kernel (its pass 2
-    // with the fused tail, its compaction, or its selection when nothing is
-    // kept): its prologue overlaps that kernel's end
-    if (tail) {
-      // the CTAs' flags of layer l carry the value l + 1 (zero after the reset)
-      const KeyScoreParams extra =
-          tail_params(P, p, w, k[l], v[l], g, nullptr, idx ? idx[l] : nullptr, kc ? kc[l] : nullptr,
-                      vc ? vc[l] : nullptr, vqc ? vqc[l] : nullptr, gammac ? gammac[l] : nullptr,
-                      l + 1);
-      if ((st = run_scoring(P, q[l], k[l], v[l], g, w, s, nullptr, l > 0, extra)) != TP_OK)
-        return st;
-      continue;
-    }
+    // layer l's pass 1 is a dependent of layer l - 1's compaction (or of its
+    // selection when nothing is kept): its prologue overlaps that kernel's tail
     if ((st = run_scoring(P, q[l], k[l], v[l], g, w, s, nullptr, l > 0)) != TP_OK) return st;
     SelectParams sp;
     fill_select(P, w, &sp);
@@ -850,10 +767,9 @@ int tp_guide_prefix_lse(const tp_problem* p, const void* q, const void* k_guide,
 int tp_compress_kernel_count(const tp_problem* p, double keep_ratio, int64_t budget, int mode) {
   Plan P;
   if (mode < 0 || mode > 2 || make_plan(p, keep_ratio, budget, true, &P) != TP_OK) return -1;
-  const bool scored = P.n_total > 0 && P.grid_x > 0;
-  int kernels = 0;
-  if (scored) kernels += mode == 2 ? 3 : 2;  // pass 1 or the V scales, [prefix fold,] pass 2
-  if (!use_tail(P, p)) kernels += P.cap > 0 ? 2 : 1;              // selection [+ compaction]
+  int kernels = P.cap > 0 ? 2 : 1;  // selection [+ compaction]
+  if (P.n_total > 0 && P.grid_x > 0)
+    kernels += mode == 2 ? 3 : 2;  // pass 1 (or the V scales for mode 1), [prefix fold,] pass 2
   return kernels;
 }
 

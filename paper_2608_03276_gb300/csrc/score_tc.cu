@@ -15,25 +15,19 @@
 //
 // Both passes stream 128-key tiles of K with TMA (128-byte swizzle) through a
 // ring of shared-memory stages; one thread issues the MMAs; four epilogue
-// warpgroups drain TMEM.  Warp roles per CTA (20 warps):
+// warpgroups drain TMEM.  Warp roles per CTA (18 warps):
 //   warp 0  TMEM owner + TMA producer      warp 1  MMA issuer
 //   warps 2-17  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
-//   warps 18-19 pass 1: Eq. 2 scales of the CTA's V rows from a TMA ring;
-//               pass 2: radix keys of the scored tiles (with the fused tail)
-// Pass 2 may go on to select and compact the layer's kept rows (tail.cuh).
 #include <math.h>
 
-#include <algorithm>
-
-#include "tail.cuh"
 #include "tp_device.cuh"
 
 namespace tp {
 
 namespace {
 
-constexpr int kThreads = 640;      // pass 2: TMA, MMA, 16 epilogue warps, 2 key warps
-constexpr int kLseThreads = 640;   // pass 1: the same, the last 2 warps for the V scales
+constexpr int kThreads = 576;      // pass 2: TMA, MMA, 16 epilogue warps
+constexpr int kLseThreads = 640;   // pass 1: the same plus 2 V-scale warps
 constexpr int kVWarp0 = 18;        // first V-scale warp of pass 1
 constexpr int kVStages = 3;        // V-tile ring depth of pass 1
 constexpr int kEpiWarp0 = 2;  // first epilogue warp
@@ -543,11 +537,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* pdone = drain + 1;    // [4] partial slots complete, one arrival per warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
-  int* tiles_done = reinterpret_cast<int*>(smem + L.misc + 8);  // scored tiles x 4 (fused tail)
-  // digit-1 counts of the key warps (fused tail), past both the scoring and
-  // the tail's shared-memory layouts
-  uint32_t* hist16 = reinterpret_cast<uint32_t*>(
-      smem + ((max(L.total, static_cast<uint32_t>(sizeof(TailSmem))) + 15u) & ~15u));
   // Row offsets as an extra K step of the contraction (32-byte swizzled,
   // K-major): key side [1, 1, 1, 0, ...], guide side (hi, mid, lo, 0, ...) with
   // hi + mid + lo = -lse[row] / sigma (three bf16 parts, exact to ~2^-24).
@@ -578,7 +567,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(drain, 1);
     for (int i = 0; i < 4; ++i) mbar_init(&pdone[i], 8 * nh);
     *abort_flag = 0;
-    *tiles_done = 0;
     fence_barrier_init();
   }
   grid_dep_launch();
@@ -688,9 +676,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0);
     }
     __syncwarp();
-  } else if (warp >= kKeyWarp0) {
-    if (p.tail)
-      tail_keys_in_loop(p, hist16, tiles_done, c, t0, nt, n, doc_lo, h, abort_flag);
   } else {
     // Two groups of eight warps take alternate jobs: job j = lt * nh + hh goes
     // to group j & 1, which drains TMEM buffer j & 1, so one group's TMEM loads
@@ -750,15 +735,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int key = (t0 + lt) * kKeyTile + kl;
           if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = s4 * p.inv_group;
         }
-        if (p.tail) {  // the tile's scores are in memory: tell the key warps (four warps per tile)
-          __syncwarp();
-          if (lane == 0) {
-            // tile 0's scores are also read by the previous CTA of the unit
-            if (lt == 0) __threadfence();
-            else __threadfence_block();
-            atomicAdd(tiles_done, 1);
-          }
-        }
       }
     }
   }
@@ -768,18 +744,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
-  if (p.tail)
-    keyscore_tail<D>(p, smem, hist16, b, h, c, p.docs.cta[b + 1] - p.docs.cta[b], t0, nt, n,
-                     doc_lo, abort_flag);
 }
 
 }  // namespace
-
-size_t keyscore_tail_smem_bytes(int head_dim, int rows_pad, int stages) {
-  const ScoreSmem L = score_layout(head_dim, rows_pad, stages, keyscore_extra_bytes(rows_pad));
-  const size_t hoff = (std::max<size_t>(L.total, sizeof(TailSmem)) + 15) & ~size_t(15);
-  return hoff + sizeof(uint32_t) * kTailBins1 / 2 + 1024;
-}
 
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
   (void)rows_pad;  // the guide rows live in tensor memory; V has its own ring

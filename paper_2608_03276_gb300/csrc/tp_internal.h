@@ -65,41 +65,7 @@ struct KeyScoreParams {
   const float* lse;  // [batch, H_kv, rows] natural log
   float* skey;       // [H_kv, N]
   int* status;
-
-  float qmax;
-
-  // The fused tail (a layer's selection and compaction run by the same CTAs
-  // after their scores; see tail.cuh).  Off when `tail` is 0.
-  int tail;
-  int pool_kernel;
-  int key_only;
-  int blend;                 // kBlendProduct or kBlendHarmonic (the normalised add is not fused)
-  int bits;
-  int64_t cap;
-  int32_t kept[kMaxBatch];   // k_b per document
-  const float* gamma;        // Eq. 2 scales [H_kv, N]
-  float* scores_out;         // optional combined scores [H_kv, N]
-  int32_t* idx;              // [batch, H_kv, cap]
-  const uint16_t* k;         // K, V [H_kv, N, d] (kept rows are copied from them)
-  const uint16_t* v;
-  uint16_t* kc;
-  uint16_t* vc;
-  int8_t* vqc;
-  float* gammac;
-  uint32_t* keys;            // [H_kv, N] radix keys of the combined scores
-  int* tsync;                // [H_kv * batch][2] arrival / departure counters, zero at launch
-  int* thist;                // [H_kv * batch][5120] radix histograms, zero at launch
-  int* tcount;               // [H_kv * grid.x][2] per-CTA (> T, == T) counts
-  int* tflag;                // [H_kv * grid.x] "first tile scored" flags, < epoch at launch
-  int epoch;                 // value a CTA writes to its flag (1 + layer index of a stack)
 };
-
-// Largest key range of one CTA for which the selection can run in pass 2's
-// tail (the range's radix keys stay in shared memory, with room for a pooling
-// half-window of slack at each end).
-constexpr int kTailMaxKeys = 16384;
-constexpr int kTailSlack = 64;
-constexpr int kTailHistInts = 2048 + 2048 + 1024;
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
 
@@ -191,8 +157,5 @@ cudaError_t set_smem_once(const void* kernel, int slot);
 // Shared-memory layout sizes of the scoring kernels (host side).
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages);
 size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages);
-// Pass 2 with the fused tail: the scoring layout, the tail's layout and the
-// digit-1 histogram that the key warps fill during the scoring loop.
-size_t keyscore_tail_smem_bytes(int head_dim, int rows_pad, int stages);
 
 }  // namespace tp

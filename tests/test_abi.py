@@ -157,19 +157,13 @@ def test_selftest_arguments(lib):
 
 
 def test_kernel_count_query(lib):
-    """The fused calls launch pass 1 (+ the prefix fold) and pass 2, which also
-    selects and compacts; the normalised add and key ranges beyond the tail's
-    shared memory add the selection and compaction kernels."""
+    """The fused calls launch pass 1 (or the V-scale pass), [the prefix fold,]
+    pass 2, the selection and, when anything is kept, the compaction."""
     p = lib.Problem(32, 8, 128, 128, [0, 131072])
-    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_TWO_PASS) == 2
-    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_CALLER_LSE) == 2
-    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_LITERAL) == 3
-    na = lib.Problem(32, 8, 128, 128, [0, 131072], flags=lib.TP_SCORE_NORM_ADD)
-    assert lib.tp_compress_kernel_count(na, 0.1, -1, lib.MODE_TWO_PASS) == 4
-    # one head of 4M tokens: over 16384 keys per CTA on any GPU of up to 256 SMs
-    big = lib.Problem(4, 1, 128, 16, [0, 1 << 22])
-    assert lib.tp_compress_kernel_count(big, 0.1, -1, lib.MODE_CALLER_LSE) == 4
-    assert lib.tp_compress_kernel_count(big, 0.0, -1, lib.MODE_CALLER_LSE) == 3
+    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_TWO_PASS) == 4
+    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_CALLER_LSE) == 4
+    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_LITERAL) == 5
+    assert lib.tp_compress_kernel_count(p, 0.0, -1, lib.MODE_TWO_PASS) == 3
     empty = lib.Problem(4, 1, 128, 16, [0, 0])
     assert lib.tp_compress_kernel_count(empty, 0.1, -1, lib.MODE_TWO_PASS) == 1
     with pytest.raises(lib.TaskPressError):
