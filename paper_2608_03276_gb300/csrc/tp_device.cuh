@@ -206,6 +206,13 @@ __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
 }
 // Waits for every cp.async this thread has issued.
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+// Closes this thread's current group of cp.async copies.
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Waits until at most N of this thread's committed groups are still in flight.
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 
 // Orders this thread's earlier generic-proxy shared-memory accesses before
 // later async-proxy ones (a TMA write into a buffer that was just read).
