@@ -447,7 +447,6 @@ cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s)
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int64_t n_max = 0;
   for (int b = 0; b < p.batch; ++b) n_max = p.off[b + 1] - p.off[b] > n_max ? p.off[b + 1] - p.off[b] : n_max;
-  if (n_max <= kSelect1MaxTokens) return launch_select1(p, dependent, s);
   // Fewer, larger slices when eight CTAs per unit would need more than one wave.
   // shared-memory attribute slots: 12..14 for four-CTA clusters, 15..17 for eight
   if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys)

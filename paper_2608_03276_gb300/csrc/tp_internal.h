@@ -145,12 +145,7 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUt
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             bool dependent, cudaStream_t s);
-// The selection: one CTA per (document, head) when every document has at most
-// kSelect1MaxTokens tokens (select1.cu), else one thread-block cluster per
-// (document, head) (select.cu).
-constexpr int64_t kSelect1MaxTokens = 65536;
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
-cudaError_t launch_select1(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
