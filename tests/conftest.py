@@ -26,9 +26,13 @@ def pytest_terminal_summary(terminalreporter):
     """Worst relative score error and near-tie kept-set differences of every
     parity test that compared scores with the oracle (tests/parity.py)."""
     from tests import parity
+    tr = terminalreporter
+    if parity.REPORTS:
+        tr.section("method-level figures (reported)")
+        for line in parity.REPORTS:
+            tr.write_line(line)
     if not parity.STATS:
         return
-    tr = terminalreporter
     tr.section("parity margins (bar: rel err <= 2e-3; kept sets equal outside near-ties)")
     worst = 0.0
     for test, st in sorted(parity.STATS.items()):

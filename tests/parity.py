@@ -25,6 +25,10 @@ TINY = 2.0 ** -100
 #: "near_tie_diffs": kept-set differences at near-ties of the cut-off}
 STATS: dict = {}
 
+#: method-level figures (recall of planted spans and the like), reported at
+#: the end of the run, not asserted
+REPORTS: list = []
+
 
 def _stat(key: str, value, how=max):
     import os
