@@ -29,7 +29,7 @@ Also reported on the same JSON line:
   clocks        nvidia-smi samples taken during the timed region;
   per_layer_calls  the same stack as one tp_compress_layer call per layer;
   graph_replay  the step's call captured as a CUDA graph and replayed;
-  lse_given     the same stack through tp_compress_layer_lse, the row
+  lse_given     the same stack through tp_compress_layers_lse, the row
                 normalisers supplied by the caller (one scoring pass over K);
   literal_normaliser  the same stack through tp_compress_layer_guide (the
                 guide's causal prefix folded into the normalisers).
@@ -563,8 +563,9 @@ def run_ours(args, w):
         lses.append(t)
 
     def step_lse():
-        for (q, k, v), o, t in zip(layers, outs, lses):
-            binding.compress(p, q, k, v, w.keep_ratio, w.budget, o, stream, lse=t)
+        # the whole stack in one call, each layer's V-scale pass beside the
+        # previous layer's selection
+        binding.tp_compress_layers_lse(p, layers, lses, w.keep_ratio, w.budget, outs, ws, stream)
 
     for _ in range(args.warmup):
         step_lse()
@@ -579,8 +580,8 @@ def run_ours(args, w):
                  "hbm_fused": hbm_fused_of(w, kept_tokens, ms_lse / L / 1e3, hbm_peak, peak_src),
                  "kernels_per_layer": binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget,
                                                                        binding.MODE_CALLER_LSE),
-                 "path": "tp_compress_layer_lse: caller row normalisers, one scoring pass over K, "
-                         "V scales from the quantiser pass"}
+                 "path": "tp_compress_layers_lse: caller row normalisers, one scoring pass over K, "
+                         "each layer's V-scale pass beside the previous layer's selection"}
     del lses
 
     # ---- the literal normaliser: guide keys given (tp_compress_layer_guide)

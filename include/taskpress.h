@@ -313,6 +313,21 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
                        void* stream);
 
 /*
+ * A stack of n_layers layers with the caller's row normalisers (as
+ * tp_compress_layer_lse, layer after layer, on `stream`); lse is a HOST array
+ * of n_layers device pointers, each [batch, H_kv, M] fp32 (natural log).
+ * Other arguments as in tp_compress_layers.  Each layer's Eq. 2 scale pass
+ * runs beside the previous layer's selection, on the SMs the selection leaves
+ * free.  Results equal n_layers calls of tp_compress_layer_lse bit for bit.
+ * ws_bytes as for tp_compress_layer.
+ */
+int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const* q,
+                           const void* const* k, const void* const* v, const float* const* lse,
+                           double keep_ratio, int64_t budget, int32_t* const* idx, void* const* kc,
+                           void* const* vc, int8_t* const* vqc, float* const* gammac, void* ws,
+                           size_t ws_bytes, void* stream);
+
+/*
  * How many kernels one fused call launches for this problem (mode 0:
  * tp_compress_layer, 1: tp_compress_layer_lse, 2: tp_compress_layer_guide;
  * tp_compress_layers launches mode 0's count per layer); -1 on invalid

@@ -33,7 +33,8 @@ EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v
            "tp_select", "tp_compact",
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
            "tp_compress_layer_guide", "tp_compress_layers", "tp_quantize_rows", "tp_check_status",
-           "tp_selftest_wait_timeout", "tp_status_string", "tp_compress_kernel_count")
+           "tp_selftest_wait_timeout", "tp_status_string", "tp_compress_kernel_count",
+           "tp_compress_layers_lse")
 
 
 class TpProblem(ctypes.Structure):
@@ -119,6 +120,10 @@ def load(path: Optional[str] = None):
     lib.tp_check_status.argtypes = [c_void_p, c_size_t, c_void_p]
     lib.tp_status_string.restype = ctypes.c_char_p
     lib.tp_status_string.argtypes = [c_int]
+    lib.tp_compress_layers_lse.restype = c_int
+    lib.tp_compress_layers_lse.argtypes = [POINTER(TpProblem), c_int, c_void_p, c_void_p, c_void_p,
+                                           c_void_p, c_double, c_int64, c_void_p, c_void_p, c_void_p,
+                                           c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]
     lib.tp_compress_kernel_count.restype = c_int
     lib.tp_compress_kernel_count.argtypes = [POINTER(TpProblem), c_double, c_int64, c_int]
     _lib = lib
@@ -406,6 +411,39 @@ def tp_compress_layers(p: Problem, layers, keep_ratio: float, budget: int, outs,
     gc = arr(_ptr(o.gammac, torch.float32, m, "gammac", nullable=True) for o in outs)
     _check("tp_compress_layers", load().tp_compress_layers(
         p.ref(), n, q, k, v, keep_ratio, budget, idx, kc, vc, vqc, gc,
+        _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
+
+
+def tp_compress_layers_lse(p: Problem, layers, lses, keep_ratio: float, budget: int, outs, ws,
+                           stream=None):
+    """A stack of layers with the caller's row normalisers: `lses` holds one
+    [batch, H_kv, M] fp32 tensor per layer; otherwise as tp_compress_layers."""
+    import torch
+    n = len(layers)
+    if len(outs) != n or len(lses) != n:
+        raise ValueError("one CompressOutputs and one lse tensor per layer")
+    hq, hkv, d, lt, nt = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
+    rows = (hq // hkv) * lt
+    cap = tp_kept_capacity(p, keep_ratio, budget)
+    m = p.batch * hkv * cap
+
+    def arr(ptrs):
+        a = (c_void_p * max(1, n))()
+        for i, x in enumerate(ptrs):
+            a[i] = x
+        return a
+
+    q = arr(_ptr(x[0], torch.bfloat16, p.batch * hq * lt * d, "q") for x in layers)
+    k = arr(_ptr(x[1], torch.bfloat16, hkv * nt * d, "k") for x in layers)
+    v = arr(_ptr(x[2], torch.bfloat16, hkv * nt * d, "v") for x in layers)
+    ls = arr(_ptr(t, torch.float32, p.batch * hkv * rows, "lse") for t in lses)
+    idx = arr(_ptr(o.idx, torch.int32, m, "idx", nullable=cap == 0) for o in outs)
+    kc = arr(_ptr(o.kc, torch.bfloat16, m * d, "kc", nullable=True) for o in outs)
+    vc = arr(_ptr(o.vc, torch.bfloat16, m * d, "vc", nullable=True) for o in outs)
+    vqc = arr(_codes(p, o.vqc, m, "vqc") for o in outs)
+    gc = arr(_ptr(o.gammac, torch.float32, m, "gammac", nullable=True) for o in outs)
+    _check("tp_compress_layers_lse", load().tp_compress_layers_lse(
+        p.ref(), n, q, k, v, ls, keep_ratio, budget, idx, kc, vc, vqc, gc,
         _ptr(ws, torch.uint8, None, "ws"), ws.numel(), _stream(stream)))
 
 

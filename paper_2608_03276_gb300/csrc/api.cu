@@ -32,7 +32,7 @@ struct Plan {
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
-  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_skey2, ws_gamma, ws_gamma2, ws_keys, ws_total;
 };
 
 int num_sms() {
@@ -151,6 +151,12 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_gamma = o;
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
+  // second key-score and scale buffers: a stack with the caller's normalisers
+  // alternates between two of each
+  P->ws_skey2 = o;
+  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
+  P->ws_gamma2 = o;
+  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_keys = o;
   o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
   P->ws_total = o;
@@ -249,7 +255,7 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
 
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
 int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const float* lse,
-                 float* skey, int* status, bool dependent, cudaStream_t s) {
+                 float* skey, int* status, bool dependent, cudaStream_t s, bool wait_at_end = false) {
   KeyScoreParams kp;
   memset(&kp, 0, sizeof(kp));
   kp.docs = doc_table(P);
@@ -265,6 +271,7 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
   kp.lse = lse;
   kp.skey = skey;
   kp.status = status;
+  kp.wait_at_end = wait_at_end ? 1 : 0;
   return cuda_status(
       launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
 }
@@ -739,6 +746,96 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
     sp.gamma = g;
     sp.idx = idx ? idx[l] : nullptr;
     if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
+    if (P.cap == 0) continue;
+    GatherParams gp;
+    fill_gather(P, &gp);
+    gp.k = static_cast<const uint16_t*>(k[l]);
+    gp.v = static_cast<const uint16_t*>(v[l]);
+    gp.gamma = g;
+    gp.idx = idx[l];
+    gp.kc = kc ? static_cast<uint16_t*>(kc[l]) : nullptr;
+    gp.vc = vc ? static_cast<uint16_t*>(vc[l]) : nullptr;
+    gp.vqc = vqc ? vqc[l] : nullptr;
+    gp.gammac = gammac ? gammac[l] : nullptr;
+    if ((st = cuda_status(launch_gather(gp, true, s))) != TP_OK) return st;
+  }
+  return TP_OK;
+}
+
+int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const* q,
+                           const void* const* k, const void* const* v, const float* const* lse,
+                           double keep_ratio, int64_t budget, int32_t* const* idx, void* const* kc,
+                           void* const* vc, int8_t* const* vqc, float* const* gammac, void* ws,
+                           size_t ws_bytes, void* stream) {
+  Plan P;
+  int st = make_plan(p, keep_ratio, budget, true, &P);
+  if (st != TP_OK) return st;
+  if (n_layers < 0 || (n_layers > 0 && (!q || !k || !v || !lse || (!idx && P.cap > 0))))
+    return TP_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!q[l] || !k[l] || !v[l] || !lse[l] || !aligned16(q[l]) || !aligned16(k[l]) ||
+        !aligned16(v[l]))
+      return TP_ERR_INVALID_ARG;
+    if (P.cap > 0 && !idx[l]) return TP_ERR_INVALID_ARG;
+    if ((kc && kc[l] && !aligned16(kc[l])) || (vc && vc[l] && !aligned16(vc[l])) ||
+        (vqc && vqc[l] && (reinterpret_cast<uintptr_t>(vqc[l]) & code_align(P))))
+      return TP_ERR_INVALID_ARG;
+  }
+  if (!ws || ws_bytes < P.ws_total || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)))
+    return TP_ERR_WORKSPACE;
+  if (n_layers == 0) return TP_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  float* const gbuf[2] = {reinterpret_cast<float*>(w + P.ws_gamma),
+                          reinterpret_cast<float*>(w + P.ws_gamma2)};
+  float* const kbuf[2] = {reinterpret_cast<float*>(w + P.ws_skey),
+                          reinterpret_cast<float*>(w + P.ws_skey2)};
+  int* const status = reinterpret_cast<int*>(w + P.ws_status);
+  const int sms = num_sms();
+  const bool scored = P.n_total > 0 && P.grid_x > 0;
+  if ((st = zero_head(P, w, s)) != TP_OK) return st;
+  // Per layer l: the V scales, pass 2, the selection, the compaction.  Layer
+  // l + 1's V scales are launched right after layer l's selection, as its
+  // dependent: they run on the SMs the selection leaves free (it occupies one
+  // cluster per document and head) and wait for it only at their end; layer
+  // l's compaction follows them.  Layers alternate between two scale and two
+  // key-score buffers.  Why no kernel overwrites what an earlier one still
+  // reads: pass 2 waits for its predecessor (the previous layer's compaction)
+  // at its end and lets its dependents start only when it exits, so layer
+  // l's selection starts after layer l - 1's compaction has completed, which
+  // itself waited for layer l's scales, which waited for layer l - 1's
+  // selection.  Layer l + 1's scales, started next to layer l's selection,
+  // therefore find layer l - 1's compaction (the last reader of their buffer)
+  // complete, and layer l + 1's pass 2 finds layer l - 1's selection (the
+  // last reader of its key-score buffer) complete.
+  auto scales = [&](int l, bool dependent) -> int {
+    if (!scored) return TP_OK;
+    const cudaError_t e =
+        dependent ? launch_vquant_dependent(static_cast<const uint16_t*>(v[l]), gbuf[l & 1],
+                                            int64_t(P.hkv) * P.n_total, P.d, P.qmax, sms, s)
+                  : launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, gbuf[l & 1],
+                                  int64_t(P.hkv) * P.n_total, P.d, P.qmax, P.bits, sms, s);
+    return cuda_status(e);
+  };
+  if ((st = scales(0, false)) != TP_OK) return st;
+  for (int l = 0; l < n_layers; ++l) {
+    float* const g = gbuf[l & 1];
+    float* const skey = kbuf[l & 1];
+    if (scored) {
+      CUtensorMap tmk, tmq;
+      if (!encode_maps(P, q[l], k[l], &tmk, &tmq)) return TP_ERR_CUDA;
+      if ((st = run_keyscore(P, tmk, tmq, lse[l], skey, status, true, s, true)) != TP_OK) return st;
+    }
+    SelectParams sp;
+    fill_select(P, w, &sp);
+    sp.pool_kernel = p->pool_kernel;
+    sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
+    sp.blend = blend_of(p->flags);
+    sp.skey = skey;
+    sp.gamma = g;
+    sp.idx = idx ? idx[l] : nullptr;
+    if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
+    if (l + 1 < n_layers && (st = scales(l + 1, true)) != TP_OK) return st;
     if (P.cap == 0) continue;
     GatherParams gp;
     fill_gather(P, &gp);

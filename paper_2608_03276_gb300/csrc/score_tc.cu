@@ -569,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  grid_dep_launch();
+  if (!p.wait_at_end) grid_dep_launch();
   if (warp == 0) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
@@ -592,7 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[lt]);
     }
   }
-  grid_dep_wait();  // the row normalisers come from pass 1
+  if (!p.wait_at_end) grid_dep_wait();  // the row normalisers come from pass 1
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
     for (int r = threadIdx.x; r < 128 + rows_pad; r += blockDim.x) {
@@ -744,6 +744,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
+  // complete only after the predecessor: the kernels after this one rely on
+  // everything before it having finished
+  if (p.wait_at_end) grid_dep_wait();
 }
 
 }  // namespace

@@ -65,6 +65,10 @@ struct KeyScoreParams {
   const float* lse;  // [batch, H_kv, rows] natural log
   float* skey;       // [H_kv, N]
   int* status;
+  // The normalisers are inputs of the call, not the previous kernel's output:
+  // no wait before reading them; the kernel waits for its predecessor at its
+  // end instead, and its dependents start only when it exits.
+  int wait_at_end;
 };
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
@@ -133,6 +137,12 @@ struct PrefixParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int bits, int num_sms, cudaStream_t s);
+// The quantiser as a programmatic dependent of the previous kernel, which it
+// lets its own dependents overlap: it starts at once (its input is the
+// layer's V, written before the call) and waits for the previous kernel only
+// at its end.
+cudaError_t launch_vquant_dependent(const uint16_t* v, float* gamma, int64_t rows, int head_dim,
+                                    float qmax, int num_sms, cudaStream_t s);
 // Pass 1.  `dependent`: launched as a programmatic dependent of the previous
 // layer's last kernel (a stack of layers in one call); it then waits for that
 // kernel before its first store.

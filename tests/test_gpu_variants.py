@@ -260,6 +260,68 @@ def test_layer_stack_matches_single_layers(cuda_lib, name, bits):
         _check_layer(w, x, single, _oracle(w, x, quant_bits=bits), bits=bits)
 
 
+@pytest.mark.parametrize("name,bits,nl", [("c2-llama-4133", 8, 4), ("c5-ragged", 8, 3),
+                                          ("c1-tiny-2k", 4, 3)])
+def test_lse_stack_matches_single_layers(cuda_lib, name, bits, nl):
+    """tp_compress_layers_lse (each layer's scale pass running beside the
+    previous layer's selection, two alternating scale and key-score buffers)
+    equals one tp_compress_layer_lse call per layer bit for bit, and the
+    oracle given the same normalisers on every layer.  The normalisers carry
+    extra per-row mass, as a prefill's would."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    xs = _stack(w, nl)
+    p = _problem(binding, w, xs[0].doc_offsets, quant_bits=bits)
+    dev = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in xs]
+    rng = np.random.Generator(np.random.PCG64(31))
+    lses = []
+    for x in xs:
+        ctx = _context_lse(w, x)
+        lses.append(np.logaddexp(ctx.astype(np.float64),
+                                 ctx + rng.uniform(-2.0, 2.0, ctx.shape)).astype(np.float32))
+    dl = [torch.tensor(t, device="cuda") for t in lses]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+    binding.tp_compress_layers_lse(p, dev, dl, w.keep_ratio, w.budget, outs, outs[0].ws)
+    assert binding.tp_check_status(outs[0].ws) == 0
+    for l, x in enumerate(xs):
+        single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *dev[l], w.keep_ratio, w.budget, single, lse=dl[l])
+        _outputs_equal(outs[l], single, f"layer {l}")
+        _check_layer(w, x, single, _oracle(w, x, quant_bits=bits, lse=lses[l].astype(np.float64)),
+                     bits=bits)
+
+
+def test_full_size_lse_stack(cuda_lib):
+    """Three 128K layers through tp_compress_layers_lse, the benchmark's
+    caller-normaliser leg: each equals a single tp_compress_layer_lse call bit
+    for bit, and every KV head of the last layer matches the oracle."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    from tests import oracle_pool
+    w = synth.WORKLOADS[3]
+    xs = [synth.make_layer(w, l) for l in (0, 1, 2)]
+    p = _problem(binding, w, xs[0].doc_offsets)
+    dev = [tuple(parity.to_device_bf16(t) for t in (y.q, y.k, y.v)) for y in xs]
+    ws = torch.empty(binding.tp_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    dl = []
+    for q, k, _ in dev:
+        t = torch.empty((w.batch, w.n_heads_kv, w.rows), dtype=torch.float32, device="cuda")
+        binding.tp_guide_lse(p, q, k, t, ws)
+        dl.append(t)
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+    binding.tp_compress_layers_lse(p, dev, dl, w.keep_ratio, w.budget, outs, outs[0].ws)
+    assert binding.tp_check_status(outs[0].ws) == 0
+    for l in range(3):
+        single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *dev[l], w.keep_ratio, w.budget, single, lse=dl[l])
+        _outputs_equal(outs[l], single, f"lse stack layer {l}")
+    x = xs[2]
+    ref = oracle_pool.compress_layer(x, w.n_heads_q, w.n_heads_kv, keep_ratio=w.keep_ratio,
+                                     lse=dl[2].cpu().numpy().astype(np.float64))
+    _check_layer(w, x, single, ref)
+
+
 def test_layer_stack_graph_replay(cuda_lib):
     """The stack captured into a CUDA graph (its memset and dependent launches
     become graph nodes) and replayed on new contents of the same input
