@@ -563,8 +563,8 @@ def run_ours(args, w):
         lses.append(t)
 
     def step_lse():
-        # the whole stack in one call, each layer's V-scale pass beside the
-        # previous layer's selection
+        # the whole stack in one call: per layer one kernel for the key scores
+        # and the V scales (K and V read once), the selection, the compaction
         binding.tp_compress_layers_lse(p, layers, lses, w.keep_ratio, w.budget, outs, ws, stream)
 
     for _ in range(args.warmup):
@@ -580,8 +580,9 @@ def run_ours(args, w):
                  "hbm_fused": hbm_fused_of(w, kept_tokens, ms_lse / L / 1e3, hbm_peak, peak_src),
                  "kernels_per_layer": binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget,
                                                                        binding.MODE_CALLER_LSE),
-                 "path": "tp_compress_layers_lse: caller row normalisers, one scoring pass over K, "
-                         "each layer's V-scale pass beside the previous layer's selection"}
+                 "path": "tp_compress_layers_lse: caller row normalisers; per layer one kernel reads K "
+                         "and V once for the key scores and the Eq. 2 scales (CTA pairs above 256 "
+                         "guide rows), then the selection and the compaction"}
     del lses
 
     # ---- the literal normaliser: guide keys given (tp_compress_layer_guide)

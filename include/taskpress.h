@@ -260,7 +260,12 @@ int tp_compress_layer(const tp_problem* p, const void* q, const void* k, const v
  * that attention's per-row log-sum-exp for the guide rows passes it here and
  * gets the paper's literal normaliser, which also counts the guide's own
  * causal prefix.  With lse from tp_guide_lse the result equals
- * tp_compress_layer's.  The Eq. 2 scales come from a separate pass over V.
+ * tp_compress_layer's.  The same kernel forms the key scores and the Eq. 2
+ * scales, so K and V are each read once: one CTA per key range for up to 256
+ * guide rows, two-CTA clusters sharing each tensor-core MMA (each CTA holding
+ * half of the guide block) above.  Where those pairs would not all be
+ * resident at once (more than 76 (document, KV head) units of more than 256
+ * rows on a 152-SM GPU) the scales come from a separate pass over V.
  * Other arguments, outputs and workspace as in tp_compress_layer.
  */
 int tp_compress_layer_lse(const tp_problem* p, const void* q, const void* k, const void* v,
@@ -316,9 +321,10 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
  * A stack of n_layers layers with the caller's row normalisers (as
  * tp_compress_layer_lse, layer after layer, on `stream`); lse is a HOST array
  * of n_layers device pointers, each [batch, H_kv, M] fp32 (natural log).
- * Other arguments as in tp_compress_layers.  Each layer's Eq. 2 scale pass
- * runs beside the previous layer's selection, on the SMs the selection leaves
- * free.  Results equal n_layers calls of tp_compress_layer_lse bit for bit.
+ * Other arguments as in tp_compress_layers.  Each layer's scoring kernel is a
+ * programmatic dependent of the previous layer's compaction: it loads and
+ * scores at once and waits for that kernel only before its first store.
+ * Results equal n_layers calls of tp_compress_layer_lse bit for bit.
  * ws_bytes as for tp_compress_layer.
  */
 int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const* q,
@@ -330,8 +336,10 @@ int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const*
 /*
  * How many kernels one fused call launches for this problem (mode 0:
  * tp_compress_layer, 1: tp_compress_layer_lse, 2: tp_compress_layer_guide;
- * tp_compress_layers launches mode 0's count per layer); -1 on invalid
- * arguments.  A planning query: it launches nothing.
+ * tp_compress_layers launches mode 0's count per layer, tp_compress_layers_lse
+ * mode 1's); -1 on invalid arguments.  A planning query: it launches nothing
+ * (for mode 1 above 256 guide rows it asks the current device how many CTA
+ * pairs can be resident; without a device it counts the separate V pass).
  */
 int tp_compress_kernel_count(const tp_problem* p, double keep_ratio, int64_t budget, int mode);
 

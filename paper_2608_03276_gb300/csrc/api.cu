@@ -26,13 +26,18 @@ struct Plan {
   int32_t cta[kMaxBatch + 1];
   int stages1, stages2;
   size_t smem1, smem2;
+  // pass 2 forming the Eq. 2 scales too (caller's normalisers): K stages and
+  // shared memory, stages2s = 0 where two K stages and the V ring do not fit
+  // next to the guide block (more than 256 guide rows: CTA pairs then)
+  int stages2s;
+  size_t smem2s;
   float c2, inv_group, sigma;
   int bits;     // Eq. 2 code width: 8 or 4
   float qmax;   // 2^(bits-1) - 1
   int32_t kept[kMaxBatch];
   int64_t cap;
   // workspace offsets
-  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_skey2, ws_gamma, ws_gamma2, ws_keys, ws_total;
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
 };
 
 int num_sms() {
@@ -117,15 +122,21 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->stages1 = 6;  // K ring of pass 1 (next to its V ring)
   while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
   P->stages2 = 4;
-  while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2) > kMaxSmem) --P->stages2;
+  while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false) > kMaxSmem)
+    --P->stages2;
   P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
   // pass 1 stages the guide block, and at the end its row statistics, through
   // its K ring
   if (size_t(P->stages1) * (P->d / 64) * 16384 <
       std::max(size_t(P->d / 64) * P->rows_pad * 128, size_t(4) * P->rows_pad * sizeof(float2)))
     return TP_ERR_UNSUPPORTED_SHAPE;
-  P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2);
+  P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false);
   if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
+  P->stages2s = 4;
+  while (P->stages2s >= 2 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) > kMaxSmem)
+    --P->stages2s;
+  if (P->stages2s < 2) P->stages2s = 0;
+  P->smem2s = P->stages2s ? keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) : 0;
 
   P->cap = 0;
   if (need_select) {
@@ -150,12 +161,6 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->ws_skey = o;
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_gamma = o;
-  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
-  // second key-score and scale buffers: a stack with the caller's normalisers
-  // alternates between two of each
-  P->ws_skey2 = o;
-  o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
-  P->ws_gamma2 = o;
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_keys = o;
   o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
@@ -253,9 +258,49 @@ int run_lse(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const
       launch_lse(tmk, tmv, tmq, lp, P.d, dim3(P.grid_x, P.hkv), P.smem1, dependent, s));
 }
 
+// Pass 2 with the Eq. 2 scales on CTA pairs: tiles of 256 keys, the smallest
+// count per pair whose pairs (over all heads) are resident at once, and the
+// deepest K ring that fits next to half of the guide block and the V ring.
+struct PairGeometry {
+  int tiles;                   // pair tiles per pair
+  int pairs;                   // pairs per head
+  int32_t cta[kMaxBatch + 1];  // pair prefix per document
+  int stages;
+  size_t smem;
+};
+
+bool pair_geometry(const Plan& P, PairGeometry* G) {
+  G->stages = 4;
+  while (G->stages > 1 && keyscore_pair_smem_bytes(P.d, P.rows_mma, G->stages) > size_t(kMaxSmem))
+    --G->stages;
+  G->smem = keyscore_pair_smem_bytes(P.d, P.rows_mma, G->stages);
+  if (G->smem > size_t(kMaxSmem)) return false;
+  const int clusters = keyscore_pair_max_clusters(P.d, G->smem);
+  if (clusters <= 0) return false;
+  int64_t tiles_total = 0;
+  for (int b = 0; b < P.batch; ++b) tiles_total += (P.off[b + 1] - P.off[b] + 255) / 256;
+  tiles_total *= P.hkv;
+  int64_t T = tiles_total > 0 ? (tiles_total + clusters - 1) / clusters : 1;
+  if (T < 1) T = 1;
+  int64_t pairs = 0;
+  for (int iter = 0; iter < 64; ++iter) {
+    pairs = 0;
+    for (int b = 0; b < P.batch; ++b) pairs += ((P.off[b + 1] - P.off[b] + 255) / 256 + T - 1) / T;
+    if (pairs * P.hkv <= clusters) break;
+    ++T;
+  }
+  if (pairs * P.hkv > clusters || pairs == 0) return false;
+  G->tiles = static_cast<int>(T);
+  G->cta[0] = 0;
+  for (int b = 0; b < P.batch; ++b)
+    G->cta[b + 1] = G->cta[b] + static_cast<int32_t>(((P.off[b + 1] - P.off[b] + 255) / 256 + T - 1) / T);
+  G->pairs = G->cta[P.batch];
+  return true;
+}
+
 // Pass 2: unpooled key scores [H_kv, N] from the row normalisers.
-int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, const float* lse,
-                 float* skey, int* status, bool dependent, cudaStream_t s, bool wait_at_end = false) {
+int run_keyscore(const Plan& P, const CUtensorMap& tmk, const void* q, const float* lse,
+                 float* skey, int* status, bool dependent, cudaStream_t s) {
   KeyScoreParams kp;
   memset(&kp, 0, sizeof(kp));
   kp.docs = doc_table(P);
@@ -271,9 +316,64 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const CUtensorMap& tmq, 
   kp.lse = lse;
   kp.skey = skey;
   kp.status = status;
-  kp.wait_at_end = wait_at_end ? 1 : 0;
+  CUtensorMap tmq;
+  if (!encode_3d(&tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv, P.rows_pad < 256 ? P.rows_pad : 256))
+    return TP_ERR_CUDA;
   return cuda_status(
-      launch_keyscore(tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
+      launch_keyscore(tmk, tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
+}
+
+// With the caller's row normalisers: the key scores and the Eq. 2 scales of
+// every token in one kernel (K and V each read once): one CTA per key range
+// with up to 256 guide rows, CTA pairs above (each CTA then holds half of the
+// guide block).  Returns kNoFusedScales, launching nothing, where neither fits
+// (pairs that would not all be resident at once); the caller then runs the
+// quantiser and pass 2.
+constexpr int kNoFusedScales = 1;  // positive: every TP_ERR_* code is negative
+
+bool fused_scales_fit(const Plan& P) {
+  PairGeometry G;
+  return P.stages2s > 0 || pair_geometry(P, &G);
+}
+
+int run_keyscore_scales(const Plan& P, const void* q, const void* k, const void* v,
+                        const float* lse, float* skey, float* gamma, int* status, bool dependent,
+                        cudaStream_t s) {
+  PairGeometry G;
+  const bool single = P.stages2s > 0;
+  if (!single && !pair_geometry(P, &G)) return kNoFusedScales;
+  CUtensorMap tmk, tmv, tmq;
+  const int qbox = single ? (P.rows_pad < 256 ? P.rows_pad : 256) : 128;
+  if (!encode_3d(&tmk, k, P.d, P.n_total, P.hkv, 128) ||
+      !encode_3d(&tmv, v, P.d, P.n_total, P.hkv, 128) ||
+      !encode_3d(&tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv, qbox))
+    return TP_ERR_CUDA;
+  KeyScoreParams kp;
+  memset(&kp, 0, sizeof(kp));
+  kp.docs = doc_table(P);
+  kp.n_heads_kv = P.hkv;
+  kp.rows = P.rows;
+  kp.rows_pad = P.rows_pad;
+  kp.rows_mma = P.rows_mma;
+  kp.c2 = P.c2;
+  kp.inv_group = P.inv_group;
+  kp.n_total = P.n_total;
+  kp.lse = lse;
+  kp.skey = skey;
+  kp.gamma = gamma;
+  kp.qmax = P.qmax;
+  kp.status = status;
+  if (single) {
+    kp.tiles_per_cta = P.tiles_per_cta;
+    kp.stages = P.stages2s;
+    return cuda_status(
+        launch_keyscore(tmk, tmv, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2s, dependent, s));
+  }
+  for (int b = 0; b <= P.batch; ++b) kp.docs.cta[b] = G.cta[b];
+  kp.tiles_per_cta = G.tiles;
+  kp.stages = G.stages;
+  return cuda_status(launch_keyscore_pair(tmk, tmv, tmq, kp, P.d, dim3(2 * G.pairs, P.hkv), G.smem,
+                                          dependent, s));
 }
 
 // The guide-prefix fold of the literal normaliser (`lse` in place).
@@ -306,7 +406,7 @@ int run_scoring(const Plan& P, const void* q, const void* k, const void* v, floa
   int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s, dependent);
   if (st != TP_OK) return st;
   if (k_guide && (st = run_prefix(P, q, k_guide, lse, true, s)) != TP_OK) return st;
-  return run_keyscore(P, tmk, tmq, lse, reinterpret_cast<float*>(ws + P.ws_skey),
+  return run_keyscore(P, tmk, q, lse, reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), true, s);
 }
 
@@ -372,14 +472,18 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   if (!lse_in) {
     if ((st = run_scoring(P, q, k, v, g, w, s, k_guide)) != TP_OK) return st;
   } else if (P.n_total > 0 && P.grid_x > 0) {
-    if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
-                      P.qmax, P.bits, num_sms(), s) != cudaSuccess)
-      return TP_ERR_CUDA;
-    CUtensorMap tmk, tmq;
-    if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-    if ((st = run_keyscore(P, tmk, tmq, lse_in, reinterpret_cast<float*>(w + P.ws_skey),
-                           reinterpret_cast<int*>(w + P.ws_status), false, s)) != TP_OK)
-      return st;
+    float* const skey = reinterpret_cast<float*>(w + P.ws_skey);
+    int* const status = reinterpret_cast<int*>(w + P.ws_status);
+    st = run_keyscore_scales(P, q, k, v, lse_in, skey, g, status, false, s);
+    if (st == kNoFusedScales) {
+      if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, g, int64_t(P.hkv) * P.n_total, P.d,
+                        P.qmax, P.bits, num_sms(), s) != cudaSuccess)
+        return TP_ERR_CUDA;
+      CUtensorMap tmk, tmq;
+      if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
+      st = run_keyscore(P, tmk, q, lse_in, skey, status, true, s);
+    }
+    if (st != TP_OK) return st;
   }
   SelectParams sp;
   fill_select(P, w, &sp);
@@ -635,7 +739,7 @@ int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_keyscore(P, tmk, tmq, lse, key_scores, nullptr, false,
+  return run_keyscore(P, tmk, q, lse, key_scores, nullptr, false,
                       static_cast<cudaStream_t>(stream));
 }
 
@@ -786,45 +890,31 @@ int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const*
   if (n_layers == 0) return TP_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  float* const gbuf[2] = {reinterpret_cast<float*>(w + P.ws_gamma),
-                          reinterpret_cast<float*>(w + P.ws_gamma2)};
-  float* const kbuf[2] = {reinterpret_cast<float*>(w + P.ws_skey),
-                          reinterpret_cast<float*>(w + P.ws_skey2)};
+  float* const g = reinterpret_cast<float*>(w + P.ws_gamma);
+  float* const skey = reinterpret_cast<float*>(w + P.ws_skey);
   int* const status = reinterpret_cast<int*>(w + P.ws_status);
-  const int sms = num_sms();
   const bool scored = P.n_total > 0 && P.grid_x > 0;
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  // Per layer l: the V scales, pass 2, the selection, the compaction.  Layer
-  // l + 1's V scales are launched right after layer l's selection, as its
-  // dependent: they run on the SMs the selection leaves free (it occupies one
-  // cluster per document and head) and wait for it only at their end; layer
-  // l's compaction follows them.  Layers alternate between two scale and two
-  // key-score buffers.  Why no kernel overwrites what an earlier one still
-  // reads: pass 2 waits for its predecessor (the previous layer's compaction)
-  // at its end and lets its dependents start only when it exits, so layer
-  // l's selection starts after layer l - 1's compaction has completed, which
-  // itself waited for layer l's scales, which waited for layer l - 1's
-  // selection.  Layer l + 1's scales, started next to layer l's selection,
-  // therefore find layer l - 1's compaction (the last reader of their buffer)
-  // complete, and layer l + 1's pass 2 finds layer l - 1's selection (the
-  // last reader of its key-score buffer) complete.
-  auto scales = [&](int l, bool dependent) -> int {
-    if (!scored) return TP_OK;
-    const cudaError_t e =
-        dependent ? launch_vquant_dependent(static_cast<const uint16_t*>(v[l]), gbuf[l & 1],
-                                            int64_t(P.hkv) * P.n_total, P.d, P.qmax, sms, s)
-                  : launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, gbuf[l & 1],
-                                  int64_t(P.hkv) * P.n_total, P.d, P.qmax, P.bits, sms, s);
-    return cuda_status(e);
-  };
-  if ((st = scales(0, false)) != TP_OK) return st;
+  // Per layer: the key scores with the Eq. 2 scales (one kernel on CTA pairs),
+  // the selection, the compaction, each a programmatic dependent of the
+  // kernel before it.  Layer l + 1's scoring kernel loads and scores while
+  // layer l's compaction finishes and waits for it only before its first
+  // store; that compaction completes after layer l's selection (it waited for
+  // it), which was the last reader of the key scores, and is itself the last
+  // reader of the scales, so one buffer of each serves every layer.  Without
+  // resident pairs each layer runs the quantiser and pass 2 instead.
   for (int l = 0; l < n_layers; ++l) {
-    float* const g = gbuf[l & 1];
-    float* const skey = kbuf[l & 1];
     if (scored) {
-      CUtensorMap tmk, tmq;
-      if (!encode_maps(P, q[l], k[l], &tmk, &tmq)) return TP_ERR_CUDA;
-      if ((st = run_keyscore(P, tmk, tmq, lse[l], skey, status, true, s, true)) != TP_OK) return st;
+      st = run_keyscore_scales(P, q[l], k[l], v[l], lse[l], skey, g, status, l > 0, s);
+      if (st == kNoFusedScales) {
+        if (launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, g, int64_t(P.hkv) * P.n_total,
+                          P.d, P.qmax, P.bits, num_sms(), s) != cudaSuccess)
+          return TP_ERR_CUDA;
+        CUtensorMap tmk, tmq;
+        if (!encode_maps(P, q[l], k[l], &tmk, &tmq)) return TP_ERR_CUDA;
+        st = run_keyscore(P, tmk, q[l], lse[l], skey, status, true, s);
+      }
+      if (st != TP_OK) return st;
     }
     SelectParams sp;
     fill_select(P, w, &sp);
@@ -835,7 +925,6 @@ int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const*
     sp.gamma = g;
     sp.idx = idx ? idx[l] : nullptr;
     if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
-    if (l + 1 < n_layers && (st = scales(l + 1, true)) != TP_OK) return st;
     if (P.cap == 0) continue;
     GatherParams gp;
     fill_gather(P, &gp);
@@ -865,8 +954,12 @@ int tp_compress_kernel_count(const tp_problem* p, double keep_ratio, int64_t bud
   Plan P;
   if (mode < 0 || mode > 2 || make_plan(p, keep_ratio, budget, true, &P) != TP_OK) return -1;
   int kernels = P.cap > 0 ? 2 : 1;  // selection [+ compaction]
-  if (P.n_total > 0 && P.grid_x > 0)
-    kernels += mode == 2 ? 3 : 2;  // pass 1 (or the V scales for mode 1), [prefix fold,] pass 2
+  if (P.n_total > 0 && P.grid_x > 0) {
+    if (mode == 1)  // the key scores with the scales in one kernel, else the quantiser and pass 2
+      kernels += fused_scales_fit(P) ? 1 : 2;
+    else
+      kernels += mode == 2 ? 3 : 2;  // pass 1, [prefix fold,] pass 2
+  }
   return kernels;
 }
 

@@ -20,6 +20,8 @@
 //   warps 2-17  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
 #include <math.h>
 
+#include <mutex>
+
 #include "tp_device.cuh"
 
 namespace tp {
@@ -30,6 +32,7 @@ constexpr int kThreads = 576;      // pass 2: TMA, MMA, 16 epilogue warps
 constexpr int kLseThreads = 640;   // pass 1: the same plus 2 V-scale warps
 constexpr int kVWarp0 = 18;        // first V-scale warp of pass 1
 constexpr int kVStages = 3;        // V-tile ring depth of pass 1
+constexpr int kVStages2 = 2;       // V-tile ring depth of pass 2 when it forms the scales
 constexpr int kEpiWarp0 = 2;  // first epilogue warp
 constexpr int kEpiWarps = 16;  // four warpgroups
 constexpr uint32_t kHalfTileBytes = 128 * 128;  // 128 keys x 64 bf16
@@ -142,6 +145,35 @@ __device__ __forceinline__ void lse_chunk64(uint32_t (&ra)[32], uint32_t (&rb)[3
   }
 }
 
+
+// Eq. 2 scales of the 128 V rows of one staged, 128-byte-swizzled tile: V
+// warp vw (of two) reduces rows 64 vw .. 64 vw + 63, two per lane.  The
+// swizzle only permutes 16-byte chunks within a row, so a row's absmax may read
+// its chunks in any order: lane l reads chunk position cc ^ (row & 7), so that
+// eight consecutive rows cover all banks at every step.  Row r's scale goes to
+// gamma_rows[r] for r < valid (absmax as bf16 bits, then one IEEE division).
+template <int NKH>
+__device__ __forceinline__ void vscale_tile(const uint8_t* tile, int vw, int lane, float* gamma_rows,
+                                            int valid, float qmax) {
+#pragma unroll
+  for (int rr = 0; rr < 2; ++rr) {
+    const int r = vw * 64 + rr * 32 + lane;
+    uint32_t mx = 0;
+#pragma unroll
+    for (int kh = 0; kh < NKH; ++kh)
+#pragma unroll
+      for (int cc = 0; cc < 8; ++cc) {
+        const uint4 u =
+            *reinterpret_cast<const uint4*>(tile + kh * kHalfTileBytes + r * 128 + ((cc ^ (r & 7)) << 4));
+        mx = __vmaxu2(mx, u.x & 0x7FFF7FFFu);
+        mx = __vmaxu2(mx, u.y & 0x7FFF7FFFu);
+        mx = __vmaxu2(mx, u.z & 0x7FFF7FFFu);
+        mx = __vmaxu2(mx, u.w & 0x7FFF7FFFu);
+      }
+    const uint32_t a16 = max(mx & 0xFFFFu, mx >> 16);
+    if (r < valid) gamma_rows[r] = __fdiv_rn(__uint_as_float(a16 << 16), qmax);
+  }
+}
 
 // One 32-column chunk of a key's logits in pass 2: sum_r 2^(D_r * c2), where
 // the accumulator D already holds logit_r - lse_r / sigma (the row offset
@@ -338,10 +370,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     }
     __syncwarp();
   } else if (warp >= kVWarp0) {
-    // Eq. 2 scales: each thread reduces 2 of the tile's 128 V rows.  The 128-byte
-    // swizzle only permutes 16-byte chunks within a row, so a row's absmax may
-    // read its 8 chunks of each K half in any order: lane l reads chunk position
-    // cc ^ (row & 7), so eight consecutive rows cover all banks at every step.
+    // Eq. 2 scales, two warps per tile
     if (with_v) {
       const int vw = warp - kVWarp0;
       // launched as a dependent of the previous layer's compaction, which may
@@ -350,28 +379,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
       for (int lt = 0; lt < nt; ++lt) {
         const int vs = lt % kVStages;
         if (!mbar_wait(&full_v[vs], (lt / kVStages) & 1, abort_flag)) break;
-        const uint8_t* tile = sV + vs * KT;
-#pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          const int r = vw * 64 + rr * 32 + lane;
-          uint32_t mx = 0;
-#pragma unroll
-          for (int kh = 0; kh < NKH; ++kh)
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              const uint4 u =
-                  *reinterpret_cast<const uint4*>(tile + kh * kHalfTileBytes + r * 128 + ((c ^ (r & 7)) << 4));
-              mx = __vmaxu2(mx, u.x & 0x7FFF7FFFu);
-              mx = __vmaxu2(mx, u.y & 0x7FFF7FFFu);
-              mx = __vmaxu2(mx, u.z & 0x7FFF7FFFu);
-              mx = __vmaxu2(mx, u.w & 0x7FFF7FFFu);
-            }
-          const uint32_t a16 = max(mx & 0xFFFFu, mx >> 16);
-          const int tok = (t0 + lt) * kKeyTile + r;
-          if (tok < n)
-            p.gamma[static_cast<size_t>(h) * p.n_total + doc_lo + tok] =
-                __fdiv_rn(__uint_as_float(a16 << 16), p.qmax);
-        }
+        const int tok0 = (t0 + lt) * kKeyTile;
+        vscale_tile<NKH>(sV + vs * KT, vw, lane, p.gamma + static_cast<size_t>(h) * p.n_total + doc_lo + tok0,
+                         n - tok0, p.qmax);
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty_v[vs]);
       }
@@ -514,20 +524,28 @@ __global__ void __launch_bounds__(kLseThreads, 1)
 // so sixteen warps drain each TMEM buffer.  A thread's partial sum for its key
 // (over its chunks of all row halves of the tile) goes to shared memory, and
 // after a named barrier warpgroup 0 adds the four partials in a fixed order.
+//
+// VS (the caller's normalisers, at most 256 guide rows): the same CTA also
+// forms the Eq. 2 scale of every token of its key range from a V ring, as in
+// pass 1, so the layer reads K and V once.  The normalisers are then inputs of
+// the call: as a programmatic dependent (the next layer of a stack) the kernel
+// waits for its predecessor only before its first store.
 // ---------------------------------------------------------------------------
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-    tp_keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmq,
-                    const __grid_constant__ KeyScoreParams p) {
+template <int D, bool VS>
+__global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
+    tp_keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                       const __grid_constant__ CUtensorMap tmq, const __grid_constant__ KeyScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = aligned_smem(smem_raw);
   constexpr int NKH = D / 64;
   constexpr uint32_t KT = NKH * kHalfTileBytes;
+  constexpr int VST = VS ? kVStages2 : 0;
   const int stages = p.stages, rows_pad = p.rows_pad, rows_mma = p.rows_mma;
   const int nh = (rows_mma + 255) / 256;
-  const ScoreSmem L = score_layout(D, rows_pad, stages, keyscore_extra_bytes(rows_pad));
+  const ScoreSmem L = score_layout(D, rows_pad, stages + VST, keyscore_extra_bytes(rows_pad));
   uint8_t* sQ = smem + L.q;
   uint8_t* sK = smem + L.k;
+  uint8_t* sV = sK + stages * KT;  // VS: the V ring after the K ring
   uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
   uint64_t* empty_k = full_k + stages;
   uint64_t* q_full = empty_k + stages;
@@ -535,6 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tempty = tfull + 2;   // [2 TMEM buffers], one arrival per epilogue warp
   uint64_t* drain = tempty + 2;
   uint64_t* pdone = drain + 1;    // [4] partial slots complete, one arrival per warp
+  uint64_t* full_v = pdone + 4;   // VS: [VST]
+  uint64_t* empty_v = full_v + VST;  // VS: [VST], one arrival per V warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
   // Row offsets as an extra K step of the contraction (32-byte swizzled,
@@ -566,10 +586,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(drain, 1);
     for (int i = 0; i < 4; ++i) mbar_init(&pdone[i], 8 * nh);
+    for (int i = 0; i < VST; ++i) {
+      mbar_init(&full_v[i], 1);
+      mbar_init(&empty_v[i], 2);
+    }
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (!p.wait_at_end) grid_dep_launch();
+  grid_dep_launch();
   if (warp == 0) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
@@ -577,12 +601,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // The guide block and the first K tiles are inputs of the whole layer: they
-  // may load while pass 1 (this kernel's predecessor) finishes.
-  const int k_pre = min(stages, nt);
+  // The guide block and the first K (and V) tiles are inputs of the whole
+  // layer: they may load while the predecessor finishes.
+  const int k_pre = min(stages, nt), v_pre = min(VST, nt);
+  auto issue_v = [&](int lt) {
+    const int vs = lt % kVStages2;
+    mbar_arrive_expect_tx(&full_v[vs], KT);
+    const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
+#pragma unroll
+    for (int kh = 0; kh < NKH; ++kh)
+      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+  };
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmk);
     prefetch_tensormap(&tmq);
+    if (VS) prefetch_tensormap(&tmv);
     load_guide<D>(sQ, &tmq, rows_pad, b * p.n_heads_kv + h, q_full);
     for (int lt = 0; lt < k_pre; ++lt) {
       mbar_arrive_expect_tx(&full_k[lt], KT);
@@ -591,8 +624,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int kh = 0; kh < NKH; ++kh)
         tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[lt]);
     }
+    for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
   }
-  if (!p.wait_at_end) grid_dep_wait();  // the row normalisers come from pass 1
+  if (!VS) grid_dep_wait();  // the row normalisers come from pass 1
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
     for (int r = threadIdx.x; r < 128 + rows_pad; r += blockDim.x) {
@@ -623,8 +657,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued = k_pre;
-      for (int lt = k_pre; lt < nt; ++lt) {
+      // K tiles as their stages free up; with VS each V tile once the V warps
+      // have released its stage (the V stream runs beside the scoring)
+      int issued = k_pre, issued_v = v_pre;
+      bool ok = true;
+      for (int lt = k_pre; ok && lt < nt; ++lt) {
         const int s = lt % stages, use = lt / stages;
         if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
         mbar_arrive_expect_tx(&full_k[s], KT);
@@ -633,14 +670,47 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kh = 0; kh < NKH; ++kh)
           tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
         issued = lt + 1;
+        if (VS) {
+          for (; issued_v <= lt && issued_v < nt; ++issued_v) {
+            const int vs = issued_v % kVStages2;
+            if (!mbar_wait(&empty_v[vs], (issued_v / kVStages2 - 1) & 1, abort_flag)) {
+              ok = false;
+              break;
+            }
+            issue_v(issued_v);
+          }
+        }
       }
-      if (*abort_flag) {
+      if (VS) {
+        for (; ok && issued_v < nt; ++issued_v) {
+          const int vs = issued_v % kVStages2;
+          if (!mbar_wait(&empty_v[vs], (issued_v / kVStages2 - 1) & 1, abort_flag)) break;
+          issue_v(issued_v);
+        }
+      }
+      if (*abort_flag) {  // let in-flight copies land before the CTA exits
         mbar_drain(q_full, 0);
         for (int lt = max(0, issued - stages); lt < issued; ++lt)
           mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
+        if (VS)
+          for (int lt = max(0, issued_v - kVStages2); lt < issued_v; ++lt)
+            mbar_drain(&full_v[lt % kVStages2], (lt / kVStages2) & 1);
       }
     }
     __syncwarp();
+  } else if (VS && warp >= kVWarp0) {
+    // Eq. 2 scales of the CTA's key range, two warps per tile
+    const int vw = warp - kVWarp0;
+    grid_dep_wait();  // the previous layer's kernels may still read the scales
+    for (int lt = 0; lt < nt; ++lt) {
+      const int vs = lt % kVStages2;
+      if (!mbar_wait(&full_v[vs], (lt / kVStages2) & 1, abort_flag)) break;
+      const int tok0 = (t0 + lt) * kKeyTile;
+      vscale_tile<NKH>(sV + vs * KT, vw, lane, p.gamma + static_cast<size_t>(h) * p.n_total + doc_lo + tok0,
+                       n - tok0, p.qmax);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_v[vs]);
+    }
   } else if (warp == 1) {
     if (lane == 0) {
       bool ok = mbar_wait(q_full, 0, abort_flag);
@@ -686,7 +756,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int e = warp - kEpiWarp0, grp = e >> 3, cg = (e >> 2) & 1, quad = warp & 3;
     const float c2 = p.c2;
     const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-    bool ok = true;
+    bool ok = true, stored = false;
     for (int lt = 0; lt < nt; ++lt) {
       float* slot = part + (lt & 3) * 4 * 128;  // partials (hh, cg) of this tile's keys
       uint64_t* done = &pdone[lt & 3];
@@ -729,6 +799,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (grp == fin && cg == 0) {
         if (ok && !mbar_wait(done, (lt >> 2) & 1, abort_flag)) ok = false;
         if (ok) {
+          if (VS && !stored) {
+            grid_dep_wait();  // the previous layer's selection may still read the key scores
+            stored = true;
+          }
           const int kl = quad * 32 + lane;
           float s4 = slot[kl] + slot[128 + kl];
           if (nh == 2) s4 = (s4 + slot[256 + kl]) + slot[384 + kl];
@@ -744,9 +818,367 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
-  // complete only after the predecessor: the kernels after this one rely on
-  // everything before it having finished
-  if (p.wait_at_end) grid_dep_wait();
+}
+
+// ---------------------------------------------------------------------------
+// Pass 2 and the Eq. 2 scales on a CTA pair (tcgen05 cta_group::2), for row
+// normalisers given by the caller: one kernel reads K and V once.
+//
+// The two CTAs of a cluster share each MMA: a pair tile is 256 keys, the even
+// CTA streaming keys 0..127 of it and the odd CTA keys 128..255 (A split along
+// M), and every job's guide rows are split in halves (B split along N).  Each
+// CTA therefore keeps only half of the guide block in shared memory, which
+// leaves room for a V ring: as in pass 1, two warps reduce each of the CTA's
+// V rows to its absmax while the scoring runs.  Each CTA's tensor memory
+// receives D[key, row] for its own 128 keys and all rows of the job, so the
+// epilogue is that of the one-CTA kernel.
+//
+// The even CTA's warp 1 issues the MMAs and multicasts every completion to
+// both CTAs (TMEM buffer full, K stage free, drain).  The odd CTA's warp 1
+// relays the arrival of each of its K stages to the even CTA, and its
+// epilogue warps release a TMEM buffer on the even CTA's barrier, so the MMA
+// thread waits for both halves of every operand and of every drained buffer.
+//
+// Launched as a programmatic dependent (the next layer of a stack after the
+// previous layer's compaction), the kernel loads and scores at once (its
+// inputs are the layer's) and waits for its predecessor only before its first
+// store of a scale or a key score.
+// ---------------------------------------------------------------------------
+
+struct PairSmem {
+  uint32_t q, k, v, bars, misc, a_aug, b_aug, part, total;
+};
+
+// Byte offsets inside the (1024-aligned) dynamic shared memory of one CTA:
+// guide half [nh jobs][D/64 halves][128 rows][128 B], the K ring, the V ring,
+// barriers, the row-offset operands (key side 128 x 32 B; guide side
+// [nh][128 rows][32 B]) and the epilogue partials [4 tiles][4][128 keys].
+__host__ __device__ inline PairSmem pair_layout(int head_dim, int nh, int stages) {
+  PairSmem L;
+  const int nkh = head_dim / 64;
+  L.q = 0;
+  L.k = static_cast<uint32_t>(nh * nkh) * kHalfTileBytes;
+  L.v = L.k + static_cast<uint32_t>(stages * nkh) * kHalfTileBytes;
+  L.bars = L.v + static_cast<uint32_t>(kVStages2 * nkh) * kHalfTileBytes;
+  L.misc = L.bars + static_cast<uint32_t>(3 * stages + 2 * kVStages2 + 16) * 8;
+  L.a_aug = (L.misc + 16 + 1023) & ~1023u;
+  L.b_aug = L.a_aug + 128u * 32u;
+  L.part = L.b_aug + static_cast<uint32_t>(nh) * 128u * 32u;
+  L.total = L.part + 4u * 4u * 128u * 4u;
+  return L;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kLseThreads, 1)
+    tp_keyscore_pair_kernel(const __grid_constant__ CUtensorMap tmk,
+                            const __grid_constant__ CUtensorMap tmv,
+                            const __grid_constant__ CUtensorMap tmq,
+                            const __grid_constant__ KeyScoreParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = aligned_smem(smem_raw);
+  constexpr int NKH = D / 64;
+  constexpr uint32_t KT = NKH * kHalfTileBytes;
+  constexpr int kPairTile = 2 * kKeyTile;
+  const int stages = p.stages, rows_mma = p.rows_mma;
+  const int nh = (rows_mma + 255) / 256;
+  const PairSmem L = pair_layout(D, nh, stages);
+  uint8_t* sQ = smem + L.q;
+  uint8_t* sK = smem + L.k;
+  uint8_t* sV = smem + L.v;
+  uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + L.bars);
+  uint64_t* empty_k = full_k + stages;  // multicast by the MMA thread's commits
+  uint64_t* pfull = empty_k + stages;   // even CTA: the odd CTA's stage has landed
+  uint64_t* full_v = pfull + stages;    // [kVStages2]
+  uint64_t* empty_v = full_v + kVStages2;  // [kVStages2], one arrival per V warp
+  uint64_t* q_full = empty_v + kVStages2;
+  uint64_t* tfull = q_full + 1;         // [2 TMEM buffers], multicast
+  uint64_t* tempty = tfull + 2;         // [2] even CTA: one arrival per epilogue warp of the pair
+  uint64_t* drain = tempty + 2;         // multicast
+  uint64_t* pdone = drain + 1;          // [4] partial slots complete, one arrival per warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L.misc + 4);
+  uint8_t* a_aug = smem + L.a_aug;
+  uint8_t* b_aug = smem + L.b_aug;
+  float* part = reinterpret_cast<float*>(smem + L.part);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0 issues the MMAs
+  const int h = blockIdx.y;
+  const int pair = static_cast<int>(blockIdx.x >> 1);
+  const int b = find_doc(p.docs, pair);
+  const int c = pair - p.docs.cta[b];
+  const int64_t doc_lo = p.docs.off[b];
+  const int n = static_cast<int>(p.docs.off[b + 1] - doc_lo);
+  const int ntiles = (n + kPairTile - 1) / kPairTile;
+  const int t0 = c * p.tiles_per_cta;
+  const int nt = min(p.tiles_per_cta, ntiles - t0);
+  const int key0 = static_cast<int>(rank) * kKeyTile;  // this CTA's half of a pair tile
+  auto tile_row = [&](int lt) {
+    return static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kPairTile + key0);
+  };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full_k[s], 1);
+      mbar_init(&empty_k[s], 1);
+      mbar_init(&pfull[s], 1);
+    }
+    for (int i = 0; i < kVStages2; ++i) {
+      mbar_init(&full_v[i], 1);
+      mbar_init(&empty_v[i], 2);
+    }
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], kEpiWarps);  // eight warps of each CTA drain a buffer
+    }
+    mbar_init(drain, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(&pdone[i], 8 * nh);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  grid_dep_launch();
+  // both CTAs are running and their barriers are initialised before the
+  // collective allocation and any remote arrival
+  cluster_sync_all();
+  if (warp == 0) {
+    tmem_alloc_pair(tmem_slot, 512);
+    tmem_relinquish_pair();
+  }
+  // This CTA's half of every job's guide rows, its first K and V tiles.
+  const int k_pre = min(stages, nt), v_pre = min(kVStages2, nt);
+  auto issue_v = [&](int lt) {
+    const int vs = lt % kVStages2;
+    mbar_arrive_expect_tx(&full_v[vs], KT);
+#pragma unroll
+    for (int kh = 0; kh < NKH; ++kh)
+      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, tile_row(lt), h, &full_v[vs]);
+  };
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmk);
+    prefetch_tensormap(&tmv);
+    prefetch_tensormap(&tmq);
+    mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(nh * NKH) * kHalfTileBytes);
+    for (int hh = 0; hh < nh; ++hh) {
+      const int half = min(256, rows_mma - 256 * hh) / 2;
+      const int r0 = 256 * hh + static_cast<int>(rank) * half;
+#pragma unroll
+      for (int kh = 0; kh < NKH; ++kh)
+        tma_load_3d(sQ + (hh * NKH + kh) * kHalfTileBytes, &tmq, kh * 64, r0, b * p.n_heads_kv + h,
+                    q_full);
+    }
+    for (int lt = 0; lt < k_pre; ++lt) {
+      mbar_arrive_expect_tx(&full_k[lt], KT);
+#pragma unroll
+      for (int kh = 0; kh < NKH; ++kh)
+        tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[lt]);
+    }
+    for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
+  }
+  {
+    // the caller's row normalisers: an input of the layer
+    const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
+    for (int r = threadIdx.x; r < 128 + nh * 128; r += blockDim.x) {
+      uint4 c0;
+      uint8_t* row;
+      int rr;
+      if (r < 128) {  // key side: three ones
+        rr = r;
+        row = a_aug + r * 32;
+        c0 = make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u);
+      } else {        // guide side: the offset of row i of this CTA's half of job hh
+        const int hh = (r - 128) >> 7, i = (r - 128) & 127;
+        const int half = min(256, rows_mma - 256 * hh) / 2;
+        const int g = 256 * hh + static_cast<int>(rank) * half + i;
+        rr = i;
+        row = b_aug + (hh * 128 + i) * 32;
+        const float v = (i < half && g < p.rows) ? -(lse[g] * 1.4426950408889634f) / p.c2 : -1.0e30f;
+        const uint32_t hi = bf16_bits_rn(v);
+        const float r1 = v - __uint_as_float(hi << 16);
+        const uint32_t mid = bf16_bits_rn(r1);
+        const uint32_t lo = bf16_bits_rn(r1 - __uint_as_float(mid << 16));
+        c0 = make_uint4(hi | (mid << 16), lo, 0u, 0u);
+      }
+      const int pos = (rr >> 2) & 1;  // 32-byte swizzle: chunk c at c ^ ((row >> 2) & 1)
+      *reinterpret_cast<uint4*>(row + pos * 16) = c0;
+      *reinterpret_cast<uint4*>(row + (pos ^ 1) * 16) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async_smem();  // read by the tensor core
+  }
+  // Before the first MMA: the odd CTA's guide half has landed and both CTAs'
+  // offset operands and tensor memory are in place.
+  if (warp == 1 && lane == 0 && rank == 1) mbar_wait(q_full, 0, abort_flag);
+  tc_fence_before();
+  cluster_sync_all();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // K tiles as their stages free up; each V tile once the V warps have
+      // released its stage (the V stream runs beside the scoring)
+      int issued = k_pre, issued_v = v_pre;
+      bool ok = true;
+      for (int lt = k_pre; ok && lt < nt; ++lt) {
+        const int s = lt % stages, use = lt / stages;
+        if (use > 0 && !mbar_wait(&empty_k[s], (use - 1) & 1, abort_flag)) break;
+        mbar_arrive_expect_tx(&full_k[s], KT);
+#pragma unroll
+        for (int kh = 0; kh < NKH; ++kh)
+          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[s]);
+        issued = lt + 1;
+        for (; issued_v <= lt && issued_v < nt; ++issued_v) {
+          const int vs = issued_v % kVStages2;
+          if (!mbar_wait(&empty_v[vs], (issued_v / kVStages2 - 1) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          issue_v(issued_v);
+        }
+      }
+      for (; ok && issued_v < nt; ++issued_v) {
+        const int vs = issued_v % kVStages2;
+        if (!mbar_wait(&empty_v[vs], (issued_v / kVStages2 - 1) & 1, abort_flag)) break;
+        issue_v(issued_v);
+      }
+      if (*abort_flag) {  // let in-flight copies land before the CTA exits
+        mbar_drain(q_full, 0);
+        for (int lt = max(0, issued - stages); lt < issued; ++lt)
+          mbar_drain(&full_k[lt % stages], (lt / stages) & 1);
+        for (int lt = max(0, issued_v - kVStages2); lt < issued_v; ++lt)
+          mbar_drain(&full_v[lt % kVStages2], (lt / kVStages2) & 1);
+      }
+    }
+    __syncwarp();
+  } else if (warp >= kVWarp0) {
+    // Eq. 2 scales of this CTA's 128 keys of each pair tile
+    const int vw = warp - kVWarp0;
+    grid_dep_wait();  // the previous layer's kernels may still read the scales
+    for (int lt = 0; lt < nt; ++lt) {
+      const int vs = lt % kVStages2;
+      if (!mbar_wait(&full_v[vs], (lt / kVStages2) & 1, abort_flag)) break;
+      const int tok0 = (t0 + lt) * kPairTile + key0;
+      vscale_tile<NKH>(sV + vs * KT, vw, lane, p.gamma + static_cast<size_t>(h) * p.n_total + doc_lo + tok0,
+                       n - tok0, p.qmax);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_v[vs]);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 1) {
+      // relay: each of this CTA's K stages has landed
+      const uint32_t pfull0 = cluster_addr(pfull, 0);
+      for (int lt = 0; lt < nt; ++lt) {
+        const int s = lt % stages;
+        if (!mbar_wait(&full_k[s], (lt / stages) & 1, abort_flag)) break;
+        mbar_arrive_cluster(pfull0 + static_cast<uint32_t>(s) * 8u);
+      }
+      mbar_drain(drain, 0);  // the pair's last MMA has completed
+    } else if (lane == 0) {
+      bool ok = mbar_wait(q_full, 0, abort_flag);
+      for (int lt = 0; ok && lt < nt; ++lt) {
+        const int s = lt % stages;
+        if (!mbar_wait(&full_k[s], (lt / stages) & 1, abort_flag)) break;
+        if (!mbar_wait_cluster(&pfull[s], (lt / stages) & 1, abort_flag)) break;
+        tc_fence_after();
+        for (int hh = 0; hh < nh; ++hh) {
+          const int j = lt * nh + hh, buf = j & 1, use = j >> 1;
+          if (use > 0 && !mbar_wait(&tempty[buf], (use - 1) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int nrows = min(256, rows_mma - 256 * hh);
+          const uint32_t idesc = idesc_bf16_f32(256, nrows);
+          const uint32_t dt = tmem + static_cast<uint32_t>(buf * 256);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const int kh = kk >> 2, k16 = kk & 3;
+            const uint64_t a = sdesc_k128(smem_u32(sK + s * KT + kh * kHalfTileBytes + k16 * 32));
+            const uint64_t bd = sdesc_k128(smem_u32(sQ + (hh * NKH + kh) * kHalfTileBytes + k16 * 32));
+            mma_bf16_ss_pair(dt, a, bd, idesc, kk > 0 ? 1u : 0u);
+          }
+          mma_bf16_ss_pair(dt, sdesc_k32(smem_u32(a_aug)), sdesc_k32(smem_u32(b_aug + hh * 128 * 32)),
+                           idesc, 1u);
+          mma_commit_pair(&tfull[buf]);
+        }
+        mma_commit_pair(&empty_k[s]);
+      }
+      mma_commit_pair(drain);
+      mbar_drain(drain, 0);
+    }
+    __syncwarp();
+  } else {
+    // The epilogue of the one-CTA kernel on this CTA's 128 keys; a drained
+    // buffer is released on the even CTA's barrier (a CTA-scope arrival: it
+    // reports completed tensor-memory loads, not data).
+    const int e = warp - kEpiWarp0, grp = e >> 3, cg = (e >> 2) & 1, quad = warp & 3;
+    const float c2 = p.c2;
+    const uint32_t tlane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const uint32_t tempty0 = cluster_addr(tempty, 0);
+    bool ok = true, stored = false;
+    for (int lt = 0; lt < nt; ++lt) {
+      float* slot = part + (lt & 3) * 4 * 128;
+      uint64_t* done = &pdone[lt & 3];
+      for (int hh = 0; hh < nh; ++hh) {
+        const int j = lt * nh + hh, buf = j & 1;
+        if (buf != grp) continue;
+        if (ok && !mbar_wait(&tfull[buf], (j >> 1) & 1, abort_flag)) ok = false;
+        if (!ok) continue;
+        tc_fence_after();
+        const int nch = min(256, rows_mma - 256 * hh) / 32;
+        const uint32_t tb = tlane + buf * 256;
+        const int ch = 4 * cg;
+        float acc = 0.f;
+        uint32_t ra[32], rb[32];
+        if (ch < nch) tmem_ld32_async(tb + ch * 32, ra);
+        if (ch + 1 < nch) tmem_ld32_async(tb + (ch + 1) * 32, rb);
+        if (ch < nch) tmem_wait(ra);
+        if (ch + 1 < nch) tmem_wait(rb);
+        if (ch < nch) acc += key_chunk(ra, c2);
+        if (ch + 2 < nch) tmem_ld32_async(tb + (ch + 2) * 32, ra);
+        if (ch + 1 < nch) acc += key_chunk(rb, c2);
+        if (ch + 3 < nch) tmem_ld32_async(tb + (ch + 3) * 32, rb);
+        if (ch + 2 < nch) tmem_wait(ra);
+        if (ch + 3 < nch) tmem_wait(rb);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 0) mbar_arrive(&tempty[buf]);
+          else mbar_arrive_remote(tempty0 + static_cast<uint32_t>(buf) * 8u);
+        }
+        if (ch + 2 < nch) acc += key_chunk(ra, c2);
+        if (ch + 3 < nch) acc += key_chunk(rb, c2);
+        slot[(hh * 2 + cg) * 128 + quad * 32 + lane] = acc;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(done);
+      }
+      const int fin = (lt * nh + nh - 1) & 1;
+      if (grp == fin && cg == 0) {
+        if (ok && !mbar_wait(done, (lt >> 2) & 1, abort_flag)) ok = false;
+        if (ok) {
+          if (!stored) {
+            grid_dep_wait();  // the previous layer's selection may still read the key scores
+            stored = true;
+          }
+          const int kl = quad * 32 + lane;
+          float s4 = slot[kl] + slot[128 + kl];
+          if (nh == 2) s4 = (s4 + slot[256 + kl]) + slot[384 + kl];
+          const int key = (t0 + lt) * kPairTile + key0 + kl;
+          if (key < n) p.skey[static_cast<size_t>(h) * p.n_total + doc_lo + key] = s4 * p.inv_group;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (*abort_flag != 0 && threadIdx.x == 0) set_status(p.status, TP_ERR_TIMEOUT);
+  // neither CTA releases its tensor memory or leaves while the pair's MMAs or
+  // the other CTA's remote arrivals may still touch it
+  tc_fence_before();
+  cluster_sync_all();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, 512);
+  }
 }
 
 }  // namespace
@@ -756,8 +1188,13 @@ size_t lse_smem_bytes(int head_dim, int rows_pad, int stages) {
   return score_layout(head_dim, 0, stages + kVStages, 0).total + 1024;
 }
 
-size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages) {
-  return score_layout(head_dim, rows_pad, stages, keyscore_extra_bytes(rows_pad)).total + 1024;
+size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages, bool scales) {
+  return score_layout(head_dim, rows_pad, stages + (scales ? kVStages2 : 0),
+                      keyscore_extra_bytes(rows_pad)).total + 1024;
+}
+
+size_t keyscore_pair_smem_bytes(int head_dim, int rows_mma, int stages) {
+  return pair_layout(head_dim, (rows_mma + 255) / 256, stages).total + 1024;
 }
 
 template <int D, int NRB>
@@ -792,16 +1229,17 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUt
   return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
-cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
-                            const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
-                            bool dependent, cudaStream_t s) {
-  const void* fn = head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_kernel<128>)
-                                   : reinterpret_cast<const void*>(tp_keyscore_kernel<64>);
-  cudaError_t e = set_smem_once(fn, head_dim == 128 ? 8 : 9);
+template <int D, bool VS>
+cudaError_t launch_keyscore_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                              const KeyScoreParams& p, dim3 grid, size_t smem, bool dependent,
+                              cudaStream_t s) {
+  // shared-memory attribute slots 8, 9 (plain) and 19, 20 (with the scales)
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<D, VS>),
+                                (VS ? 19 : 8) + (D == 128 ? 0 : 1));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(VS ? kLseThreads : kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -809,8 +1247,81 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 1 : 0;
-  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<128>, tmk, tmq, p)
-                         : cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<64>, tmk, tmq, p);
+  return cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<D, VS>, tmk, tmv, tmq, p);
+}
+
+cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                            const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
+                            bool dependent, cudaStream_t s) {
+  if (p.gamma)
+    return head_dim == 128 ? launch_keyscore_t<128, true>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                           : launch_keyscore_t<64, true>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  return head_dim == 128 ? launch_keyscore_t<128, false>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                         : launch_keyscore_t<64, false>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+}
+
+namespace {
+
+const void* keyscore_pair_fn(int head_dim) {
+  return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128>)
+                         : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64>);
+}
+
+cudaLaunchConfig_t pair_config(dim3 grid, size_t smem, cudaStream_t s, cudaLaunchAttribute (&attr)[2],
+                               bool dependent) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kLseThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = dependent ? 2 : 1;
+  return cfg;
+}
+
+}  // namespace
+
+int keyscore_pair_max_clusters(int head_dim, size_t smem) {
+  constexpr int kDevs = 64, kEntries = 8;
+  struct Entry {
+    int d;
+    size_t smem;
+    int clusters;
+  };
+  static std::mutex mu;
+  static Entry cache[kDevs][kEntries];
+  static int used[kDevs];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used[dev]; ++i)
+    if (cache[dev][i].d == head_dim && cache[dev][i].smem == smem) return cache[dev][i].clusters;
+  if (set_smem_once(keyscore_pair_fn(head_dim), head_dim == 128 ? 10 : 11) != cudaSuccess) return 0;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = pair_config(dim3(2, 1), smem, 0, attr, false);
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, keyscore_pair_fn(head_dim), &cfg) != cudaSuccess)
+    clusters = 0;
+  cudaGetLastError();  // a refused query leaves no error behind
+  if (used[dev] < kEntries) cache[dev][used[dev]++] = Entry{head_dim, smem, clusters};
+  return clusters;
+}
+
+cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
+                                 const CUtensorMap& tmq, const KeyScoreParams& p, int head_dim,
+                                 dim3 grid, size_t smem, bool dependent, cudaStream_t s) {
+  cudaError_t e = set_smem_once(keyscore_pair_fn(head_dim), head_dim == 128 ? 10 : 11);
+  if (e != cudaSuccess) return e;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = pair_config(grid, smem, s, attr, dependent);
+  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128>, tmk, tmv, tmq, p)
+                         : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64>, tmk, tmv, tmq, p);
 }
 
 }  // namespace tp

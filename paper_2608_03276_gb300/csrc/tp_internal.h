@@ -52,23 +52,21 @@ struct LseParams {
 
 // Pass 2: per-key sum over all guide rows of exp(logit - lse).
 struct KeyScoreParams {
-  DocTable docs;
+  DocTable docs;     // CTA prefix per document (pair prefix for the pair kernel)
   int n_heads_kv;
   int rows;
   int rows_pad;
   int rows_mma;      // rows rounded up to 32 (the MMA N extent, split in 256s)
-  int tiles_per_cta;
+  int tiles_per_cta; // 128-key tiles per CTA (256-key pair tiles per pair)
   int stages;
   float c2;
   float inv_group;
   int64_t n_total;
   const float* lse;  // [batch, H_kv, rows] natural log
   float* skey;       // [H_kv, N]
+  float* gamma;      // Eq. 2 scales [H_kv, N] written alongside, or null
+  float qmax;
   int* status;
-  // The normalisers are inputs of the call, not the previous kernel's output:
-  // no wait before reading them; the kernel waits for its predecessor at its
-  // end instead, and its dependents start only when it exits.
-  int wait_at_end;
 };
 
 constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
@@ -137,24 +135,33 @@ struct PrefixParams {
 // Launchers (return cudaError_t of the launch).
 cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int bits, int num_sms, cudaStream_t s);
-// The quantiser as a programmatic dependent of the previous kernel, which it
-// lets its own dependents overlap: it starts at once (its input is the
-// layer's V, written before the call) and waits for the previous kernel only
-// at its end.
-cudaError_t launch_vquant_dependent(const uint16_t* v, float* gamma, int64_t rows, int head_dim,
-                                    float qmax, int num_sms, cudaStream_t s);
 // Pass 1.  `dependent`: launched as a programmatic dependent of the previous
 // layer's last kernel (a stack of layers in one call); it then waits for that
 // kernel before its first store.
 cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                        const LseParams& p, int head_dim, dim3 grid, size_t smem, bool dependent,
                        cudaStream_t s);
-// `dependent`: launch as a programmatic dependent of the previous kernel in
-// the stream (only where that kernel and this one belong to one layer's
-// sequence, whose inputs were written before its first kernel started).
-cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmq,
+// Pass 2, one CTA per key range.  `dependent`: launch as a programmatic
+// dependent of the previous kernel in the stream (only where that kernel and
+// this one belong to one layer's sequence, whose inputs were written before
+// its first kernel started); it waits for it before reading the normalisers.
+// With p.gamma set (the caller's normalisers, at most 256 guide rows) it also
+// forms the Eq. 2 scales from V (map tmv) and waits only before its first
+// store.
+cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             bool dependent, cudaStream_t s);
+// Pass 2 with the caller's normalisers and the Eq. 2 scales (p.gamma) in one
+// kernel on CTA pairs (two-CTA clusters sharing each MMA); grid.x is twice the
+// number of pairs.  The guide map has 128-row boxes (each CTA loads half of
+// every job's rows).  `dependent`: it waits for the previous kernel only
+// before its first store.
+cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
+                                 const CUtensorMap& tmq, const KeyScoreParams& p, int head_dim,
+                                 dim3 grid, size_t smem, bool dependent, cudaStream_t s);
+// How many CTA pairs of the pair kernel can be resident at once (0 when the
+// device or the query refuses a two-CTA cluster of that size).
+int keyscore_pair_max_clusters(int head_dim, size_t smem);
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
@@ -166,6 +173,7 @@ cudaError_t set_smem_once(const void* kernel, int slot);
 
 // Shared-memory layout sizes of the scoring kernels (host side).
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages);
-size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages);
+size_t keyscore_smem_bytes(int head_dim, int rows_pad, int stages, bool scales);
+size_t keyscore_pair_smem_bytes(int head_dim, int rows_mma, int stages);
 
 }  // namespace tp

@@ -18,17 +18,13 @@ namespace {
 
 // One row = LPR lanes x 8 bf16.  Rows are processed UNROLL at a time per
 // lane group so that several 16-byte loads are in flight per thread.
-// With `chained` set the kernel runs as a programmatic dependent: it lets
-// its own dependent be scheduled at once, and waits for its predecessor only
-// after its last store (so its completion implies the predecessor's).
 template <int LPR, int UNROLL>
 __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict__ v,
                                                       void* __restrict__ vq,
                                                       float* __restrict__ gamma, int64_t rows,
-                                                      float qmax, int bits, int chained) {
+                                                      float qmax, int bits) {
   constexpr int RPW = 32 / LPR;  // rows per warp instruction
   const int lane = threadIdx.x & 31;
-  if (chained) grid_dep_launch();
   const int sub = lane / LPR, part = lane % LPR;
   const int64_t warps_total = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
   const int64_t gw = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -61,7 +57,6 @@ __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict_
       }
     }
   }
-  if (chained) grid_dep_wait();
 }
 
 // Compaction: a group of LPR lanes moves one (document, head, slot): lane
@@ -134,38 +129,10 @@ cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t row
   if (blocks > cap) blocks = cap;
   const uint4* vv = reinterpret_cast<const uint4*>(v);
   if (head_dim == 128)
-    tp_vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits, 0);
+    tp_vquant_kernel<16, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits);
   else
-    tp_vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits, 0);
+    tp_vquant_kernel<8, kUnroll><<<static_cast<unsigned>(blocks), threads, 0, s>>>(vv, vq, gamma, rows, qmax, bits);
   return cudaGetLastError();
-}
-
-cudaError_t launch_vquant_dependent(const uint16_t* v, float* gamma, int64_t rows, int head_dim,
-                                    float qmax, int num_sms, cudaStream_t s) {
-  if (rows <= 0) return cudaSuccess;
-  constexpr int kUnroll = 4;
-  const int threads = 256;
-  const int lpr = head_dim / 8;
-  const int64_t rows_per_block = static_cast<int64_t>(threads / 32) * (32 / lpr) * kUnroll;
-  int64_t blocks = (rows + rows_per_block - 1) / rows_per_block;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
-  if (blocks > cap) blocks = cap;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(blocks));
-  cfg.blockDim = dim3(threads);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  const uint4* vv = reinterpret_cast<const uint4*>(v);
-  void* vq = nullptr;
-  const float q = qmax;
-  const int bits = 8, chained = 1;
-  return head_dim == 128
-             ? cudaLaunchKernelEx(&cfg, tp_vquant_kernel<16, kUnroll>, vv, vq, gamma, rows, q, bits, chained)
-             : cudaLaunchKernelEx(&cfg, tp_vquant_kernel<8, kUnroll>, vv, vq, gamma, rows, q, bits, chained);
 }
 
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s) {

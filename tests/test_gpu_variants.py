@@ -471,3 +471,28 @@ def test_full_size_variants(cuda_lib, variant):
                                          k_guide_bits=kg)
     assert binding.tp_check_status(out.ws) == 0
     _check_layer(w, x, out, ref)
+
+
+# With the caller's normalisers, more than 256 guide rows take the key scores
+# and the V scales from one kernel on CTA pairs (256-key pair tiles, so a
+# document's last pair tile may be half or wholly past its end), and fall back
+# to the quantiser and pass 2 when the pairs would not all be resident at once
+# (here 10 documents x 8 KV heads > 76 pairs).
+PAIR_WORKLOADS = {
+    "pair-ragged-m512": synth.small_variant(synth.WORKLOADS[3], [1000, 300, 5000]),
+    "fallback-m512-80-units": synth.small_variant(synth.WORKLOADS[3], [200] * 10),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PAIR_WORKLOADS))
+def test_caller_lse_pairs_and_fallback(cuda_lib, name):
+    from paper_2608_03276_gb300 import binding
+    w = PAIR_WORKLOADS[name]
+    x = synth.make_layer(w)
+    p = _problem(binding, w, x.doc_offsets)
+    kernels = binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget, binding.MODE_CALLER_LSE)
+    assert kernels == (4 if name.startswith("fallback") else 3), kernels
+    lse = _context_lse(w, x)
+    out = _run_lse(binding, w, x, lse)
+    ref = _oracle(w, x, lse=lse.astype(np.float64))
+    _check_layer(w, x, out, ref)
