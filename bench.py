@@ -345,16 +345,18 @@ def hbm_fused_of(w, kept_tokens, t_layer_s, hbm_peak, peak_src):
 def staged_times(binding, torch, p, w, layers, outs, ws, stream, reps, keep_ratio=None):
     """Per-kernel CUDA-event times, one entry point at a time on the launching
     stream: pass 1 with the Eq. 2 scales (tp_guide_lse), pass 2 (tp_guide_key_scores),
-    the selection (tp_select) and the compaction (tp_compact) as standalone kernels."""
+    pass 2 forming the Eq. 2 scales as well (tp_guide_key_scores with V: the scoring
+    kernel of the caller-normaliser path), the selection (tp_select) and the
+    compaction (tp_compact) as standalone kernels."""
     dev = outs[0].idx.device
     r = w.keep_ratio if keep_ratio is None else keep_ratio
     lse = torch.empty((w.batch, w.n_heads_kv, w.rows), dtype=torch.float32, device=dev)
     skey = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
     gamma = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
     scores = torch.empty((w.n_heads_kv, w.n_total), dtype=torch.float32, device=dev)
-    names = ["lse+vscale", "keyscore", "select", "gather"]
+    names = ["lse+vscale", "keyscore", "keyscore+vscale", "select", "gather"]
     acc = {s: 0.0 for s in names}
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
     nl = min(len(layers), 8)
     for _ in range(max(1, reps)):
         for li in range(nl):
@@ -365,10 +367,12 @@ def staged_times(binding, torch, p, w, layers, outs, ws, stream, reps, keep_rati
             evs[1].record(stream)
             binding.tp_guide_key_scores(p, q, k, lse, skey, stream)
             evs[2].record(stream)
-            binding.tp_select(p, scores, r, w.budget, o.idx, ws, stream)
+            binding.tp_guide_key_scores(p, q, k, lse, skey, stream, v=v, gamma=gamma)
             evs[3].record(stream)
-            binding.tp_compact(p, k, v, gamma, o.idx, r, w.budget, o.kc, o.vc, o.vqc, o.gammac, stream)
+            binding.tp_select(p, scores, r, w.budget, o.idx, ws, stream)
             evs[4].record(stream)
+            binding.tp_compact(p, k, v, gamma, o.idx, r, w.budget, o.kc, o.vc, o.vqc, o.gammac, stream)
+            evs[5].record(stream)
             torch.cuda.synchronize()
             for i, name in enumerate(names):
                 acc[name] += evs[i].elapsed_time(evs[i + 1])
@@ -630,6 +634,13 @@ def run_ours(args, w):
                           "hbm_frac": 4 * d * w.n_total * w.n_heads_kv / (stage_ms["lse+vscale"] / 1e3) / 1e9 / hbm_peak},
         "tp_keyscore_kernel": {"ms": stage_ms["keyscore"], "bound": "tensor",
                                "frac": flops1 / (stage_ms["keyscore"] / 1e3) / 1e12 / tf_burst},
+        "keyscore_with_scales": {
+            "ms": stage_ms["keyscore+vscale"], "bound": "tensor",
+            "kernel": "tp_keyscore_pair_kernel" if w.rows > 256 else "tp_keyscore_kernel with V",
+            "frac": flops1 / (stage_ms["keyscore+vscale"] / 1e3) / 1e12 / tf_burst,
+            "hbm_frac": 4 * d * w.n_total * w.n_heads_kv / (stage_ms["keyscore+vscale"] / 1e3) / 1e9 / hbm_peak,
+            "note": "the scoring kernel of the caller-normaliser path: one QK^T, the Eq. 2 scales, "
+                    "K and V read once"},
         "tp_select_kernel": {"ms": stage_ms["select"], "bound": "latency"},
         "tp_gather_kernel": {"ms": stage_ms["gather"], "bound": "hbm", "bytes_touched": gather_bytes,
                              "touched_frac": gather_bytes / (stage_ms["gather"] / 1e3) / 1e9 / hbm_peak,
@@ -637,6 +648,7 @@ def run_ours(args, w):
                                      "part of the writes is absorbed by L2 and reaches DRAM after the "
                                      "kernel, so this is a throughput of bytes touched, not DRAM bandwidth"},
     }
+    lse_given["scoring_kernel"] = kernels["keyscore_with_scales"]
     fused_tail_ms = ms / L - stage_ms["lse+vscale"] - stage_ms["keyscore"]
     hbm_fused = hbm_fused_of(w, kept_tokens, t_layer_s, hbm_peak, peak_src)
 

@@ -210,9 +210,14 @@ int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const
  * unpooled key score of every context token,
  *   key_scores[h, off_b + i] = (1/G) sum_r exp(sigma * q_r . k_i - lse[b, h, r]).
  * Needs no workspace.  key_scores: [H_kv, N] fp32 out.
+ * With v ([H_kv, N, d] bf16) and gamma ([H_kv, N] fp32 out) both non-NULL, the
+ * same kernel also writes the Eq. 2 scales of every token (as tp_quantize_v),
+ * reading V alongside K (one CTA per key range up to 256 guide rows, two-CTA
+ * clusters above; a separate V pass where those pairs would not all be
+ * resident at once); both NULL skips that.
  */
-int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
-                        float* key_scores, void* stream);
+int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const void* v,
+                        const float* lse, float* key_scores, float* gamma, void* stream);
 
 /*
  * Top-budget selection per (document, KV head) (Sec. 3.4; Sec. 4 uniform

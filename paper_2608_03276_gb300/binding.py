@@ -89,7 +89,7 @@ def load(path: Optional[str] = None):
                                         c_void_p, c_void_p]
     lib.tp_guide_key_scores.restype = c_int
     lib.tp_guide_key_scores.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p,
-                                        c_void_p]
+                                        c_void_p, c_void_p, c_void_p]
     lib.tp_select.restype = c_int
     lib.tp_select.argtypes = [POINTER(TpProblem), c_void_p, c_double, c_int64, c_void_p, c_void_p,
                               c_size_t, c_void_p]
@@ -272,15 +272,17 @@ def tp_guide_lse_static(p: Problem, q, k, lse, stream=None, v=None, gamma=None):
         _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True), _stream(stream)))
 
 
-def tp_guide_key_scores(p: Problem, q, k, lse, key_scores, stream=None):
+def tp_guide_key_scores(p: Problem, q, k, lse, key_scores, stream=None, v=None, gamma=None):
     import torch
     hq, hkv, d, lt, n = p.c.n_heads_q, p.c.n_heads_kv, p.c.head_dim, p.c.guide_len, p.n_total
     rows = (hq // hkv) * lt
     _check("tp_guide_key_scores", load().tp_guide_key_scores(
         p.ref(), _ptr(q, torch.bfloat16, p.batch * hq * lt * d, "q"),
         _ptr(k, torch.bfloat16, hkv * n * d, "k"),
+        _ptr(v, torch.bfloat16, hkv * n * d, "v", nullable=True),
         _ptr(lse, torch.float32, p.batch * hkv * rows, "lse"),
-        _ptr(key_scores, torch.float32, hkv * n, "key_scores"), _stream(stream)))
+        _ptr(key_scores, torch.float32, hkv * n, "key_scores"),
+        _ptr(gamma, torch.float32, hkv * n, "gamma", nullable=True), _stream(stream)))
 
 
 def tp_guide_prefix_lse(p: Problem, q, k_guide, lse, stream=None):

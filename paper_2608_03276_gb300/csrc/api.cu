@@ -730,17 +730,25 @@ int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const
   return run_lse(P, tmk, tmq, q, v, gamma, lse, w, s);
 }
 
-int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const float* lse,
-                        float* key_scores, void* stream) {
+int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const void* v,
+                        const float* lse, float* key_scores, float* gamma, void* stream) {
   Plan P;
   int st = make_plan(p, 0.0, 0, false, &P);
   if (st != TP_OK) return st;
   if (!q || !k || !lse || !key_scores || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
+  if ((v == nullptr) != (gamma == nullptr) || (v && !aligned16(v))) return TP_ERR_INVALID_ARG;
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (v) {
+    st = run_keyscore_scales(P, q, k, v, lse, key_scores, gamma, nullptr, false, s);
+    if (st != kNoFusedScales) return st;
+    if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, gamma, int64_t(P.hkv) * P.n_total,
+                      P.d, P.qmax, P.bits, num_sms(), s) != cudaSuccess)
+      return TP_ERR_CUDA;
+  }
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_keyscore(P, tmk, q, lse, key_scores, nullptr, false,
-                      static_cast<cudaStream_t>(stream));
+  return run_keyscore(P, tmk, q, lse, key_scores, nullptr, false, s);
 }
 
 int tp_select(const tp_problem* p, const float* scores, double keep_ratio, int64_t budget,

@@ -142,7 +142,7 @@ def test_guide_scores_entry_point(cuda_lib, name):
                 parity.assert_scores_close(sc[h, lo:hi], want, f"key_only={key_only} {b},{h}")
 
 
-@pytest.mark.parametrize("name", ["c3-guide128-2053", "c5-ragged", "c4-gqa7-3001"])
+@pytest.mark.parametrize("name", ["c3-guide128-2053", "c5-ragged", "c4-gqa7-3001", "c1-tiny-2k"])
 def test_stage_entry_points(cuda_lib, name):
     """tp_guide_lse against the oracle's row normalisers; tp_guide_key_scores fed the
     oracle's normalisers against the oracle's unpooled key scores."""
@@ -181,6 +181,15 @@ def test_stage_entry_points(cuda_lib, name):
     skey = torch.empty((w.n_heads_kv, p.n_total), dtype=torch.float32, device="cuda")
     binding.tp_guide_key_scores(p, q, k, torch.tensor(ref_lse, device="cuda"), skey)
     parity.assert_scores_close(skey.cpu().numpy(), ref_key, "key scores from given lse")
+    # the same pass forming the Eq. 2 scales too (one CTA per key range up to 256
+    # guide rows, CTA pairs above): every scale written, bit-exact, and the key
+    # scores unchanged bit for bit
+    skey2 = torch.empty_like(skey)
+    gam2 = torch.full_like(gam, float("nan"))
+    binding.tp_guide_key_scores(p, q, k, torch.tensor(ref_lse, device="cuda"), skey2,
+                                v=parity.to_device_bf16(x.v), gamma=gam2)
+    assert np.array_equal(gam2.cpu().numpy().view(np.uint32), rg.view(np.uint32)), "gamma of pass 2"
+    assert torch.equal(skey, skey2), "key scores differ with and without the fused V scales"
 
 
 def test_key_only_layer(cuda_lib):
