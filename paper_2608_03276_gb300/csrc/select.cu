@@ -346,20 +346,41 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
         else if (key == thr) ++eq;
       }
     }
-    gt = block_sum(gt, sm.scratch);
-    eq = block_sum(eq, sm.scratch);
+    if (s1 - s0 < 32768) {  // one block sum of (> T) << 16 | (== T), no overflow
+      const int both = block_sum((gt << 16) | eq, sm.scratch);
+      gt = both >> 16;
+      eq = both & 0xFFFF;
+    } else {
+      gt = block_sum(gt, sm.scratch);
+      eq = block_sum(eq, sm.scratch);
+    }
     if (threadIdx.x == 0) {
       sm.counts[0] = gt;
       sm.counts[1] = eq;
     }
   }
   cluster.sync();
-  int gt_before = 0, eq_before = 0;
-  for (int r = 0; r < rank; ++r) {
-    const int* c = cluster.map_shared_rank(sm.counts, r);
-    gt_before += c[0];
-    eq_before += c[1];
+  // counts of the slices before this one: lane r < rank reads CTA r's (one
+  // round trip), a warp sum, shared with the block
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    int g = 0, e = 0;
+    if (lane < rank) {
+      g = ld_dsmem(dsmem(&sm.counts[0], lane));
+      e = ld_dsmem(dsmem(&sm.counts[1], lane));
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      g += __shfl_xor_sync(0xffffffffu, g, o);
+      e += __shfl_xor_sync(0xffffffffu, e, o);
+    }
+    if (lane == 0) {
+      sm.result[0] = g;
+      sm.result[1] = e;
+    }
   }
+  __syncthreads();
+  int gt_before = sm.result[0], eq_before = sm.result[1];
   cluster.sync();  // no CTA leaves while another may still read its counts
 
   if (kk <= 0) return;
