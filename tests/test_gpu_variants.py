@@ -194,11 +194,12 @@ def test_int4_fused_layer(cuda_lib, name):
     assert out.vqc.dtype.itemsize == 1 and out.vqc.shape[-1] == w.head_dim // 2
 
 
-def test_int4_caller_lse_layer(cuda_lib):
-    """b = 4 through tp_compress_layer_lse, whose scales come from the
-    standalone quantiser kernel."""
+@pytest.mark.parametrize("name", ["c4-gqa7-3001", "c3-guide128-2053"])
+def test_int4_caller_lse_layer(cuda_lib, name):
+    """b = 4 through tp_compress_layer_lse, whose scales come from the key-score
+    kernel's V warps: one CTA per key range at 224 guide rows, CTA pairs at 512."""
     from paper_2608_03276_gb300 import binding
-    w = SMALL["c4-gqa7-3001"]
+    w = SMALL[name]
     x = synth.make_layer(w)
     lse = _context_lse(w, x)
     import torch
@@ -261,11 +262,12 @@ def test_layer_stack_matches_single_layers(cuda_lib, name, bits):
 
 
 @pytest.mark.parametrize("name,bits,nl", [("c2-llama-4133", 8, 4), ("c5-ragged", 8, 3),
-                                          ("c1-tiny-2k", 4, 3)])
+                                          ("c1-tiny-2k", 4, 3), ("c3-guide128-2053", 8, 3)])
 def test_lse_stack_matches_single_layers(cuda_lib, name, bits, nl):
-    """tp_compress_layers_lse (each layer's scale pass running beside the
-    previous layer's selection, two alternating scale and key-score buffers)
-    equals one tp_compress_layer_lse call per layer bit for bit, and the
+    """tp_compress_layers_lse (each layer's scoring kernel loading and scoring
+    while the previous layer's compaction finishes, then waiting for it before
+    its first store; one scale and one key-score buffer; CTA pairs at 512 guide
+    rows) equals one tp_compress_layer_lse call per layer bit for bit, and the
     oracle given the same normalisers on every layer.  The normalisers carry
     extra per-row mass, as a prefill's would."""
     import torch
