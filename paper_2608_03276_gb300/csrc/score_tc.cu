@@ -248,6 +248,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   float2* stats = reinterpret_cast<float2*>(sK);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t kv_policy = l2_evict_first_policy();  // K and V are read once
   const int h = blockIdx.y;
   const int b = find_doc(p.docs, blockIdx.x);
   const int c = blockIdx.x - p.docs.cta[b];
@@ -300,7 +301,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
 #pragma unroll
     for (int kh = 0; kh < NKH; ++kh)
-      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+      tma_load_3d_hint(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs], kv_policy);
   };
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmq);
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
 #pragma unroll
         for (int kh = 0; kh < NKH; ++kh)
-          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
+          tma_load_3d_hint(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s], kv_policy);
         issued = lt + 1;
         if (lt >= v_pre && with_v) {
           if (!mbar_wait(&empty_v[lt % kVStages], (lt / kVStages - 1) & 1, abort_flag)) break;
@@ -565,6 +566,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
   float* part = reinterpret_cast<float*>(b_aug + rows_pad * 32);      // [4][4][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t kv_policy = l2_evict_first_policy();  // K and V are read once
   const int h = blockIdx.y;
   const int b = find_doc(p.docs, blockIdx.x);
   const int c = blockIdx.x - p.docs.cta[b];
@@ -610,7 +612,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
     const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
 #pragma unroll
     for (int kh = 0; kh < NKH; ++kh)
-      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs]);
+      tma_load_3d_hint(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, y, h, &full_v[vs], kv_policy);
   };
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmk);
@@ -622,7 +624,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
       const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
 #pragma unroll
       for (int kh = 0; kh < NKH; ++kh)
-        tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[lt]);
+        tma_load_3d_hint(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[lt], kv_policy);
     }
     for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
   }
@@ -668,7 +670,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
         const int y = static_cast<int>(doc_lo + static_cast<int64_t>(t0 + lt) * kKeyTile);
 #pragma unroll
         for (int kh = 0; kh < NKH; ++kh)
-          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s]);
+          tma_load_3d_hint(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, y, h, &full_k[s], kv_policy);
         issued = lt + 1;
         if (VS) {
           for (; issued_v <= lt && issued_v < nt; ++issued_v) {
@@ -902,6 +904,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   float* part = reinterpret_cast<float*>(smem + L.part);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t kv_policy = l2_evict_first_policy();  // K and V are read once
   const uint32_t rank = cluster_ctarank();  // 0 issues the MMAs
   const int h = blockIdx.y;
   const int pair = static_cast<int>(blockIdx.x >> 1);
@@ -952,7 +955,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     mbar_arrive_expect_tx(&full_v[vs], KT);
 #pragma unroll
     for (int kh = 0; kh < NKH; ++kh)
-      tma_load_3d(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, tile_row(lt), h, &full_v[vs]);
+      tma_load_3d_hint(sV + vs * KT + kh * kHalfTileBytes, &tmv, kh * 64, tile_row(lt), h, &full_v[vs], kv_policy);
   };
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmk);
@@ -971,7 +974,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
       mbar_arrive_expect_tx(&full_k[lt], KT);
 #pragma unroll
       for (int kh = 0; kh < NKH; ++kh)
-        tma_load_3d(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[lt]);
+        tma_load_3d_hint(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[lt], kv_policy);
     }
     for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
   }
@@ -1025,7 +1028,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         mbar_arrive_expect_tx(&full_k[s], KT);
 #pragma unroll
         for (int kh = 0; kh < NKH; ++kh)
-          tma_load_3d(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[s]);
+          tma_load_3d_hint(sK + s * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[s], kv_policy);
         issued = lt + 1;
         for (; issued_v <= lt && issued_v < nt; ++issued_v) {
           const int vs = issued_v % kVStages2;
