@@ -63,7 +63,9 @@ __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict_
 // `part` copies the 16-byte part `part` of both the K and the V row and forms
 // the int8 codes of its 8 V values, so every lane runs the same code.  Each
 // lane keeps kUnroll slots in flight; idx < 0 marks an unused slot
-// (zero-filled).
+// (zero-filled).  The cache is written with streaming stores (evict-first in
+// L2): nothing here reads it again, and the next layer's scales and key scores
+// should find L2 room for the selection.
 template <int LPR>
 __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ GatherParams p) {
   constexpr int SPW = 32 / LPR;  // slots per warp instruction
@@ -103,15 +105,15 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
     if (j[u] == -2) continue;
     const int64_t slot = unit * p.cap + t0 + u * SPW;
     const int64_t dst = slot * LPR + part;
-    if (p.kc) reinterpret_cast<uint4*>(p.kc)[dst] = kv[u];
-    if (p.vc) reinterpret_cast<uint4*>(p.vc)[dst] = vv[u];
+    if (p.kc) __stcs(reinterpret_cast<uint4*>(p.kc) + dst, kv[u]);
+    if (p.vc) __stcs(reinterpret_cast<uint4*>(p.vc) + dst, vv[u]);
     if (p.vqc) {
       if (p.bits == 8)
-        reinterpret_cast<uint2*>(p.vqc)[dst] = j[u] >= 0 ? quant8_packed(vv[u], g[u], p.qmax) : make_uint2(0, 0);
+        __stcs(reinterpret_cast<uint2*>(p.vqc) + dst, j[u] >= 0 ? quant8_packed(vv[u], g[u], p.qmax) : make_uint2(0, 0));
       else
-        reinterpret_cast<uint32_t*>(p.vqc)[dst] = j[u] >= 0 ? quant4_packed(vv[u], g[u], p.qmax) : 0u;
+        __stcs(reinterpret_cast<unsigned int*>(p.vqc) + dst, j[u] >= 0 ? quant4_packed(vv[u], g[u], p.qmax) : 0u);
     }
-    if (p.gammac && part == 0) p.gammac[slot] = g[u];
+    if (p.gammac && part == 0) __stcs(p.gammac + slot, g[u]);
   }
 }
 
