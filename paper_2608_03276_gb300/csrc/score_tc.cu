@@ -595,16 +595,9 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  grid_dep_launch();
-  if (warp == 0) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
   // The guide block and the first K (and V) tiles are inputs of the whole
-  // layer: they may load while the predecessor finishes.
+  // layer: they may load while the predecessor finishes, requested by the
+  // thread that initialised their barriers, before the allocation.
   const int k_pre = min(stages, nt), v_pre = min(VST, nt);
   auto issue_v = [&](int lt) {
     const int vs = lt % kVStages2;
@@ -628,6 +621,15 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
     }
     for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
   }
+  __syncwarp();  // warp 0 reconverges before its collective allocation
+  grid_dep_launch();
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
   if (!VS) grid_dep_wait();  // the row normalisers come from pass 1
   {
     const float* lse = p.lse + (static_cast<size_t>(b) * p.n_heads_kv + h) * p.rows;
@@ -940,15 +942,9 @@ __global__ void __launch_bounds__(kLseThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  grid_dep_launch();
-  // both CTAs are running and their barriers are initialised before the
-  // collective allocation and any remote arrival
-  cluster_sync_all();
-  if (warp == 0) {
-    tmem_alloc_pair(tmem_slot, 512);
-    tmem_relinquish_pair();
-  }
-  // This CTA's half of every job's guide rows, its first K and V tiles.
+  // This CTA's half of every job's guide rows, its first K and V tiles,
+  // requested by the thread that initialised their barriers, before the
+  // cluster barrier and the allocation.
   const int k_pre = min(stages, nt), v_pre = min(kVStages2, nt);
   auto issue_v = [&](int lt) {
     const int vs = lt % kVStages2;
@@ -977,6 +973,15 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         tma_load_3d_hint(sK + lt * KT + kh * kHalfTileBytes, &tmk, kh * 64, tile_row(lt), h, &full_k[lt], kv_policy);
     }
     for (int lt = 0; lt < v_pre; ++lt) issue_v(lt);
+  }
+  __syncwarp();  // warp 0 reconverges before the cluster barrier and the allocation
+  grid_dep_launch();
+  // both CTAs are running and their barriers are initialised before the
+  // collective allocation and any remote arrival
+  cluster_sync_all();
+  if (warp == 0) {
+    tmem_alloc_pair(tmem_slot, 512);
+    tmem_relinquish_pair();
   }
   {
     // the caller's row normalisers: an input of the layer
