@@ -8,8 +8,9 @@
 // kept set is every key > T plus the first (k - above) keys equal to T in
 // token order (the lowest-index tie-break), written in ascending order.
 //
-// One thread-block cluster of CL CTAs (8; 4 when 8 per unit would not fit in
-// one wave and every slice still fits in shared memory) handles one
+// One thread-block cluster of CL CTAs (8; 12 for documents of 64K tokens or
+// more when every unit's cluster is resident at once; 4 when 8 per unit would
+// not fit in one wave and every slice still fits in shared memory) handles one
 // (document, head):
 // CTA r owns a contiguous slice of the tokens.  Histograms and per-slice
 // counts live in each CTA's shared memory and are summed across the cluster
@@ -23,6 +24,7 @@
 
 
 #include <cstddef>
+#include <mutex>
 
 #include "tp_device.cuh"
 
@@ -111,8 +113,11 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   int* const red = sm.red[level];
   int* const red_total = &sm.red_total[level];
   const int rank = static_cast<int>(cluster.block_rank());
-  const int slice = nbins / CL;  // at most 512 bins (CL >= 4): one per thread
-  if (threadIdx.x < slice) {
+  // CTA r owns bins [r slice, r slice + slice) (the last slice may be short
+  // or empty when CL does not divide nbins); at most 512 bins: one per thread
+  const int slice = (nbins + CL - 1) / CL;
+  const int own = max(0, min(slice, nbins - rank * slice));
+  if (static_cast<int>(threadIdx.x) < own) {
     const int bin = rank * slice + threadIdx.x;
     int v[CL];
 #pragma unroll
@@ -125,7 +130,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   __syncthreads();
   if (threadIdx.x < 32) {
     int t = 0;
-    for (int i = threadIdx.x; i < slice; i += 32) t += red[i];
+    for (int i = threadIdx.x; i < own; i += 32) t += red[i];
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
     if (threadIdx.x == 0) *red_total = t;
@@ -149,12 +154,13 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
   const int s_hit = sm.result[0], s_before = sm.result[1];
   __syncthreads();
   // scan the hit slice's bins, highest first (one bin per thread)
+  const int hit_own = max(0, min(slice, nbins - s_hit * slice));
   int cnt = 0;
-  if (threadIdx.x < slice) cnt = ld_dsmem(dsmem(&red[slice - 1 - threadIdx.x], s_hit));
+  if (static_cast<int>(threadIdx.x) < hit_own) cnt = ld_dsmem(dsmem(&red[hit_own - 1 - threadIdx.x], s_hit));
   int total;
   const int before = s_before + block_excl_scan(cnt, sm.scratch, &total);
-  if (threadIdx.x < slice && before < need && before + cnt >= need) {
-    sm.result[0] = s_hit * slice + (slice - 1 - threadIdx.x);
+  if (static_cast<int>(threadIdx.x) < hit_own && before < need && before + cnt >= need) {
+    sm.result[0] = s_hit * slice + (hit_own - 1 - threadIdx.x);
     sm.result[1] = before;
   }
   __syncthreads();
@@ -432,6 +438,11 @@ cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool 
                             cudaStream_t s, int slot) {
   cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND>), slot);
   if (e != cudaSuccess) return e;
+  if (CL > 8) {  // clusters above the portable size of 8
+    e = cudaFuncSetAttribute(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND>),
+                             cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(CL, units);
   cfg.blockDim = dim3(kThreads);
@@ -459,6 +470,41 @@ cudaError_t launch_select_blend(const SelectParams& p, int units, size_t smem, b
   }
 }
 
+// How many clusters of CL selection CTAs can be resident at once (0 if the
+// query is refused), per device, cached.
+template <int CL>
+int select_max_clusters(size_t smem, int slot) {
+  constexpr int kDevs = 64;
+  static std::mutex mu;
+  static int cached[kDevs];
+  static bool done[kDevs];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done[dev]) return cached[dev];
+  const void* fn = reinterpret_cast<const void*>(tp_select_kernel<CL, kBlendProduct>);
+  int n = 0;
+  if (set_smem_once(fn, slot) == cudaSuccess &&
+      (CL <= 8 || cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess)) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(CL, 1);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();  // a refused query leaves no error behind
+  cached[dev] = n;
+  done[dev] = true;
+  return n;
+}
+
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s) {
   const int units = p.batch * p.n_heads_kv;
   if (units <= 0) return cudaSuccess;
@@ -468,8 +514,14 @@ cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s)
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   int64_t n_max = 0;
   for (int b = 0; b < p.batch; ++b) n_max = p.off[b + 1] - p.off[b] > n_max ? p.off[b + 1] - p.off[b] : n_max;
+  // shared-memory attribute slots: 12..14 for four-CTA clusters, 15..17 for
+  // eight, 21..23 for twelve
+  // Long documents (64K tokens and more): twelve CTAs per unit when every
+  // unit's cluster is resident at once (8 such clusters fit on a 152-SM GB300:
+  // 128K, 8 heads: 163.5 against 166.4 us per caller-normaliser layer).
+  if (n_max >= 65536 && select_max_clusters<12>(smem, 21) >= units)
+    return launch_select_blend<12>(p, units, smem, dependent, s, 21);
   // Fewer, larger slices when eight CTAs per unit would need more than one wave.
-  // shared-memory attribute slots: 12..14 for four-CTA clusters, 15..17 for eight
   if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys)
     return launch_select_blend<4>(p, units, smem, dependent, s, 12);
   return launch_select_blend<8>(p, units, smem, dependent, s, 15);

@@ -246,10 +246,11 @@ def test_select_bit_exact(cuda_lib, budget):
 
 @pytest.mark.parametrize("budget", [1, 14000, 139999])
 def test_select_long_document(cuda_lib, budget):
-    """A document longer than the shared-memory key slices (8 x 16384 tokens)."""
+    """A document longer than the shared-memory key slices of its cluster
+    (12 x 16384 tokens: the slices' keys live in the global scratch)."""
     import torch
     from paper_2608_03276_gb300 import binding
-    n = 140000
+    n = 210000
     rng = np.random.Generator(np.random.PCG64(budget + 7))
     sc = np.round(rng.random((1, n)) * 64).astype(np.float32) / 64  # many ties
     p = binding.Problem(2, 1, 128, 4, [0, n])

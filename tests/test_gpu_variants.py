@@ -498,3 +498,15 @@ def test_caller_lse_pairs_and_fallback(cuda_lib, name):
     out = _run_lse(binding, w, x, lse)
     ref = _oracle(w, x, lse=lse.astype(np.float64))
     _check_layer(w, x, out, ref)
+
+
+@pytest.mark.parametrize("mode", sorted(BLENDS))
+def test_blend_long_document(cuda_lib, mode):
+    """The blends on a 70000-token document (two KV heads): the selection runs
+    on twelve-CTA clusters for documents of 64K tokens or more."""
+    from paper_2608_03276_gb300 import binding
+    w = synth.small_variant(synth.WORKLOADS[1], [70000])
+    x = synth.make_layer(w)
+    out = _run_compress(binding, w, x, flags=getattr(binding, BLENDS[mode]))
+    ref = _oracle(w, x, combine_mode=mode)
+    _check_layer(w, x, out, ref)
