@@ -36,8 +36,10 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kPer = kChunk / kThreads;  // tokens per thread in one compaction round
-constexpr int kBins1 = 2048;             // bits 31..21
-constexpr int kBins2 = 2048;             // bits 20..10
+// Digits of a key (bit 31 is always 0: keys are the bits of non-negative
+// floats), so the first digit spends its 2048 bins on bits that vary
+constexpr int kBins1 = 2048;             // bits 30..20
+constexpr int kBins2 = 1024;             // bits 19..10
 constexpr int kBins3 = 1024;             // bits 9..0
 
 constexpr int kSliceKeys = 16384;  // keys of a CTA's slice kept in shared memory
@@ -200,10 +202,8 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   };
 
   grid_dep_launch();
-  for (int i = threadIdx.x; i < kBins1; i += kThreads) {
-    sm.hist1[i] = 0;
-    sm.hist2[i] = 0;
-  }
+  for (int i = threadIdx.x; i < kBins1; i += kThreads) sm.hist1[i] = 0;
+  for (int i = threadIdx.x; i < kBins2; i += kThreads) sm.hist2[i] = 0;
   for (int i = threadIdx.x; i < kBins3; i += kThreads) sm.hist3[i] = 0;
   grid_dep_wait();  // key scores and scales come from the scoring kernels
   __syncthreads();
@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
         }
         const uint32_t key = score_key(sc);
         keys_base[kpos(i)] = key;
-        if (!p.scores_only) atomicAdd(&sm.hist1[key >> 21], 1);
+        if (!p.scores_only) atomicAdd(&sm.hist1[key >> 20], 1);
       }
       __syncthreads();
     }
@@ -319,12 +319,12 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 #pragma unroll 4
     for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
       const uint32_t key = keys_base[kpos(i)];
-      if ((key >> 21) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x7FF], 1);
+      if ((key >> 20) == static_cast<uint32_t>(d1)) atomicAdd(&sm.hist2[(key >> 10) & 0x3FF], 1);
     }
     cluster.sync();
     const int d2 = cluster_digit<CL>(cluster, sm, sm.hist2, kBins2, need, &above, 1);
     need -= above;
-    const uint32_t pre = (static_cast<uint32_t>(d1) << 11) | static_cast<uint32_t>(d2);
+    const uint32_t pre = (static_cast<uint32_t>(d1) << 10) | static_cast<uint32_t>(d2);
 #pragma unroll 4
     for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
       const uint32_t key = keys_base[kpos(i)];
