@@ -13,11 +13,20 @@
 //                            thread per key sums exp(x*sigma - lse[row]) over all
 //                            rows of the group: s_key[key] (mean over G).
 //
-// Both passes stream 128-key tiles of K with TMA (128-byte swizzle) through a
-// ring of shared-memory stages; one thread issues the MMAs; four epilogue
-// warpgroups drain TMEM.  Warp roles per CTA (18 warps):
+// Both passes stream 128-key tiles of K with TMA (128-byte swizzle, an
+// evict-first L2 policy: read once) through a ring of shared-memory stages;
+// one thread issues the MMAs; four epilogue warpgroups drain TMEM.  Warp roles
+// per CTA (18 warps, 20 with the V-scale warps):
 //   warp 0  TMEM owner + TMA producer      warp 1  MMA issuer
 //   warps 2-17  epilogue warpgroups 0-3 (warp w reads TMEM lanes 32*(w%4)..)
+//   warps 18-19 Eq. 2 scales from a V ring (pass 1; pass 2 with the caller's
+//               normalisers)
+//
+// With row normalisers given by the caller there is no pass 1: pass 2 forms
+// the scales too (tp_keyscore_kernel<D, true>, up to 256 guide rows), or, for
+// more rows, tp_keyscore_pair_kernel runs it on two-CTA clusters sharing each
+// MMA (tcgen05 cta_group::2), each CTA holding half of the guide block so that
+// the V ring fits beside it.
 #include <math.h>
 
 #include <mutex>

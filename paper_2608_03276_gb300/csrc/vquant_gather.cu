@@ -62,7 +62,7 @@ __global__ void __launch_bounds__(256) tp_vquant_kernel(const uint4* __restrict_
 // Compaction: a group of LPR lanes moves one (document, head, slot): lane
 // `part` copies the 16-byte part `part` of both the K and the V row and forms
 // the int8 codes of its 8 V values, so every lane runs the same code.  Each
-// lane keeps kUnroll slots in flight; idx < 0 marks an unused slot
+// lane keeps UNR slots in flight; idx < 0 marks an unused slot
 // (zero-filled).  The cache is written with streaming stores (evict-first in
 // L2): nothing here reads it again, and the next layer's scales and key scores
 // should find L2 room for the selection.
