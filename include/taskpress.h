@@ -37,6 +37,10 @@
  *    the kernels run surface at the next synchronisation of the stream.
  *  - Return value: TP_OK (0) or a negative TP_ERR_* code; outputs are
  *    undefined after an error.
+ *  - CUDA graphs: every call can be captured.  The first call of a problem
+ *    shape on a device sets kernel attributes and asks the device how many
+ *    thread-block clusters fit at once (the launch geometry depends on it);
+ *    make one call of the shape outside the capture first.
  *  - Inputs must be finite.  NaN scores are ranked as 0 (never preferred).
  */
 #ifndef TASKPRESS_H_

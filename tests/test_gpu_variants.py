@@ -510,3 +510,38 @@ def test_blend_long_document(cuda_lib, mode):
     out = _run_compress(binding, w, x, flags=getattr(binding, BLENDS[mode]))
     ref = _oracle(w, x, combine_mode=mode)
     _check_layer(w, x, out, ref)
+
+
+def test_lse_stack_graph_replay(cuda_lib):
+    """The caller-normaliser stack on CTA pairs (512 guide rows: cluster launches,
+    dependent launches) captured into a CUDA graph and replayed on new contents
+    of the same buffers gives the eager results."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL["c3-guide128-2053"]
+    xs = _stack(w, 3)
+    p = _problem(binding, w, xs[0].doc_offsets)
+    bufs = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in xs]
+    lses = [torch.tensor(_context_lse(w, x), device="cuda") for x in xs]
+    outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda", with_scores=False) for _ in xs]
+    for o in outs[1:]:
+        o.ws = outs[0].ws
+    binding.tp_compress_layers_lse(p, bufs, lses, w.keep_ratio, w.budget, outs, outs[0].ws)  # eager
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        binding.tp_compress_layers_lse(p, bufs, lses, w.keep_ratio, w.budget, outs, outs[0].ws)
+    # new contents: the layers (and their normalisers) in reverse order
+    for dst, s_ in zip(bufs, [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in reversed(xs)]):
+        for a, b in zip(dst, s_):
+            a.copy_(b)
+    rl = [l.clone() for l in reversed(lses)]
+    for dst, s_ in zip(lses, rl):
+        dst.copy_(s_)
+    g.replay()
+    torch.cuda.synchronize()
+    assert binding.tp_check_status(outs[0].ws) == 0
+    for l, x in enumerate(reversed(xs)):
+        single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+        binding.compress(p, *bufs[l], w.keep_ratio, w.budget, single, lse=lses[l])
+        _outputs_equal(outs[l], single, f"layer {l}")
