@@ -512,21 +512,6 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
 
 }  // namespace
 
-cudaError_t set_smem_once(const void* kernel, int slot) {
-  constexpr int kSlots = 32, kDevs = 64;
-  static std::mutex mu;
-  static bool done[kSlots][kDevs];
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (slot < 0 || slot >= kSlots || dev < 0 || dev >= kDevs)
-    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
-  std::lock_guard<std::mutex> lock(mu);
-  if (done[slot][dev]) return cudaSuccess;
-  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
-  if (e == cudaSuccess) done[slot][dev] = true;
-  return e;
-}
 
 // ---------------------------------------------------------------------------
 // Fixed device scratch for tp_guide_lse_static: the status word, the per-
@@ -613,6 +598,31 @@ int static_scratch(char** out) {
 }
 
 }  // namespace
+
+unsigned long long context_key() {
+  unsigned long long id = 0;
+  return current_ctx_id(&id) == TP_OK ? id : 0ull;
+}
+
+// Kernel attributes belong to a CUDA context as well: the cache is keyed by
+// the context's ID, so a context created after cudaDeviceReset, or a second
+// context on the device, sets them again.
+cudaError_t set_smem_once(const void* kernel, int slot) {
+  constexpr int kSlots = 32, kCtxPerSlot = 8;
+  static std::mutex mu;
+  static unsigned long long done[kSlots][kCtxPerSlot];
+  static int used[kSlots];
+  const unsigned long long key = context_key();
+  if (slot < 0 || slot >= kSlots || key == 0)
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used[slot]; ++i)
+    if (done[slot][i] == key) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+  if (e == cudaSuccess && used[slot] < kCtxPerSlot) done[slot][used[slot]++] = key;
+  return e;
+}
+
 }  // namespace tp
 
 using namespace tp;

@@ -1305,20 +1305,23 @@ cudaLaunchConfig_t pair_config(dim3 grid, size_t smem, cudaStream_t s, cudaLaunc
 }  // namespace
 
 int keyscore_pair_max_clusters(int head_dim, size_t smem) {
-  constexpr int kDevs = 64, kEntries = 8;
+  // answers cached per (CUDA context, head dim, shared memory)
+  constexpr int kEntries = 32;
   struct Entry {
+    unsigned long long ctx;
     int d;
     size_t smem;
     int clusters;
   };
   static std::mutex mu;
-  static Entry cache[kDevs][kEntries];
-  static int used[kDevs];
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  for (int i = 0; i < used[dev]; ++i)
-    if (cache[dev][i].d == head_dim && cache[dev][i].smem == smem) return cache[dev][i].clusters;
+  static Entry cache[kEntries];
+  static int used;
+  const unsigned long long ctx = context_key();
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < used; ++i)
+      if (cache[i].ctx == ctx && cache[i].d == head_dim && cache[i].smem == smem) return cache[i].clusters;
+  }
   if (set_smem_once(keyscore_pair_fn(head_dim), head_dim == 128 ? 10 : 11) != cudaSuccess) return 0;
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = pair_config(dim3(2, 1), smem, 0, attr, false);
@@ -1326,7 +1329,8 @@ int keyscore_pair_max_clusters(int head_dim, size_t smem) {
   if (cudaOccupancyMaxActiveClusters(&clusters, keyscore_pair_fn(head_dim), &cfg) != cudaSuccess)
     clusters = 0;
   cudaGetLastError();  // a refused query leaves no error behind
-  if (used[dev] < kEntries) cache[dev][used[dev]++] = Entry{head_dim, smem, clusters};
+  std::lock_guard<std::mutex> lock(mu);
+  if (ctx != 0 && used < kEntries) cache[used++] = Entry{ctx, head_dim, smem, clusters};
   return clusters;
 }
 

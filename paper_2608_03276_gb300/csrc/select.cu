@@ -471,17 +471,20 @@ cudaError_t launch_select_blend(const SelectParams& p, int units, size_t smem, b
 }
 
 // How many clusters of CL selection CTAs can be resident at once (0 if the
-// query is refused), per device, cached.
+// query is refused), cached per CUDA context.
 template <int CL>
 int select_max_clusters(size_t smem, int slot) {
-  constexpr int kDevs = 64;
+  constexpr int kEntries = 16;
   static std::mutex mu;
-  static int cached[kDevs];
-  static bool done[kDevs];
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kDevs) return 0;
-  std::lock_guard<std::mutex> lock(mu);
-  if (done[dev]) return cached[dev];
+  static unsigned long long ctxs[kEntries];
+  static int answers[kEntries];
+  static int used;
+  const unsigned long long ctx = context_key();
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < used; ++i)
+      if (ctxs[i] == ctx) return answers[i];
+  }
   const void* fn = reinterpret_cast<const void*>(tp_select_kernel<CL, kBlendProduct>);
   int n = 0;
   if (set_smem_once(fn, slot) == cudaSuccess &&
@@ -500,8 +503,11 @@ int select_max_clusters(size_t smem, int slot) {
     if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
   }
   cudaGetLastError();  // a refused query leaves no error behind
-  cached[dev] = n;
-  done[dev] = true;
+  std::lock_guard<std::mutex> lock(mu);
+  if (ctx != 0 && used < kEntries) {
+    ctxs[used] = ctx;
+    answers[used++] = n;
+  }
   return n;
 }
 

@@ -168,8 +168,13 @@ cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s)
 cudaError_t launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
 
 // Raises a kernel's dynamic shared-memory limit to the device maximum, once per
-// (kernel slot, device); `slot` names the kernel in a small registry.
+// (kernel slot, CUDA context); `slot` names the kernel in a small registry.
 cudaError_t set_smem_once(const void* kernel, int slot);
+// The current CUDA context's process-unique ID (cuCtxGetId; the device's
+// primary context is bound first when none is current), 0 if unavailable.
+// Caches of per-context state (kernel attributes, co-residency answers) are
+// keyed by it.
+unsigned long long context_key();
 
 // Shared-memory layout sizes of the scoring kernels (host side).
 size_t lse_smem_bytes(int head_dim, int rows_pad, int stages);
