@@ -275,7 +275,7 @@ bool pair_geometry(const Plan& P, PairGeometry* G) {
     --G->stages;
   G->smem = keyscore_pair_smem_bytes(P.d, P.rows_mma, G->stages);
   if (G->smem > size_t(kMaxSmem)) return false;
-  const int clusters = keyscore_pair_max_clusters(P.d, G->smem);
+  const int clusters = keyscore_pair_max_clusters(P.d, P.rows_mma, G->smem);
   if (clusters <= 0) return false;
   int64_t tiles_total = 0;
   for (int b = 0; b < P.batch; ++b) tiles_total += (P.off[b + 1] - P.off[b] + 255) / 256;

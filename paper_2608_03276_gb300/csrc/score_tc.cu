@@ -23,7 +23,8 @@
 //               normalisers)
 //
 // With row normalisers given by the caller there is no pass 1: pass 2 forms
-// the scales too (tp_keyscore_kernel<D, true>, up to 256 guide rows), or, for
+// the scales too (tp_keyscore_kernel<D, true, NH>, where the guide block fits beside
+// two K and two V stages: up to 256 guide rows at d = 128), or, for
 // more rows, tp_keyscore_pair_kernel runs it on two-CTA clusters sharing each
 // MMA (tcgen05 cta_group::2), each CTA holding half of the guide block so that
 // the V ring fits beside it.
@@ -541,7 +542,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
 // the call: as a programmatic dependent (the next layer of a stack) the kernel
 // waits for its predecessor only before its first store.
 // ---------------------------------------------------------------------------
-template <int D, bool VS>
+template <int D, bool VS, int NH>
 __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
     tp_keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                        const __grid_constant__ CUtensorMap tmq, const __grid_constant__ KeyScoreParams p) {
@@ -551,7 +552,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
   constexpr uint32_t KT = NKH * kHalfTileBytes;
   constexpr int VST = VS ? kVStages2 : 0;
   const int stages = p.stages, rows_pad = p.rows_pad, rows_mma = p.rows_mma;
-  const int nh = (rows_mma + 255) / 256;
+  constexpr int nh = NH;  // 256-row parts of the guide block per key tile
   const ScoreSmem L = score_layout(D, rows_pad, stages + VST, keyscore_extra_bytes(rows_pad));
   uint8_t* sQ = smem + L.q;
   uint8_t* sK = smem + L.k;
@@ -881,7 +882,7 @@ __host__ __device__ inline PairSmem pair_layout(int head_dim, int nh, int stages
   return L;
 }
 
-template <int D>
+template <int D, int NH>
 __global__ void __launch_bounds__(kLseThreads, 1)
     tp_keyscore_pair_kernel(const __grid_constant__ CUtensorMap tmk,
                             const __grid_constant__ CUtensorMap tmv,
@@ -893,7 +894,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
   constexpr uint32_t KT = NKH * kHalfTileBytes;
   constexpr int kPairTile = 2 * kKeyTile;
   const int stages = p.stages, rows_mma = p.rows_mma;
-  const int nh = (rows_mma + 255) / 256;
+  constexpr int nh = NH;  // 256-row parts of the guide block per pair tile
   const PairSmem L = pair_layout(D, nh, stages);
   uint8_t* sQ = smem + L.q;
   uint8_t* sK = smem + L.k;
@@ -1246,13 +1247,14 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUt
   return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
-template <int D, bool VS>
+template <int D, bool VS, int NH>
 cudaError_t launch_keyscore_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                               const KeyScoreParams& p, dim3 grid, size_t smem, bool dependent,
                               cudaStream_t s) {
-  // shared-memory attribute slots 8, 9 (plain) and 19, 20 (with the scales)
-  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<D, VS>),
-                                (VS ? 19 : 8) + (D == 128 ? 0 : 1));
+  // shared-memory attribute slots: 8, 9 and 24, 25 (one and two row parts);
+  // with the scales 19, 20 and 26, 27
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<D, VS, NH>),
+                                (VS ? (NH == 2 ? 26 : 19) : (NH == 2 ? 24 : 8)) + (D == 128 ? 0 : 1));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
@@ -1264,24 +1266,46 @@ cudaError_t launch_keyscore_t(const CUtensorMap& tmk, const CUtensorMap& tmv, co
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<D, VS>, tmk, tmv, tmq, p);
+  return cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<D, VS, NH>, tmk, tmv, tmq, p);
 }
 
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             bool dependent, cudaStream_t s) {
-  if (p.gamma)
-    return head_dim == 128 ? launch_keyscore_t<128, true>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                           : launch_keyscore_t<64, true>(tmk, tmv, tmq, p, grid, smem, dependent, s);
-  return head_dim == 128 ? launch_keyscore_t<128, false>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                         : launch_keyscore_t<64, false>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  // The guide block is taken in 256-row parts per key tile, one or two: a
+  // compile-time count, so each shape gets its own unrolled epilogue (at 512
+  // rows 149 against 161 us per 128K layer, at 256 rows 162 against 177 on the
+  // ragged batch, with a runtime count).
+  const bool two = p.rows_mma > 256;
+  if (p.gamma) {
+    if (two)
+      return head_dim == 128 ? launch_keyscore_t<128, true, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                             : launch_keyscore_t<64, true, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+    return head_dim == 128 ? launch_keyscore_t<128, true, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                           : launch_keyscore_t<64, true, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  }
+  if (two)
+    return head_dim == 128 ? launch_keyscore_t<128, false, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                           : launch_keyscore_t<64, false, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  return head_dim == 128 ? launch_keyscore_t<128, false, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                         : launch_keyscore_t<64, false, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
 namespace {
 
-const void* keyscore_pair_fn(int head_dim) {
-  return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128>)
-                         : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64>);
+// The guide block in one or two 256-row parts per pair tile (a compile-time
+// count, as in tp_keyscore_kernel).
+const void* keyscore_pair_fn(int head_dim, int rows_mma) {
+  if (rows_mma > 256)
+    return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128, 2>)
+                           : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64, 2>);
+  return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128, 1>)
+                         : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64, 1>);
+}
+
+// shared-memory attribute slots 10, 11 (two row parts) and 28, 29 (one)
+int keyscore_pair_slot(int head_dim, int rows_mma) {
+  return (rows_mma > 256 ? 10 : 28) + (head_dim == 128 ? 0 : 1);
 }
 
 cudaLaunchConfig_t pair_config(dim3 grid, size_t smem, cudaStream_t s, cudaLaunchAttribute (&attr)[2],
@@ -1304,12 +1328,13 @@ cudaLaunchConfig_t pair_config(dim3 grid, size_t smem, cudaStream_t s, cudaLaunc
 
 }  // namespace
 
-int keyscore_pair_max_clusters(int head_dim, size_t smem) {
-  // answers cached per (CUDA context, head dim, shared memory)
+int keyscore_pair_max_clusters(int head_dim, int rows_mma, size_t smem) {
+  // answers cached per (CUDA context, kernel, shared memory)
   constexpr int kEntries = 32;
+  const void* fn = keyscore_pair_fn(head_dim, rows_mma);
   struct Entry {
     unsigned long long ctx;
-    int d;
+    const void* fn;
     size_t smem;
     int clusters;
   };
@@ -1320,29 +1345,33 @@ int keyscore_pair_max_clusters(int head_dim, size_t smem) {
   {
     std::lock_guard<std::mutex> lock(mu);
     for (int i = 0; i < used; ++i)
-      if (cache[i].ctx == ctx && cache[i].d == head_dim && cache[i].smem == smem) return cache[i].clusters;
+      if (cache[i].ctx == ctx && cache[i].fn == fn && cache[i].smem == smem) return cache[i].clusters;
   }
-  if (set_smem_once(keyscore_pair_fn(head_dim), head_dim == 128 ? 10 : 11) != cudaSuccess) return 0;
+  if (set_smem_once(fn, keyscore_pair_slot(head_dim, rows_mma)) != cudaSuccess) return 0;
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = pair_config(dim3(2, 1), smem, 0, attr, false);
   int clusters = 0;
-  if (cudaOccupancyMaxActiveClusters(&clusters, keyscore_pair_fn(head_dim), &cfg) != cudaSuccess)
+  if (cudaOccupancyMaxActiveClusters(&clusters, fn, &cfg) != cudaSuccess)
     clusters = 0;
   cudaGetLastError();  // a refused query leaves no error behind
   std::lock_guard<std::mutex> lock(mu);
-  if (ctx != 0 && used < kEntries) cache[used++] = Entry{ctx, head_dim, smem, clusters};
+  if (ctx != 0 && used < kEntries) cache[used++] = Entry{ctx, fn, smem, clusters};
   return clusters;
 }
 
 cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
                                  const CUtensorMap& tmq, const KeyScoreParams& p, int head_dim,
                                  dim3 grid, size_t smem, bool dependent, cudaStream_t s) {
-  cudaError_t e = set_smem_once(keyscore_pair_fn(head_dim), head_dim == 128 ? 10 : 11);
+  cudaError_t e =
+      set_smem_once(keyscore_pair_fn(head_dim, p.rows_mma), keyscore_pair_slot(head_dim, p.rows_mma));
   if (e != cudaSuccess) return e;
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = pair_config(grid, smem, s, attr, dependent);
-  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128>, tmk, tmv, tmq, p)
-                         : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64>, tmk, tmv, tmq, p);
+  if (p.rows_mma > 256)
+    return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128, 2>, tmk, tmv, tmq, p)
+                           : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64, 2>, tmk, tmv, tmq, p);
+  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128, 1>, tmk, tmv, tmq, p)
+                         : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64, 1>, tmk, tmv, tmq, p);
 }
 
 }  // namespace tp

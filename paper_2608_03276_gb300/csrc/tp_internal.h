@@ -159,9 +159,10 @@ cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmv, cons
 cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
                                  const CUtensorMap& tmq, const KeyScoreParams& p, int head_dim,
                                  dim3 grid, size_t smem, bool dependent, cudaStream_t s);
-// How many CTA pairs of the pair kernel can be resident at once (0 when the
-// device or the query refuses a two-CTA cluster of that size).
-int keyscore_pair_max_clusters(int head_dim, size_t smem);
+// How many CTA pairs of the pair kernel for this head dim and guide block can
+// be resident at once (0 when the device or the query refuses a two-CTA
+// cluster of that size).
+int keyscore_pair_max_clusters(int head_dim, int rows_mma, size_t smem);
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
