@@ -608,7 +608,7 @@ unsigned long long context_key() {
 // the context's ID, so a context created after cudaDeviceReset, or a second
 // context on the device, sets them again.
 cudaError_t set_smem_once(const void* kernel, int slot) {
-  constexpr int kSlots = 32, kCtxPerSlot = 8;
+  constexpr int kSlots = 64, kCtxPerSlot = 8;
   static std::mutex mu;
   static unsigned long long done[kSlots][kCtxPerSlot];
   static int used[kSlots];

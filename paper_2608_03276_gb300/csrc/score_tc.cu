@@ -530,11 +530,13 @@ __global__ void __launch_bounds__(kLseThreads, 1)
 // Pass 2: s_key[key] = (1/G) sum over rows of 2^(x*c2 - lse[row]*log2(e)).
 //
 // Keys sit on TMEM lanes (D[key, row] = K Q^T); each MMA job covers one
-// 128-key tile and up to 256 guide rows (N).  All four epilogue warpgroups
-// share every job: warpgroup g reduces the 32-column chunks c = g, g+4 of it,
-// so sixteen warps drain each TMEM buffer.  A thread's partial sum for its key
-// (over its chunks of all row halves of the tile) goes to shared memory, and
-// after a named barrier warpgroup 0 adds the four partials in a fixed order.
+// 128-key tile and one 256-row part of the guide block (N).  Two groups of
+// eight epilogue warps take alternate jobs, each draining one of two TMEM
+// buffers; a warp's partial sum for its key over its chunks of a job goes to
+// one of four rotating shared-memory slots, and a tile's partials are added in
+// a fixed order once all have arrived (bounded mbarrier waits).  NH (one or two
+// parts) and FULL (every part eight 32-row chunks) are template parameters,
+// so the epilogue is unrolled for the shape with no per-chunk guards.
 //
 // VS (the caller's normalisers, at most 256 guide rows): the same CTA also
 // forms the Eq. 2 scale of every token of its key range from a V ring, as in
@@ -542,7 +544,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
 // the call: as a programmatic dependent (the next layer of a stack) the kernel
 // waits for its predecessor only before its first store.
 // ---------------------------------------------------------------------------
-template <int D, bool VS, int NH>
+template <int D, bool VS, int NH, bool FULL>
 __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
     tp_keyscore_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                        const __grid_constant__ CUtensorMap tmq, const __grid_constant__ KeyScoreParams p) {
@@ -780,7 +782,7 @@ __global__ void __launch_bounds__(VS ? kLseThreads : kThreads, 1)
         if (ok && !mbar_wait(&tfull[buf], (j >> 1) & 1, abort_flag)) ok = false;
         if (!ok) continue;
         tc_fence_after();
-        const int nch = min(256, rows_mma - 256 * hh) / 32;
+        const int nch = FULL ? 8 : min(256, rows_mma - 256 * hh) / 32;
         const uint32_t tb = tlane + buf * 256;
         const int ch = 4 * cg;
         float acc = 0.f;
@@ -882,7 +884,7 @@ __host__ __device__ inline PairSmem pair_layout(int head_dim, int nh, int stages
   return L;
 }
 
-template <int D, int NH>
+template <int D, int NH, bool FULL>
 __global__ void __launch_bounds__(kLseThreads, 1)
     tp_keyscore_pair_kernel(const __grid_constant__ CUtensorMap tmk,
                             const __grid_constant__ CUtensorMap tmv,
@@ -1143,7 +1145,7 @@ __global__ void __launch_bounds__(kLseThreads, 1)
         if (ok && !mbar_wait(&tfull[buf], (j >> 1) & 1, abort_flag)) ok = false;
         if (!ok) continue;
         tc_fence_after();
-        const int nch = min(256, rows_mma - 256 * hh) / 32;
+        const int nch = FULL ? 8 : min(256, rows_mma - 256 * hh) / 32;
         const uint32_t tb = tlane + buf * 256;
         const int ch = 4 * cg;
         float acc = 0.f;
@@ -1247,14 +1249,13 @@ cudaError_t launch_lse(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUt
   return launch_lse_t<64, 4>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
-template <int D, bool VS, int NH>
+template <int D, bool VS, int NH, bool FULL>
 cudaError_t launch_keyscore_t(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                               const KeyScoreParams& p, dim3 grid, size_t smem, bool dependent,
                               cudaStream_t s) {
-  // shared-memory attribute slots: 8, 9 and 24, 25 (one and two row parts);
-  // with the scales 19, 20 and 26, 27
-  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<D, VS, NH>),
-                                (VS ? (NH == 2 ? 26 : 19) : (NH == 2 ? 24 : 8)) + (D == 128 ? 0 : 1));
+  // shared-memory attribute slots 32..47, one per instantiation
+  const int slot = 32 + ((D == 64) << 3 | VS << 2 | (NH == 2) << 1 | !FULL);
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_keyscore_kernel<D, VS, NH, FULL>), slot);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
@@ -1266,46 +1267,69 @@ cudaError_t launch_keyscore_t(const CUtensorMap& tmk, const CUtensorMap& tmv, co
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<D, VS, NH>, tmk, tmv, tmq, p);
+  return cudaLaunchKernelEx(&cfg, tp_keyscore_kernel<D, VS, NH, FULL>, tmk, tmv, tmq, p);
 }
 
+template <int D, bool VS>
+cudaError_t launch_keyscore_d(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
+                              const KeyScoreParams& p, dim3 grid, size_t smem, bool dependent,
+                              cudaStream_t s) {
+  const bool full = p.rows_mma % 256 == 0;
+  if (p.rows_mma > 256)
+    return full ? launch_keyscore_t<D, VS, 2, true>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                : launch_keyscore_t<D, VS, 2, false>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  return full ? launch_keyscore_t<D, VS, 1, true>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+              : launch_keyscore_t<D, VS, 1, false>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+}
+
+// The guide block is taken in 256-row parts per key tile, one or two, each of
+// eight 32-row chunks except perhaps the last: both are compile-time, so each
+// shape gets its own unrolled epilogue with no per-chunk guards where every
+// part is whole.  Against run-time counts, per 128K layer at 512 rows, pass 2
+// takes 88.6 against 107.8 us.
 cudaError_t launch_keyscore(const CUtensorMap& tmk, const CUtensorMap& tmv, const CUtensorMap& tmq,
                             const KeyScoreParams& p, int head_dim, dim3 grid, size_t smem,
                             bool dependent, cudaStream_t s) {
-  // The guide block is taken in 256-row parts per key tile, one or two: a
-  // compile-time count, so each shape gets its own unrolled epilogue (at 512
-  // rows 149 against 161 us per 128K layer, at 256 rows 162 against 177 on the
-  // ragged batch, with a runtime count).
-  const bool two = p.rows_mma > 256;
-  if (p.gamma) {
-    if (two)
-      return head_dim == 128 ? launch_keyscore_t<128, true, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                             : launch_keyscore_t<64, true, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
-    return head_dim == 128 ? launch_keyscore_t<128, true, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                           : launch_keyscore_t<64, true, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
-  }
-  if (two)
-    return head_dim == 128 ? launch_keyscore_t<128, false, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                           : launch_keyscore_t<64, false, 2>(tmk, tmv, tmq, p, grid, smem, dependent, s);
-  return head_dim == 128 ? launch_keyscore_t<128, false, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s)
-                         : launch_keyscore_t<64, false, 1>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  if (p.gamma)
+    return head_dim == 128 ? launch_keyscore_d<128, true>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                           : launch_keyscore_d<64, true>(tmk, tmv, tmq, p, grid, smem, dependent, s);
+  return head_dim == 128 ? launch_keyscore_d<128, false>(tmk, tmv, tmq, p, grid, smem, dependent, s)
+                         : launch_keyscore_d<64, false>(tmk, tmv, tmq, p, grid, smem, dependent, s);
 }
 
 namespace {
 
-// The guide block in one or two 256-row parts per pair tile (a compile-time
-// count, as in tp_keyscore_kernel).
-const void* keyscore_pair_fn(int head_dim, int rows_mma) {
+// The pair kernel for a head dim and guide block: one or two 256-row parts per
+// pair tile, whole or not (compile-time, as in tp_keyscore_kernel).
+template <int D>
+const void* keyscore_pair_fn_d(int rows_mma) {
+  const bool full = rows_mma % 256 == 0;
   if (rows_mma > 256)
-    return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128, 2>)
-                           : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64, 2>);
-  return head_dim == 128 ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<128, 1>)
-                         : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<64, 1>);
+    return full ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<D, 2, true>)
+                : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<D, 2, false>);
+  return full ? reinterpret_cast<const void*>(tp_keyscore_pair_kernel<D, 1, true>)
+              : reinterpret_cast<const void*>(tp_keyscore_pair_kernel<D, 1, false>);
 }
 
-// shared-memory attribute slots 10, 11 (two row parts) and 28, 29 (one)
+const void* keyscore_pair_fn(int head_dim, int rows_mma) {
+  return head_dim == 128 ? keyscore_pair_fn_d<128>(rows_mma) : keyscore_pair_fn_d<64>(rows_mma);
+}
+
+// The instantiation keyscore_pair_fn names, launched.
+template <int D>
+cudaError_t launch_pair_d(const cudaLaunchConfig_t& cfg, const CUtensorMap& tmk, const CUtensorMap& tmv,
+                          const CUtensorMap& tmq, const KeyScoreParams& p) {
+  const bool full = p.rows_mma % 256 == 0;
+  if (p.rows_mma > 256)
+    return full ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<D, 2, true>, tmk, tmv, tmq, p)
+                : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<D, 2, false>, tmk, tmv, tmq, p);
+  return full ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<D, 1, true>, tmk, tmv, tmq, p)
+              : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<D, 1, false>, tmk, tmv, tmq, p);
+}
+
+// shared-memory attribute slots 48..55, one per instantiation
 int keyscore_pair_slot(int head_dim, int rows_mma) {
-  return (rows_mma > 256 ? 10 : 28) + (head_dim == 128 ? 0 : 1);
+  return 48 + ((head_dim == 64) << 2 | (rows_mma > 256) << 1 | (rows_mma % 256 != 0));
 }
 
 cudaLaunchConfig_t pair_config(dim3 grid, size_t smem, cudaStream_t s, cudaLaunchAttribute (&attr)[2],
@@ -1367,11 +1391,8 @@ cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
   if (e != cudaSuccess) return e;
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = pair_config(grid, smem, s, attr, dependent);
-  if (p.rows_mma > 256)
-    return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128, 2>, tmk, tmv, tmq, p)
-                           : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64, 2>, tmk, tmv, tmq, p);
-  return head_dim == 128 ? cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<128, 1>, tmk, tmv, tmq, p)
-                         : cudaLaunchKernelEx(&cfg, tp_keyscore_pair_kernel<64, 1>, tmk, tmv, tmq, p);
+  return head_dim == 128 ? launch_pair_d<128>(cfg, tmk, tmv, tmq, p)
+                         : launch_pair_d<64>(cfg, tmk, tmv, tmq, p);
 }
 
 }  // namespace tp
