@@ -18,7 +18,8 @@
 // so the whole selection is one launch:
 //   A  form keys (Eq. 1 pooling x gamma in the fused path), digit-1 histogram
 //   B  digit-2 histogram under the chosen prefix        C  digit-3 histogram
-//   D  (> T, == T) counts per slice, then the ordered compaction into idx.
+//   D  (> T, == T) counts per slice (read off its histograms), then the
+//      ordered compaction into idx.
 // The kept rows are then copied by the grid-wide gather kernel.
 #include <cooperative_groups.h>
 
@@ -312,6 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 
   uint32_t thr = 0;
   int need_eq = -1;  // -1: keep every token of the document
+  // this thread's share of the slice's counts of keys above T and equal to T
+  int gt_part = 0, eq_part = 0;
   if (kk > 0 && kk < n) {
     int above;
     const int d1 = cluster_digit<CL>(cluster, sm, sm.hist1, kBins1, kk, &above, 0);
@@ -334,6 +337,15 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
     const int d3 = cluster_digit<CL>(cluster, sm, sm.hist3, kBins3, need, &above, 2);
     need_eq = need - above;
     thr = (pre << 10) | static_cast<uint32_t>(d3);
+    // The slice's own histograms give its counts: a key above T lies in a
+    // higher digit-1 bin, or shares digit 1 and lies in a higher digit-2 bin,
+    // or shares both and lies in a higher digit-3 bin; keys equal to T fill
+    // digit-3 bin d3.  (cluster_digit ends with a block barrier, so every
+    // local histogram update is visible.)
+    for (int i = d1 + 1 + static_cast<int>(threadIdx.x); i < kBins1; i += kThreads) gt_part += sm.hist1[i];
+    for (int i = d2 + 1 + static_cast<int>(threadIdx.x); i < kBins2; i += kThreads) gt_part += sm.hist2[i];
+    for (int i = d3 + 1 + static_cast<int>(threadIdx.x); i < kBins3; i += kThreads) gt_part += sm.hist3[i];
+    if (threadIdx.x == 0) eq_part = sm.hist3[d3];
   } else {
     // the same cluster-wide barriers as the other branch: one per digit
     // search (three searches) and one after each of the two later histograms
@@ -343,15 +355,9 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 
   // D: counts of this slice, then prefix over the slices before it
   {
-    int gt = 0, eq = 0;
-    if (kk > 0) {
-#pragma unroll 4
-      for (int i = s0 + threadIdx.x; i < s1; i += kThreads) {
-        const uint32_t key = keys_base[kpos(i)];
-        if (need_eq < 0 || key > thr) ++gt;
-        else if (key == thr) ++eq;
-      }
-    }
+    // with every token kept (need_eq < 0) the slice counts entirely above T
+    int gt = need_eq < 0 ? (kk > 0 && threadIdx.x == 0 ? s1 - s0 : 0) : gt_part;
+    int eq = need_eq < 0 ? 0 : eq_part;
     if (s1 - s0 < 32768) {  // one block sum of (> T) << 16 | (== T), no overflow
       const int both = block_sum((gt << 16) | eq, sm.scratch);
       gt = both >> 16;

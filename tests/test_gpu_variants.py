@@ -545,3 +545,38 @@ def test_lse_stack_graph_replay(cuda_lib):
         single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
         binding.compress(p, *bufs[l], w.keep_ratio, w.budget, single, lse=lses[l])
         _outputs_equal(outs[l], single, f"layer {l}")
+
+
+# Guide blocks of one or two 256-row parts per key tile, whole or not, at both
+# head dims.  Each (part count, whole) pair is its own compiled instance of the
+# pass-2 kernels: one CTA per key range without the scales (two-pass layer) and
+# with them (caller's normalisers), and the CTA-pair kernel (caller's
+# normalisers above 256 rows at d 128).  Both paths are checked against the
+# oracle for every shape.
+PART_SHAPES = {
+    # name: (query heads, KV heads, head dim, guide tokens, document lengths)
+    "d128-m224": (28, 4, 128, 32, [1100]),      # one part, not whole
+    "d128-m320": (10, 2, 128, 64, [700, 300]),  # two parts, the second not whole; CTA pairs
+    "d128-m384": (12, 4, 128, 128, [900]),      # two parts, the second not whole; CTA pairs
+    "d64-m288": (18, 2, 64, 32, [600, 257]),    # two parts at d 64: one CTA forms the scales
+    "d64-m512": (8, 2, 64, 128, [513]),         # two whole parts at d 64
+}
+
+
+@pytest.mark.parametrize("name", sorted(PART_SHAPES))
+def test_guide_part_shapes(cuda_lib, name):
+    from paper_2608_03276_gb300 import binding
+    hq, hkv, d, lt, lens = PART_SHAPES[name]
+    w = synth.small_variant(synth.WORKLOADS[2], lens).with_(
+        n_heads_q=hq, n_heads_kv=hkv, head_dim=d, guide_len=lt)
+    assert w.group * lt == {"d128-m224": 224, "d128-m320": 320, "d128-m384": 384,
+                            "d64-m288": 288, "d64-m512": 512}[name]
+    x = synth.make_layer(w)
+    p = _problem(binding, w, x.doc_offsets)
+    # the scales are formed inside the scoring kernel (no separate quantiser)
+    assert binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget, binding.MODE_CALLER_LSE) == 3
+    out = _run_compress(binding, w, x)
+    _check_layer(w, x, out, _oracle(w, x))
+    lse = _context_lse(w, x)
+    out = _run_lse(binding, w, x, lse)
+    _check_layer(w, x, out, _oracle(w, x, lse=lse.astype(np.float64)))
