@@ -36,7 +36,6 @@ namespace tp {
 namespace {
 
 constexpr int kThreads = 512;
-constexpr int kPer = kChunk / kThreads;  // tokens per thread in one compaction round
 // Digits of a key (bit 31 is always 0: keys are the bits of non-negative
 // floats), so the first digit spends its 2048 bins on bits that vary
 constexpr int kBins1 = 2048;             // bits 30..20
@@ -176,7 +175,7 @@ __device__ int cluster_digit(cg::cluster_group& cluster, SelectSmem& sm, const i
 // CL: CTAs per (document, head) cluster.  BLEND: how the fused path combines
 // the pooled key score with the scale (a compile-time choice, so the product
 // kernel's per-token loop carries nothing for the other blends).
-template <int CL, int BLEND>
+template <int CL, int BLEND, int KP>
 __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_constant__ SelectParams p) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
@@ -396,14 +395,14 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   cluster.sync();  // no CTA leaves while another may still read its counts
 
   if (kk <= 0) return;
-  // ordered compaction in rounds of kChunk tokens: a token's slot is
+  // ordered compaction in rounds of KP tokens per thread: a token's slot is
   // (tokens > T before it) + min(tokens == T before it, need_eq)
-  for (int base = s0; base < s1; base += kChunk) {
-    const int j0 = base + threadIdx.x * kPer;
+  for (int base = s0; base < s1; base += KP * kThreads) {
+    const int j0 = base + threadIdx.x * KP;
     int ngt = 0, neq = 0;
-    uint32_t kv[kPer];
+    uint32_t kv[KP];
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) {
+    for (int e = 0; e < KP; ++e) {
       const int j = j0 + e;
       kv[e] = j < s1 ? keys_base[kpos(j)] : 0u;
       if (j < s1) {
@@ -418,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
     int gt_rank = gt_before + (pre >> 16);
     int eq_rank = eq_before + (pre & 0xFFFF);
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) {
+    for (int e = 0; e < KP; ++e) {
       const int j = j0 + e;
       if (j >= s1) break;
       const bool is_gt = need_eq < 0 || kv[e] > thr;
@@ -439,13 +438,13 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
 
 size_t select_smem_bytes() { return sizeof(SelectSmem); }
 
-template <int CL, int BLEND>
+template <int CL, int BLEND, int KP>
 cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool dependent,
                             cudaStream_t s, int slot) {
-  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND>), slot);
+  cudaError_t e = set_smem_once(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND, KP>), slot);
   if (e != cudaSuccess) return e;
   if (CL > 8) {  // clusters above the portable size of 8
-    e = cudaFuncSetAttribute(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND>),
+    e = cudaFuncSetAttribute(reinterpret_cast<const void*>(tp_select_kernel<CL, BLEND, KP>),
                              cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
   }
@@ -463,16 +462,18 @@ cudaError_t launch_select_t(const SelectParams& p, int units, size_t smem, bool 
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = dependent ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL, BLEND>, p);
+  return cudaLaunchKernelEx(&cfg, tp_select_kernel<CL, BLEND, KP>, p);
 }
 
-template <int CL>
+template <int CL, int KP = 16>
 cudaError_t launch_select_blend(const SelectParams& p, int units, size_t smem, bool dependent,
                                 cudaStream_t s, int slot0) {
   switch (p.blend) {
-    case kBlendNormAdd: return launch_select_t<CL, kBlendNormAdd>(p, units, smem, dependent, s, slot0 + 1);
-    case kBlendHarmonic: return launch_select_t<CL, kBlendHarmonic>(p, units, smem, dependent, s, slot0 + 2);
-    default: return launch_select_t<CL, kBlendProduct>(p, units, smem, dependent, s, slot0);
+    case kBlendNormAdd:
+      return launch_select_t<CL, kBlendNormAdd, KP>(p, units, smem, dependent, s, slot0 + 1);
+    case kBlendHarmonic:
+      return launch_select_t<CL, kBlendHarmonic, KP>(p, units, smem, dependent, s, slot0 + 2);
+    default: return launch_select_t<CL, kBlendProduct, KP>(p, units, smem, dependent, s, slot0);
   }
 }
 
@@ -491,7 +492,7 @@ int select_max_clusters(size_t smem, int slot) {
     for (int i = 0; i < used; ++i)
       if (ctxs[i] == ctx) return answers[i];
   }
-  const void* fn = reinterpret_cast<const void*>(tp_select_kernel<CL, kBlendProduct>);
+  const void* fn = reinterpret_cast<const void*>(tp_select_kernel<CL, kBlendProduct, 16>);
   int n = 0;
   if (set_smem_once(fn, slot) == cudaSuccess &&
       (CL <= 8 || cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess)) {
@@ -527,12 +528,18 @@ cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s)
   int64_t n_max = 0;
   for (int b = 0; b < p.batch; ++b) n_max = p.off[b + 1] - p.off[b] > n_max ? p.off[b + 1] - p.off[b] : n_max;
   // shared-memory attribute slots: 12..14 for four-CTA clusters, 15..17 for
-  // eight, 21..23 for twelve
+  // eight, 21..23 and 56..58 for twelve
   // Long documents (64K tokens and more): twelve CTAs per unit when every
   // unit's cluster is resident at once (8 such clusters fit on a 152-SM GB300:
   // 128K, 8 heads: 163.5 against 166.4 us per caller-normaliser layer).
-  if (n_max >= 65536 && select_max_clusters<12>(smem, 21) >= units)
+  // Slices above 16 tokens per thread (128K: 10.9K tokens) compact in one
+  // round of 22 per thread rather than two of 16 (1.8 us per 128K layer; 22
+  // per thread everywhere was slower on shorter slices).
+  if (n_max >= 65536 && select_max_clusters<12>(smem, 21) >= units) {
+    const int64_t per_cta = (((n_max + 11) / 12) + 3) & ~int64_t(3);
+    if (per_cta > 16 * kThreads) return launch_select_blend<12, 22>(p, units, smem, dependent, s, 56);
     return launch_select_blend<12>(p, units, smem, dependent, s, 21);
+  }
   // Fewer, larger slices when eight CTAs per unit would need more than one wave.
   if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys)
     return launch_select_blend<4>(p, units, smem, dependent, s, 12);

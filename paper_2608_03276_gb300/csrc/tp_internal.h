@@ -69,7 +69,6 @@ struct KeyScoreParams {
   int* status;
 };
 
-constexpr int kChunk = 8192;       // tokens per compaction round in the selection kernel
 
 // Blends of the pooled key score a and the scale g (Eq. 3 and the Sec. 4.4
 // aggregation ablation): a * g; a / ||a||_2 + g / ||g||_2 per (document,
