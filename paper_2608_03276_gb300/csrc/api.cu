@@ -420,6 +420,13 @@ void fill_select(const Plan& P, char* ws, SelectParams* sp) {
   memset(sp, 0, sizeof(*sp));
   for (int b = 0; b <= P.batch; ++b) sp->off[b] = P.off[b];
   for (int b = 0; b < P.batch; ++b) sp->kept[b] = P.kept[b];
+  // the selection launches the longest documents' clusters first (ties in
+  // document order): with more clusters than fit at once, the last wave then
+  // holds the shortest documents
+  for (int b = 0; b < P.batch; ++b) sp->order[b] = static_cast<int16_t>(b);
+  std::stable_sort(sp->order, sp->order + P.batch, [&](int16_t x, int16_t y) {
+    return P.off[x + 1] - P.off[x] > P.off[y + 1] - P.off[y];
+  });
   sp->batch = P.batch;
   sp->n_heads_kv = P.hkv;
   sp->head_dim = P.d;

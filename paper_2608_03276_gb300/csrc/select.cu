@@ -181,8 +181,10 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
-  const int unit = blockIdx.y;
-  const int b = unit / p.n_heads_kv, h = unit % p.n_heads_kv;
+  // clusters launch in blockIdx.y order: the longest documents' units first,
+  // so that a second wave holds the shortest ones
+  const int b = p.order[blockIdx.y / p.n_heads_kv], h = blockIdx.y % p.n_heads_kv;
+  const int unit = b * p.n_heads_kv + h;
   const int64_t lo = p.off[b];
   const int n = static_cast<int>(p.off[b + 1] - lo);
   const int k = p.kept[b];

@@ -80,6 +80,7 @@ constexpr int kBlendHarmonic = 2;
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
   int32_t kept[kMaxBatch];   // k_b per document
+  int16_t order[kMaxBatch];  // documents in the order their clusters launch (longest first)
   int batch;
   int n_heads_kv;
   int head_dim;
