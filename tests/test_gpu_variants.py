@@ -500,12 +500,14 @@ def test_caller_lse_pairs_and_fallback(cuda_lib, name):
     _check_layer(w, x, out, ref)
 
 
+@pytest.mark.parametrize("n", [70000, 131072])
 @pytest.mark.parametrize("mode", sorted(BLENDS))
-def test_blend_long_document(cuda_lib, mode):
-    """The blends on a 70000-token document (two KV heads): the selection runs
-    on twelve-CTA clusters for documents of 64K tokens or more."""
+def test_blend_long_document(cuda_lib, mode, n):
+    """The blends on a long document (two KV heads): the selection runs on
+    twelve-CTA clusters for documents of 64K tokens or more, and at 131072
+    tokens (10924 per CTA) compacts in one round of 22 tokens per thread."""
     from paper_2608_03276_gb300 import binding
-    w = synth.small_variant(synth.WORKLOADS[1], [70000])
+    w = synth.small_variant(synth.WORKLOADS[1], [n])
     x = synth.make_layer(w)
     out = _run_compress(binding, w, x, flags=getattr(binding, BLENDS[mode]))
     ref = _oracle(w, x, combine_mode=mode)
