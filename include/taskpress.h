@@ -74,10 +74,21 @@ extern "C" {
 
 /* Limits. */
 #define TP_MAX_BATCH 256   /* documents per call                              */
-#define TP_MAX_ROWS 512    /* G * L_t stacked guide rows per KV head          */
-/* TP_MAX_ROWS bounds the guide: at most 512 / G tokens (128 at G = 4, 64 at
- * G = 8).  Longer guides, such as the 256- and 1024-token guides of the
- * paper's TTFT study (Sec. 4.2.3), return TP_ERR_UNSUPPORTED_SHAPE. */
+#define TP_MAX_ROWS 512    /* stacked guide rows one scoring pass holds        */
+#define TP_MAX_GUIDE_ROWS 8192 /* G * L_t stacked guide rows per KV head      */
+/* A guide of more than TP_MAX_ROWS stacked rows (more than 512 / G tokens,
+ * such as the 256- and 1024-token guides of the paper's TTFT study, Sec.
+ * 4.2.3, at G = 4) is scored in blocks of TP_MAX_ROWS rows.  A row's
+ * normaliser involves only that row, so each block runs both scoring passes on
+ * its own rows (one more pass over K per block and pass; the Eq. 2 scales come
+ * with the first block); the key scores, a sum over all rows (Eq. 1), are the
+ * blocks' fp32 sums added in block order.  The fused entry points,
+ * tp_guide_scores, tp_guide_lse and tp_guide_prefix_lse take such guides, and
+ * their workspace grows by one fp32 normaliser per guide row, document and
+ * head plus one fp32 key score per token and head.  tp_guide_key_scores and
+ * tp_guide_lse_static, which take no workspace, return
+ * TP_ERR_UNSUPPORTED_SHAPE for them, and every entry point does above
+ * TP_MAX_GUIDE_ROWS rows. */
 
 /*
  * One layer's compression problem.
@@ -191,6 +202,8 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
  * results are those of tp_guide_lse; the scratch it needs (status word,
  * counters, partial sums) lives in a fixed 2 MiB device array inside the
  * library, which every GPU that loads the library keeps until exit.
+ *  - Guides of more than TP_MAX_ROWS stacked rows return
+ *    TP_ERR_UNSUPPORTED_SHAPE (their blocks need a workspace).
  *  - Problems whose pass-1 scratch exceeds 2 MiB are rejected with
  *    TP_ERR_WORKSPACE (typical shapes need well under 1 MiB: about
  *    8 bytes x number of SMs x guide rows, plus 4 bytes per document and head).
@@ -213,7 +226,9 @@ int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const
  * tp_guide_lse or from the caller's own prefill attention), writes the
  * unpooled key score of every context token,
  *   key_scores[h, off_b + i] = (1/G) sum_r exp(sigma * q_r . k_i - lse[b, h, r]).
- * Needs no workspace.  key_scores: [H_kv, N] fp32 out.
+ * Needs no workspace.  key_scores: [H_kv, N] fp32 out.  Guides of more than
+ * TP_MAX_ROWS stacked rows return TP_ERR_UNSUPPORTED_SHAPE (their blocks need
+ * a workspace: use tp_guide_scores or a fused entry point).
  * With v ([H_kv, N, d] bf16) and gamma ([H_kv, N] fp32 out) both non-NULL, the
  * same kernel also writes the Eq. 2 scales of every token (as tp_quantize_v),
  * reading V alongside K (one CTA per key range up to 256 guide rows, two-CTA

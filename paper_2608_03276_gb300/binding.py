@@ -27,6 +27,7 @@ TP_SCORE_NORM_ADD = 0x2
 TP_SCORE_HARMONIC = 0x4
 TP_MAX_BATCH = 256
 TP_MAX_ROWS = 512
+TP_MAX_GUIDE_ROWS = 8192
 #: every symbol include/taskpress.h declares
 EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v",
            "tp_guide_scores", "tp_guide_lse", "tp_guide_lse_static", "tp_guide_key_scores",

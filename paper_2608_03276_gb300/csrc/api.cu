@@ -21,6 +21,10 @@ struct Plan {
   int hq, hkv, d, lt, g, batch;
   int64_t n_total;
   int64_t off[kMaxBatch + 1];
+  // The scoring kernels see one block of at most TP_MAX_ROWS stacked guide
+  // rows, [row0, row0 + rows) of the rows_full = G * L_t rows; a plan made by
+  // make_plan holds the first block, block_plan the others.
+  int rows_full, blocks, row0;
   int rows, nrb, rows_pad, rows_mma;
   int tiles_per_cta, grid_x;
   int32_t cta[kMaxBatch + 1];
@@ -36,8 +40,10 @@ struct Plan {
   float qmax;   // 2^(bits-1) - 1
   int32_t kept[kMaxBatch];
   int64_t cap;
-  // workspace offsets
-  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_total;
+  // workspace offsets (ws_lse holds one block's normalisers; with more than
+  // one block, ws_lse_full all of them and ws_skey_part a block's key scores)
+  size_t ws_status, ws_partials, ws_lse, ws_skey, ws_gamma, ws_keys, ws_lse_full, ws_skey_part,
+      ws_total;
 };
 
 int num_sms() {
@@ -45,6 +51,36 @@ int num_sms() {
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   return sms > 0 ? sms : 148;
+}
+
+// The row-block fields of a plan for a block of `rows` stacked guide rows:
+// 128-row blocks of pass 1, the MMA extent of pass 2, and the deepest K-tile
+// rings that fit next to the guide block.
+int set_rows(Plan* P, int rows) {
+  P->rows = rows;
+  const int rb = (rows + 127) / 128;
+  P->nrb = rb <= 1 ? 1 : (rb <= 2 ? 2 : 4);
+  P->rows_pad = 128 * P->nrb;
+  P->rows_mma = (rows + 31) / 32 * 32;
+  P->stages1 = 6;  // K ring of pass 1 (next to its V ring)
+  while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
+  P->stages2 = 4;
+  while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false) > kMaxSmem)
+    --P->stages2;
+  P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
+  // pass 1 stages the guide block, and at the end its row statistics, through
+  // its K ring
+  if (size_t(P->stages1) * (P->d / 64) * 16384 <
+      std::max(size_t(P->d / 64) * P->rows_pad * 128, size_t(4) * P->rows_pad * sizeof(float2)))
+    return TP_ERR_UNSUPPORTED_SHAPE;
+  P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false);
+  if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
+  P->stages2s = 4;
+  while (P->stages2s >= 2 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) > kMaxSmem)
+    --P->stages2s;
+  if (P->stages2s < 2) P->stages2s = 0;
+  P->smem2s = P->stages2s ? keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) : 0;
+  return TP_OK;
 }
 
 int64_t kept_for(int64_t n, double ratio, int64_t budget) {
@@ -84,12 +120,10 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   P->n_total = P->off[p->batch];
   if (P->n_total > (int64_t(1) << 31) - 256) return TP_ERR_UNSUPPORTED_SHAPE;
   const int64_t rows = int64_t(P->g) * P->lt;
-  if (rows > TP_MAX_ROWS) return TP_ERR_UNSUPPORTED_SHAPE;
-  P->rows = static_cast<int>(rows);
-  const int rb = (P->rows + 127) / 128;
-  P->nrb = rb <= 1 ? 1 : (rb <= 2 ? 2 : 4);
-  P->rows_pad = 128 * P->nrb;
-  P->rows_mma = (P->rows + 31) / 32 * 32;
+  if (rows > TP_MAX_GUIDE_ROWS) return TP_ERR_UNSUPPORTED_SHAPE;
+  P->rows_full = static_cast<int>(rows);
+  P->blocks = static_cast<int>((rows + TP_MAX_ROWS - 1) / TP_MAX_ROWS);
+  P->row0 = 0;
   const double sigma = p->softmax_scale > 0 ? double(p->softmax_scale) : 1.0 / sqrt(double(P->d));
   P->c2 = static_cast<float>(sigma * 1.4426950408889634);
   P->sigma = static_cast<float>(sigma);
@@ -118,25 +152,9 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   }
   P->grid_x = P->cta[P->batch];
 
-  // Deepest K-tile ring that fits next to the resident guide block.
-  P->stages1 = 6;  // K ring of pass 1 (next to its V ring)
-  while (P->stages1 > 1 && lse_smem_bytes(P->d, P->rows_pad, P->stages1) > kMaxSmem) --P->stages1;
-  P->stages2 = 4;
-  while (P->stages2 > 1 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false) > kMaxSmem)
-    --P->stages2;
-  P->smem1 = lse_smem_bytes(P->d, P->rows_pad, P->stages1);
-  // pass 1 stages the guide block, and at the end its row statistics, through
-  // its K ring
-  if (size_t(P->stages1) * (P->d / 64) * 16384 <
-      std::max(size_t(P->d / 64) * P->rows_pad * 128, size_t(4) * P->rows_pad * sizeof(float2)))
-    return TP_ERR_UNSUPPORTED_SHAPE;
-  P->smem2 = keyscore_smem_bytes(P->d, P->rows_pad, P->stages2, false);
-  if (P->smem1 > size_t(kMaxSmem) || P->smem2 > size_t(kMaxSmem)) return TP_ERR_UNSUPPORTED_SHAPE;
-  P->stages2s = 4;
-  while (P->stages2s >= 2 && keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) > kMaxSmem)
-    --P->stages2s;
-  if (P->stages2s < 2) P->stages2s = 0;
-  P->smem2s = P->stages2s ? keyscore_smem_bytes(P->d, P->rows_pad, P->stages2s, true) : 0;
+  // The first block of guide rows (all of them up to TP_MAX_ROWS).
+  const int st_rows = set_rows(P, static_cast<int>(std::min<int64_t>(rows, TP_MAX_ROWS)));
+  if (st_rows != TP_OK) return st_rows;
 
   P->cap = 0;
   if (need_select) {
@@ -164,6 +182,13 @@ int make_plan(const tp_problem* p, double ratio, int64_t budget, bool need_selec
   o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
   P->ws_keys = o;
   o = align_up(o + sizeof(uint32_t) * size_t(P->hkv) * P->n_total);
+  P->ws_lse_full = P->ws_skey_part = o;
+  if (P->blocks > 1) {
+    P->ws_lse_full = o;
+    o = align_up(o + sizeof(float) * size_t(P->batch) * P->hkv * P->rows_full);
+    P->ws_skey_part = o;
+    o = align_up(o + sizeof(float) * size_t(P->hkv) * P->n_total);
+  }
   P->ws_total = o;
   return TP_OK;
 }
@@ -188,13 +213,15 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 3-D bf16 view {d, rows, planes} with a {64, box_rows, 1} box, 128-byte swizzle.
+// 3-D bf16 view {d, rows, planes} with a {64, box_rows, 1} box, 128-byte
+// swizzle; consecutive planes lie plane_rows rows apart (rows by default).
 bool encode_3d(CUtensorMap* map, const void* base, int d, int64_t rows, int64_t planes,
-               int box_rows) {
+               int box_rows, int64_t plane_rows = -1) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
+  if (plane_rows < 0) plane_rows = rows;
   cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(rows), cuuint64_t(planes)};
-  cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(d) * 2 * cuuint64_t(rows)};
+  cuuint64_t strides[2] = {cuuint64_t(d) * 2, cuuint64_t(d) * 2 * cuuint64_t(plane_rows)};
   cuuint32_t box[3] = {64, cuuint32_t(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
@@ -207,10 +234,17 @@ bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15)
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? TP_OK : TP_ERR_CUDA; }
 
+// The guide rows of a plan's block: rows [row0, row0 + rows) of every
+// (document, head) group of G * L_t rows (a row offset of a multiple of
+// TP_MAX_ROWS keeps the base 16-byte aligned).
+bool encode_q(CUtensorMap* map, const Plan& P, const void* q, int box_rows) {
+  const char* base = static_cast<const char*>(q) + size_t(P.row0) * P.d * 2;
+  return encode_3d(map, base, P.d, P.rows, int64_t(P.batch) * P.hkv, box_rows, P.rows_full);
+}
+
 bool encode_maps(const Plan& P, const void* q, const void* k, CUtensorMap* tmk, CUtensorMap* tmq) {
   return encode_3d(tmk, k, P.d, P.n_total, P.hkv, 128) &&
-         encode_3d(tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv,
-                   P.rows_pad < 256 ? P.rows_pad : 256);
+         encode_q(tmq, P, q, P.rows_pad < 256 ? P.rows_pad : 256);
 }
 
 // Alignment mask of a code buffer: a thread stores 8 codes at once (8 bytes,
@@ -317,8 +351,7 @@ int run_keyscore(const Plan& P, const CUtensorMap& tmk, const void* q, const flo
   kp.skey = skey;
   kp.status = status;
   CUtensorMap tmq;
-  if (!encode_3d(&tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv, P.rows_pad < 256 ? P.rows_pad : 256))
-    return TP_ERR_CUDA;
+  if (!encode_q(&tmq, P, q, P.rows_pad < 256 ? P.rows_pad : 256)) return TP_ERR_CUDA;
   return cuda_status(
       launch_keyscore(tmk, tmk, tmq, kp, P.d, dim3(P.grid_x, P.hkv), P.smem2, dependent, s));
 }
@@ -346,7 +379,7 @@ int run_keyscore_scales(const Plan& P, const void* q, const void* k, const void*
   const int qbox = single ? (P.rows_pad < 256 ? P.rows_pad : 256) : 128;
   if (!encode_3d(&tmk, k, P.d, P.n_total, P.hkv, 128) ||
       !encode_3d(&tmv, v, P.d, P.n_total, P.hkv, 128) ||
-      !encode_3d(&tmq, q, P.d, P.rows, int64_t(P.batch) * P.hkv, qbox))
+      !encode_q(&tmq, P, q, qbox))
     return TP_ERR_CUDA;
   KeyScoreParams kp;
   memset(&kp, 0, sizeof(kp));
@@ -387,11 +420,98 @@ int run_prefix(const Plan& P, const void* q, const void* k_guide, float* lse, bo
   pp.lse = lse;
   pp.batch = P.batch;
   pp.n_heads_kv = P.hkv;
-  pp.rows = P.rows;
+  pp.rows = P.rows_full;  // the fold reads and rewrites whole rows of every block
   pp.guide_len = P.lt;
   pp.head_dim = P.d;
   pp.sigma = P.sigma;
   return cuda_status(launch_prefix(pp, dependent, s));
+}
+
+// The plan of block `blk` of the guide rows (rows blk * TP_MAX_ROWS onwards).
+int block_plan(const Plan& P, int blk, Plan* B) {
+  *B = P;
+  B->row0 = blk * TP_MAX_ROWS;
+  return set_rows(B, std::min(TP_MAX_ROWS, P.rows_full - B->row0));
+}
+
+// Columns [col0, col0 + cols) of `units` rows of floats, from rows src_pitch
+// floats apart to rows dst_pitch floats apart (device to device, in stream
+// order).
+int copy_cols(float* dst, int dst_pitch, const float* src, int src_pitch, int cols, size_t units,
+              cudaStream_t s) {
+  if (units == 0 || cols == 0) return TP_OK;
+  return cuda_status(cudaMemcpy2DAsync(dst, sizeof(float) * dst_pitch, src, sizeof(float) * src_pitch,
+                                       sizeof(float) * cols, units, cudaMemcpyDeviceToDevice, s));
+}
+
+// Scoring of a guide longer than one block of TP_MAX_ROWS stacked rows
+// (P.blocks > 1), leaving the unpooled key scores in the workspace like
+// run_scoring.  A row's normaliser involves that row alone, so every block
+// runs the passes on its own rows; the key scores (Eq. 1: a sum over all rows
+// of the group) are the blocks' sums added in block order, and the Eq. 2
+// scales come with block 0's pass over V.  Without the caller's normalisers
+// or a guide-prefix fold, block b's pass 2 follows its own pass 1.  Otherwise
+// the normalisers are first gathered into their full [batch, H_kv, M] layout
+// (the caller's, or pass 1's followed by the fold, which reads whole rows),
+// and each block's columns are copied out before its pass 2.  Launches go in
+// plain stream order.
+int run_scoring_blocks(const Plan& P, const void* q, const void* k, const void* v, float* gamma,
+                       const float* lse_in, const void* k_guide, char* ws, cudaStream_t s) {
+  float* const lse_b = reinterpret_cast<float*>(ws + P.ws_lse);
+  float* const lse_f = reinterpret_cast<float*>(ws + P.ws_lse_full);
+  float* const skey = reinterpret_cast<float*>(ws + P.ws_skey);
+  float* const part = reinterpret_cast<float*>(ws + P.ws_skey_part);
+  int* const status = reinterpret_cast<int*>(ws + P.ws_status);
+  const size_t units = size_t(P.batch) * P.hkv;
+  const int64_t nkey = int64_t(P.hkv) * P.n_total;
+  const bool gathered = lse_in || k_guide;
+  CUtensorMap tmk;
+  if (!encode_3d(&tmk, k, P.d, P.n_total, P.hkv, 128)) return TP_ERR_CUDA;
+  int st;
+  if (!lse_in) {
+    for (int blk = 0; blk < P.blocks; ++blk) {
+      Plan B;
+      if ((st = block_plan(P, blk, &B)) != TP_OK) return st;
+      CUtensorMap tmq;
+      if (!encode_q(&tmq, B, q, B.rows_pad < 256 ? B.rows_pad : 256)) return TP_ERR_CUDA;
+      if ((st = run_lse(B, tmk, tmq, q, blk == 0 ? v : nullptr, blk == 0 ? gamma : nullptr, lse_b,
+                        ws, s)) != TP_OK)
+        return st;
+      if (gathered) {
+        if ((st = copy_cols(lse_f + B.row0, P.rows_full, lse_b, B.rows, B.rows, units, s)) != TP_OK)
+          return st;
+        continue;
+      }
+      if ((st = run_keyscore(B, tmk, q, lse_b, blk == 0 ? skey : part, status, false, s)) != TP_OK)
+        return st;
+      if (blk > 0 && launch_add(skey, part, nkey, num_sms(), s) != cudaSuccess) return TP_ERR_CUDA;
+    }
+    if (!gathered) return TP_OK;
+    if (k_guide && (st = run_prefix(P, q, k_guide, lse_f, false, s)) != TP_OK) return st;
+  }
+  const float* const src = lse_in ? lse_in : lse_f;
+  for (int blk = 0; blk < P.blocks; ++blk) {
+    Plan B;
+    if ((st = block_plan(P, blk, &B)) != TP_OK) return st;
+    if ((st = copy_cols(lse_b, B.rows, src + B.row0, P.rows_full, B.rows, units, s)) != TP_OK)
+      return st;
+    float* const out = blk == 0 ? skey : part;
+    if (lse_in && blk == 0 && gamma) {
+      // the caller's normalisers: block 0's kernel also forms the scales
+      st = run_keyscore_scales(B, q, k, v, lse_b, out, gamma, status, false, s);
+      if (st == kNoFusedScales) {
+        if (launch_vquant(static_cast<const uint16_t*>(v), nullptr, gamma, nkey, P.d, P.qmax, P.bits,
+                          num_sms(), s) != cudaSuccess)
+          return TP_ERR_CUDA;
+        st = run_keyscore(B, tmk, q, lse_b, out, status, false, s);
+      }
+    } else {
+      st = run_keyscore(B, tmk, q, lse_b, out, status, false, s);
+    }
+    if (st != TP_OK) return st;
+    if (blk > 0 && launch_add(skey, part, nkey, num_sms(), s) != cudaSuccess) return TP_ERR_CUDA;
+  }
+  return TP_OK;
 }
 
 // Both scoring passes (with the Eq. 2 scales fused into the first when gamma
@@ -400,6 +520,7 @@ int run_prefix(const Plan& P, const void* q, const void* k_guide, float* lse, bo
 int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
                 cudaStream_t s, const void* k_guide = nullptr, bool dependent = false) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
+  if (P.blocks > 1) return run_scoring_blocks(P, q, k, v, gamma, nullptr, k_guide, ws, s);
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
@@ -478,6 +599,8 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
   if (!lse_in) {
     if ((st = run_scoring(P, q, k, v, g, w, s, k_guide)) != TP_OK) return st;
+  } else if (P.n_total > 0 && P.grid_x > 0 && P.blocks > 1) {
+    if ((st = run_scoring_blocks(P, q, k, v, g, lse_in, nullptr, w, s)) != TP_OK) return st;
   } else if (P.n_total > 0 && P.grid_x > 0) {
     float* const skey = reinterpret_cast<float*>(w + P.ws_skey);
     int* const status = reinterpret_cast<int*>(w + P.ws_status);
@@ -725,7 +848,21 @@ int tp_guide_lse(const tp_problem* p, const void* q, const void* k, const void* 
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
-  return run_lse(P, tmk, tmq, q, v, gamma, lse, w, s);
+  if (P.blocks == 1) return run_lse(P, tmk, tmq, q, v, gamma, lse, w, s);
+  // a long guide: block by block through the workspace into lse's columns
+  float* const lse_b = reinterpret_cast<float*>(w + P.ws_lse);
+  for (int blk = 0; blk < P.blocks; ++blk) {
+    Plan B;
+    if ((st = block_plan(P, blk, &B)) != TP_OK) return st;
+    if (!encode_q(&tmq, B, q, B.rows_pad < 256 ? B.rows_pad : 256)) return TP_ERR_CUDA;
+    if ((st = run_lse(B, tmk, tmq, q, blk == 0 ? v : nullptr, blk == 0 ? gamma : nullptr, lse_b, w,
+                      s)) != TP_OK)
+      return st;
+    if ((st = copy_cols(lse + B.row0, P.rows_full, lse_b, B.rows, B.rows, size_t(P.batch) * P.hkv,
+                        s)) != TP_OK)
+      return st;
+  }
+  return TP_OK;
 }
 
 int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const void* v,
@@ -735,6 +872,7 @@ int tp_guide_lse_static(const tp_problem* p, const void* q, const void* k, const
   if (st != TP_OK) return st;
   if (!q || !k || !lse || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
   if ((v == nullptr) != (gamma == nullptr) || (v && !aligned16(v))) return TP_ERR_INVALID_ARG;
+  if (P.blocks > 1) return TP_ERR_UNSUPPORTED_SHAPE;  // the blocks need a workspace
   // pass 1 touches the workspace only up to the end of its partial sums
   if (P.ws_lse > kStaticScratchBytes) return TP_ERR_WORKSPACE;
   char* w = nullptr;
@@ -754,6 +892,7 @@ int tp_guide_key_scores(const tp_problem* p, const void* q, const void* k, const
   if (st != TP_OK) return st;
   if (!q || !k || !lse || !key_scores || !aligned16(q) || !aligned16(k)) return TP_ERR_INVALID_ARG;
   if ((v == nullptr) != (gamma == nullptr) || (v && !aligned16(v))) return TP_ERR_INVALID_ARG;
+  if (P.blocks > 1) return TP_ERR_UNSUPPORTED_SHAPE;  // the blocks' sums need a workspace
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (v) {
@@ -929,7 +1068,10 @@ int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const*
   // reader of the scales, so one buffer of each serves every layer.  Without
   // resident pairs each layer runs the quantiser and pass 2 instead.
   for (int l = 0; l < n_layers; ++l) {
-    if (scored) {
+    if (scored && P.blocks > 1) {
+      // a long guide: plain stream order (layer l's compaction has finished)
+      if ((st = run_scoring_blocks(P, q[l], k[l], v[l], g, lse[l], nullptr, w, s)) != TP_OK) return st;
+    } else if (scored) {
       st = run_keyscore_scales(P, q[l], k[l], v[l], lse[l], skey, g, status, l > 0, s);
       if (st == kNoFusedScales) {
         if (launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, g, int64_t(P.hkv) * P.n_total,
@@ -980,10 +1122,13 @@ int tp_compress_kernel_count(const tp_problem* p, double keep_ratio, int64_t bud
   if (mode < 0 || mode > 2 || make_plan(p, keep_ratio, budget, true, &P) != TP_OK) return -1;
   int kernels = P.cap > 0 ? 2 : 1;  // selection [+ compaction]
   if (P.n_total > 0 && P.grid_x > 0) {
+    // per further block of guide rows: its passes and one addition of its key
+    // scores (the copies of normalisers between blocks are not kernels)
+    const int more = P.blocks - 1;
     if (mode == 1)  // the key scores with the scales in one kernel, else the quantiser and pass 2
-      kernels += fused_scales_fit(P) ? 1 : 2;
+      kernels += (fused_scales_fit(P) ? 1 : 2) + 2 * more;
     else
-      kernels += mode == 2 ? 3 : 2;  // pass 1, [prefix fold,] pass 2
+      kernels += (mode == 2 ? 3 : 2) + 3 * more;  // pass 1, [prefix fold,] pass 2
   }
   return kernels;
 }

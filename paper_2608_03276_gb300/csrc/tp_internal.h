@@ -163,6 +163,9 @@ cudaError_t launch_keyscore_pair(const CUtensorMap& tmk, const CUtensorMap& tmv,
 // be resident at once (0 when the device or the query refuses a two-CTA
 // cluster of that size).
 int keyscore_pair_max_clusters(int head_dim, int rows_mma, size_t smem);
+// acc[i] += x[i] for i < n (16-byte aligned buffers): the key scores of a
+// later block of guide rows added to the earlier blocks' sum.
+cudaError_t launch_add(float* acc, const float* x, int64_t n, int num_sms, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);

@@ -117,7 +117,40 @@ __global__ void __launch_bounds__(256) tp_gather_kernel(const __grid_constant__ 
   }
 }
 
+// acc[i] += x[i] over n floats: a guide longer than one scoring block adds
+// each later block's key scores to the sum of the blocks before it, in block
+// order (both buffers 16-byte aligned; a tail of n mod 4 floats one at a time).
+__global__ void __launch_bounds__(256) tp_add_kernel(float* __restrict__ acc,
+                                                     const float* __restrict__ x, int64_t n) {
+  const int64_t n4 = n >> 2;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  float4* a4 = reinterpret_cast<float4*>(acc);
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  for (int64_t i = t; i < n4; i += stride) {
+    float4 a = a4[i];
+    const float4 b = x4[i];
+    a.x += b.x;
+    a.y += b.y;
+    a.z += b.z;
+    a.w += b.w;
+    a4[i] = a;
+  }
+  for (int64_t i = (n4 << 2) + t; i < n; i += stride) acc[i] += x[i];
+}
+
 }  // namespace
+
+cudaError_t launch_add(float* acc, const float* x, int64_t n, int num_sms, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int threads = 256;
+  int64_t blocks = ((n >> 2) + threads - 1) / threads;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  tp_add_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(acc, x, n);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_vquant(const uint16_t* v, void* vq, float* gamma, int64_t rows, int head_dim,
                           float qmax, int bits, int num_sms, cudaStream_t s) {

@@ -63,12 +63,43 @@ def test_capacity_and_workspace(lib):
 
 @pytest.mark.parametrize("kw", [
     dict(head_dim=96), dict(head_dim=256), dict(pool_kernel=4), dict(pool_kernel=0), dict(pool_kernel=35),
-    dict(quant_bits=2), dict(quant_bits=16), dict(n_heads_q=7), dict(guide_len=0), dict(guide_len=65, n_heads_q=16),
+    dict(quant_bits=2), dict(quant_bits=16), dict(n_heads_q=7), dict(guide_len=0), dict(guide_len=1025, n_heads_q=16),
 ])
 def test_rejects_unsupported(lib, kw):
     p = _prob(lib, [0, 100], **kw)
     assert lib.tp_kept_capacity(p, 0.5, -1) == -1
     assert lib.tp_workspace_bytes(p, 0.5, -1) == 0
+
+
+def test_long_guide_plan(lib):
+    """More than TP_MAX_ROWS stacked guide rows run in blocks of 512: the
+    workspace adds one fp32 normaliser per row, document and head and one
+    fp32 key score per token and head; the two entry points without a
+    workspace refuse such guides before any launch; above TP_MAX_GUIDE_ROWS
+    nothing takes them.  The addresses below are never dereferenced."""
+    offs = [0, 1000, 3000]
+    shape = dict(n_heads_q=8, n_heads_kv=2, head_dim=128)
+    w512 = lib.tp_workspace_bytes(_prob(lib, offs, guide_len=128, **shape), 0.25, -1)  # M 512
+    p1024 = _prob(lib, offs, guide_len=256, **shape)                                   # M 1024
+    up = lambda b: (b + 255) // 256 * 256
+    assert lib.tp_workspace_bytes(p1024, 0.25, -1) == w512 + up(4 * 2 * 2 * 1024) + up(4 * 2 * 3000)
+    assert lib.TP_MAX_GUIDE_ROWS == 8192
+    assert lib.tp_workspace_bytes(_prob(lib, offs, guide_len=2048, **shape), 0.25, -1) > 0   # M 8192
+    assert lib.tp_workspace_bytes(_prob(lib, offs, guide_len=2049, **shape), 0.25, -1) == 0  # M 8196
+    cdll = lib.load()
+    ok = 0x10000
+    assert cdll.tp_guide_key_scores(p1024.ref(), ok, ok, None, ok, ok, None, None) == \
+        lib.TP_ERR_UNSUPPORTED_SHAPE
+    assert cdll.tp_guide_lse_static(p1024.ref(), ok, ok, None, ok, None, None) == \
+        lib.TP_ERR_UNSUPPORTED_SHAPE
+    # per further block: pass 1, pass 2 and the addition of its key scores
+    # (two-pass); pass 2 and the addition (caller's normalisers)
+    p = lib.Problem(32, 8, 128, 275, [0, 65536])  # M 1100: blocks of 512, 512, 76
+    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_TWO_PASS) == 4 + 2 * 3
+    assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_LITERAL) == 5 + 2 * 3
+    import torch
+    if not torch.cuda.is_available():
+        assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_CALLER_LSE) == 4 + 2 * 2
 
 
 def test_rejects_bad_offsets(lib):
