@@ -22,7 +22,8 @@ Also reported on the same JSON line:
   workload_legs the other workloads of the metric, each through the same
                 call: the 32K Llama layer, the 64K wide-GQA layer at its four
                 keep ratios and the ragged 8-document batch (value, hbm_fused,
-                staged kernel times);
+                staged kernel times), and the guide sweep of the paper's
+                prefill table (64K layer, 64-, 256- and 1024-token guides);
   e2e           the same metric through the public API with the inputs in
                 pinned host memory, H2D and D2H copies inside the timed region;
   cpu_baseline  the CPU oracle on every host core (a bounded sample of layer 0);
@@ -439,6 +440,55 @@ def workload_leg(binding, torch, synth, w, n_layers, args, dev, stream, hbm_peak
     return out
 
 
+def guide_sweep_leg(binding, torch, synth, args, dev, stream, tf_burst):
+    """The setting of the paper's prefill table (Sec. 4.2.3): a Llama-3-8B-shaped
+    layer (32 q / 8 KV heads, d = 128) at 64K context with 64-, 256- and
+    1024-token guides at 75% eviction (keep 25%), through tp_compress_layers
+    over two layers per step.  Guides above 512 stacked rows run in blocks of
+    512 rows; the two exact passes then cost 4 * M * n * d flops per head."""
+    base = synth.WORKLOADS[2].with_(name="llama8b-64k-guides", doc_lens=(65536,), keep_ratio=0.25)
+    out = {"workload": base.name, "n_ctx": base.n_total, "layers_per_step": 2, "keep_ratio": 0.25,
+           "heads_q": base.n_heads_q, "heads_kv": base.n_heads_kv}
+    res = {}
+    for lt in (64, 256, 1024):
+        w = base.with_(guide_len=lt)
+        L = 2
+        p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, w.doc_offsets())
+        layers = [synth.make_layer_torch(w, l, dev) for l in range(L)]
+        outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, dev, with_scores=False)
+                for _ in range(L)]
+        ws = outs[0].ws
+        for o in outs[1:]:
+            o.ws = ws
+
+        def step():
+            binding.tp_compress_layers(p, layers, w.keep_ratio, w.budget, outs, ws, stream)
+
+        with ClockSampler(dev.index or 0) as clocks:
+            for _ in range(max(args.warmup, 3)):
+                step()
+            torch.cuda.synchronize()
+            clocks.mark_start()
+            ms = time_calls(torch, step, max(args.steps, 10), 0, stream)
+            clocks.mark_end()
+        st = binding.tp_check_status(ws)
+        if st != 0:
+            raise RuntimeError(f"guide {lt}: device status {binding.tp_status_string(st)}")
+        t_layer = ms / L / 1e3
+        flops = 4.0 * w.rows * w.n_total * w.head_dim * w.n_heads_kv
+        res[f"guide_{lt}"] = {
+            "rows": w.rows, "row_blocks": -(-w.rows // binding.TP_MAX_ROWS),
+            "value": w.n_total / t_layer, "unit": UNIT, "ms_per_layer": ms / L,
+            "tensor_frac_of_burst": flops / t_layer / 1e12 / tf_burst,
+            "kernels_per_layer": binding.tp_compress_kernel_count(p, w.keep_ratio, w.budget,
+                                                                  binding.MODE_TWO_PASS),
+            "clocks": clocks.summary()}
+        del outs, ws, layers
+    out["results"] = res
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args, w):
     import numpy as np
     import torch
@@ -470,6 +520,7 @@ def run_ours(args, w):
             wl = synth.WORKLOADS[cfg]
             legs[wl.name] = workload_leg(binding, torch, synth, wl.with_(seed=replicas.rank_seed(wl.seed, rank)),
                                          nl, args, dev, stream, hbm_peak, peak_src, ratios)
+        legs["guide_sweep"] = guide_sweep_leg(binding, torch, synth, args, dev, stream, tf_burst)
     L = w.layers
     p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, w.doc_offsets())
     # each rank compresses its own stack (weak scaling; no data-path collective)
