@@ -407,8 +407,10 @@ def workload_leg(binding, torch, synth, w, n_layers, args, dev, stream, hbm_peak
     legs = {}
     for r in (keep_ratios or (w.keep_ratio,)):
         outs = [binding.CompressOutputs(p, r, w.budget, dev, with_scores=False) for _ in range(L)]
-        ws = outs[0].ws
-        for o in outs[1:]:
+        # the stack's workspace: short layers are selected several per launch
+        ws = torch.empty(binding.tp_workspace_bytes_stack(p, r, w.budget, L), dtype=torch.uint8,
+                         device=dev)
+        for o in outs:
             o.ws = ws
 
         def step():
@@ -432,6 +434,7 @@ def workload_leg(binding, torch, synth, w, n_layers, args, dev, stream, hbm_peak
             "hbm_fused": hbm_fused_of(w, kept, t_layer, hbm_peak, peak_src),
             "stages_ms": staged_times(binding, torch, p, w, layers, outs, ws, stream, 3, r),
             "kernels_per_layer": binding.tp_compress_kernel_count(p, r, w.budget, binding.MODE_TWO_PASS),
+            "layers_per_selection": binding.tp_stack_layers_per_selection(p, r, w.budget, L, ws.numel()),
             "clocks": clocks.summary()}
         del outs, ws
     out["results"] = legs

@@ -142,6 +142,36 @@ int64_t tp_kept_capacity(const tp_problem* p, double keep_ratio, int64_t budget)
 size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget);
 
 /*
+ * Workspace for tp_compress_layers / tp_compress_layers_lse over n_layers
+ * layers (0 on invalid arguments).  For documents of at most 65536 tokens it
+ * adds, for up to 7 further layers, room for one more layer's key scores,
+ * scales and selection scratch (12 bytes per token and head each); otherwise,
+ * and for one layer, it equals tp_workspace_bytes.  Given such a workspace the
+ * stack calls select several consecutive layers in one launch, as many as the
+ * workspace holds and as the device runs at once (one four-CTA cluster per
+ * layer, document and head, all resident); the product, harmonic and
+ * key-only scores only (the normalised-add score sums its norms over a
+ * cluster, so it keeps one layer per launch).  The kept sets are the exact
+ * top-k of the same scores either way, so results do not depend on the
+ * grouping.  (A selection launch is bound by latency, not bandwidth: its
+ * cluster barriers and distributed shared-memory round trips cost the same
+ * for one layer as for several.)
+ */
+size_t tp_workspace_bytes_stack(const tp_problem* p, double keep_ratio, int64_t budget,
+                                int n_layers);
+
+/*
+ * How many consecutive layers tp_compress_layers / tp_compress_layers_lse
+ * select per launch for this problem, stack depth and workspace size (a
+ * planning query: 1 when the workspace has no room for more, for documents
+ * above 65536 tokens, for the normalised-add score, or where the device's
+ * answer to the cluster co-residency query is not available); -1 on invalid
+ * arguments.  Needs the device current, as the stack calls do.
+ */
+int tp_stack_layers_per_selection(const tp_problem* p, double keep_ratio, int64_t budget,
+                                  int n_layers, size_t ws_bytes);
+
+/*
  * Eq. 2 (Sec. 3.3) for every token of V: gamma_i = max_c |v_ic| / qmax with
  * qmax = 2^(b-1) - 1 (127 or 7; fp32, IEEE round-to-nearest division) and
  * codes q_ic = clamp(rint(v_ic / gamma_i), -qmax, qmax) (IEEE fp32 quotient,
@@ -333,7 +363,9 @@ int tp_compress_layer_guide(const tp_problem* p, const void* q, const void* k, c
  * whole stack and layer l's first kernel is launched as a programmatic
  * dependent of layer l - 1's last one, so consecutive layers overlap at their
  * boundary.  Results equal n_layers calls of tp_compress_layer.  ws_bytes as
- * for tp_compress_layer (one layer's workspace serves the whole stack).
+ * for tp_compress_layer (one layer's workspace serves the whole stack), or
+ * tp_workspace_bytes_stack(p, keep_ratio, budget, n_layers) bytes, with which
+ * short layers are selected several at a time (see there).
  */
 int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
                        const void* const* k, const void* const* v, double keep_ratio,
@@ -346,10 +378,10 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
  * tp_compress_layer_lse, layer after layer, on `stream`); lse is a HOST array
  * of n_layers device pointers, each [batch, H_kv, M] fp32 (natural log).
  * Other arguments as in tp_compress_layers.  Each layer's scoring kernel is a
- * programmatic dependent of the previous layer's compaction: it loads and
- * scores at once and waits for that kernel only before its first store.
- * Results equal n_layers calls of tp_compress_layer_lse bit for bit.
- * ws_bytes as for tp_compress_layer.
+ * programmatic dependent of the kernel before it: it loads and scores at once
+ * and waits for that kernel only before its first store.  Results equal
+ * n_layers calls of tp_compress_layer_lse bit for bit.  ws_bytes as for
+ * tp_compress_layers (tp_workspace_bytes or tp_workspace_bytes_stack).
  */
 int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const* q,
                            const void* const* k, const void* const* v, const float* const* lse,

@@ -35,7 +35,7 @@ EXPORTS = ("tp_budget", "tp_kept_capacity", "tp_workspace_bytes", "tp_quantize_v
            "tp_compress_layer", "tp_compress_layer_lse", "tp_guide_prefix_lse",
            "tp_compress_layer_guide", "tp_compress_layers", "tp_quantize_rows", "tp_check_status",
            "tp_selftest_wait_timeout", "tp_status_string", "tp_compress_kernel_count",
-           "tp_compress_layers_lse")
+           "tp_compress_layers_lse", "tp_workspace_bytes_stack", "tp_stack_layers_per_selection")
 
 
 class TpProblem(ctypes.Structure):
@@ -77,6 +77,10 @@ def load(path: Optional[str] = None):
     lib.tp_kept_capacity.argtypes = [POINTER(TpProblem), c_double, c_int64]
     lib.tp_workspace_bytes.restype = c_size_t
     lib.tp_workspace_bytes.argtypes = [POINTER(TpProblem), c_double, c_int64]
+    lib.tp_workspace_bytes_stack.restype = c_size_t
+    lib.tp_workspace_bytes_stack.argtypes = [POINTER(TpProblem), c_double, c_int64, c_int]
+    lib.tp_stack_layers_per_selection.restype = c_int
+    lib.tp_stack_layers_per_selection.argtypes = [POINTER(TpProblem), c_double, c_int64, c_int, c_size_t]
     lib.tp_quantize_v.restype = c_int
     lib.tp_quantize_v.argtypes = [POINTER(TpProblem), c_void_p, c_void_p, c_void_p, c_void_p]
     lib.tp_guide_scores.restype = c_int
@@ -211,6 +215,18 @@ def tp_kept_capacity(p: Problem, keep_ratio: float, budget: int) -> int:
 
 def tp_workspace_bytes(p: Problem, keep_ratio: float = 0.0, budget: int = 0) -> int:
     return int(load().tp_workspace_bytes(p.ref(), keep_ratio, budget))
+
+
+def tp_workspace_bytes_stack(p: Problem, keep_ratio: float, budget: int, n_layers: int) -> int:
+    return int(load().tp_workspace_bytes_stack(p.ref(), keep_ratio, budget, n_layers))
+
+
+def tp_stack_layers_per_selection(p: Problem, keep_ratio: float, budget: int, n_layers: int,
+                                  ws_bytes: int) -> int:
+    n = int(load().tp_stack_layers_per_selection(p.ref(), keep_ratio, budget, n_layers, ws_bytes))
+    if n < 0:
+        raise TaskPressError("tp_stack_layers_per_selection", TP_ERR_INVALID_ARG)
+    return n
 
 
 def tp_quantize_v(p: Problem, v, vq, gamma, stream=None):

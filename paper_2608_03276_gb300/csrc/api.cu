@@ -456,10 +456,11 @@ int copy_cols(float* dst, int dst_pitch, const float* src, int src_pitch, int co
 // and each block's columns are copied out before its pass 2.  Launches go in
 // plain stream order.
 int run_scoring_blocks(const Plan& P, const void* q, const void* k, const void* v, float* gamma,
-                       const float* lse_in, const void* k_guide, char* ws, cudaStream_t s) {
+                       const float* lse_in, const void* k_guide, char* ws, cudaStream_t s,
+                       float* skey_out = nullptr) {
   float* const lse_b = reinterpret_cast<float*>(ws + P.ws_lse);
   float* const lse_f = reinterpret_cast<float*>(ws + P.ws_lse_full);
-  float* const skey = reinterpret_cast<float*>(ws + P.ws_skey);
+  float* const skey = skey_out ? skey_out : reinterpret_cast<float*>(ws + P.ws_skey);
   float* const part = reinterpret_cast<float*>(ws + P.ws_skey_part);
   int* const status = reinterpret_cast<int*>(ws + P.ws_status);
   const size_t units = size_t(P.batch) * P.hkv;
@@ -516,19 +517,68 @@ int run_scoring_blocks(const Plan& P, const void* q, const void* k, const void* 
 
 // Both scoring passes (with the Eq. 2 scales fused into the first when gamma
 // is given, and the guide prefix folded into the normalisers between them when
-// k_guide is given); leaves the unpooled key scores in the workspace.
+// k_guide is given); leaves the unpooled key scores in the workspace (or in
+// skey_out).
 int run_scoring(const Plan& P, const void* q, const void* k, const void* v, float* gamma, char* ws,
-                cudaStream_t s, const void* k_guide = nullptr, bool dependent = false) {
+                cudaStream_t s, const void* k_guide = nullptr, bool dependent = false,
+                float* skey_out = nullptr) {
   if (P.n_total == 0 || P.grid_x == 0) return TP_OK;
-  if (P.blocks > 1) return run_scoring_blocks(P, q, k, v, gamma, nullptr, k_guide, ws, s);
+  if (P.blocks > 1) return run_scoring_blocks(P, q, k, v, gamma, nullptr, k_guide, ws, s, skey_out);
   CUtensorMap tmk, tmq;
   if (!encode_maps(P, q, k, &tmk, &tmq)) return TP_ERR_CUDA;
   float* lse = reinterpret_cast<float*>(ws + P.ws_lse);
   int st = run_lse(P, tmk, tmq, q, v, gamma, lse, ws, s, dependent);
   if (st != TP_OK) return st;
   if (k_guide && (st = run_prefix(P, q, k_guide, lse, true, s)) != TP_OK) return st;
-  return run_keyscore(P, tmk, q, lse, reinterpret_cast<float*>(ws + P.ws_skey),
+  return run_keyscore(P, tmk, q, lse, skey_out ? skey_out : reinterpret_cast<float*>(ws + P.ws_skey),
                       reinterpret_cast<int*>(ws + P.ws_status), true, s);
+}
+
+// Stacks of layers of short documents select several layers in one launch
+// when the caller's workspace holds their key scores, scales and key scratch
+// side by side (tp_workspace_bytes_stack): slot 0 is the plan's own regions,
+// slots 1.. follow the plan's workspace.
+constexpr int64_t kMergeMaxTokens = 65536;  // four-CTA slices stay in shared memory
+
+int64_t max_doc_len(const Plan& P) {
+  int64_t m = 0;
+  for (int b = 0; b < P.batch; ++b) m = std::max(m, P.off[b + 1] - P.off[b]);
+  return m;
+}
+
+int stack_slots(const Plan& P, int n_layers) {
+  if (n_layers < 2 || max_doc_len(P) > kMergeMaxTokens) return 1;
+  return std::min(n_layers, kMaxSelectLayers);
+}
+
+size_t slot_bytes(const Plan& P) { return 3 * align_up(sizeof(float) * size_t(P.hkv) * P.n_total); }
+
+struct Slot {
+  float* skey;
+  float* gamma;
+  uint32_t* keys;
+};
+
+Slot stack_slot(const Plan& P, char* ws, int i) {
+  if (i == 0)
+    return {reinterpret_cast<float*>(ws + P.ws_skey), reinterpret_cast<float*>(ws + P.ws_gamma),
+            reinterpret_cast<uint32_t*>(ws + P.ws_keys)};
+  const size_t a = align_up(sizeof(float) * size_t(P.hkv) * P.n_total);
+  char* base = ws + P.ws_total + size_t(i - 1) * slot_bytes(P);
+  return {reinterpret_cast<float*>(base), reinterpret_cast<float*>(base + a),
+          reinterpret_cast<uint32_t*>(base + 2 * a)};
+}
+
+// Layers per selection launch for a stack: as many as the workspace holds
+// slots for and as fit in one wave of four-CTA selection clusters; 1 for the
+// normalised-add score (its per-document norms are summed over a cluster, so
+// the cluster size must not change with the grouping).
+int stack_group(const Plan& P, uint32_t flags, int n_layers, size_t ws_bytes) {
+  int g = stack_slots(P, n_layers);
+  if (g < 2 || (flags & TP_SCORE_NORM_ADD)) return 1;
+  while (g > 1 && P.ws_total + size_t(g - 1) * slot_bytes(P) > ws_bytes) --g;
+  if (g < 2) return 1;
+  return std::min(g, select_merge_layers(P.batch * P.hkv, max_doc_len(P)));
 }
 
 int blend_of(uint32_t flags) {
@@ -638,6 +688,51 @@ int compress_layer(const tp_problem* p, const void* q, const void* k, const void
   gp.vqc = vqc;
   gp.gammac = gammac;
   return cuda_status(launch_gather(gp, true, s));
+}
+
+// The selection of layers l0 .. l0 + gl - 1 of a stack (one launch; their key
+// scores and scales in slots 0 .. gl - 1) and their compactions, each a
+// programmatic dependent of the kernel before it.
+int stack_tail(const Plan& P, const tp_problem* p, int l0, int gl, const void* const* k,
+               const void* const* v, int32_t* const* idx, void* const* kc, void* const* vc,
+               int8_t* const* vqc, float* const* gammac, char* w, cudaStream_t s) {
+  SelectParams sp;
+  fill_select(P, w, &sp);
+  sp.pool_kernel = p->pool_kernel;
+  sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
+  sp.blend = blend_of(p->flags);
+  const Slot s0 = stack_slot(P, w, 0);
+  sp.skey = s0.skey;
+  sp.gamma = s0.gamma;
+  sp.idx = idx ? idx[l0] : nullptr;
+  if (gl > 1) {
+    sp.layers = gl;
+    for (int i = 0; i < gl; ++i) {
+      const Slot sl = stack_slot(P, w, i);
+      sp.skey_l[i] = sl.skey;
+      sp.gamma_l[i] = sl.gamma;
+      sp.keys_l[i] = sl.keys;
+      sp.idx_l[i] = idx ? idx[l0 + i] : nullptr;
+    }
+  }
+  if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
+  if (P.cap == 0) return TP_OK;
+  for (int i = 0; i < gl; ++i) {
+    const int l = l0 + i;
+    GatherParams gp;
+    fill_gather(P, &gp);
+    gp.k = static_cast<const uint16_t*>(k[l]);
+    gp.v = static_cast<const uint16_t*>(v[l]);
+    gp.gamma = stack_slot(P, w, i).gamma;
+    gp.idx = idx[l];
+    gp.kc = kc ? static_cast<uint16_t*>(kc[l]) : nullptr;
+    gp.vc = vc ? static_cast<uint16_t*>(vc[l]) : nullptr;
+    gp.vqc = vqc ? vqc[l] : nullptr;
+    gp.gammac = gammac ? gammac[l] : nullptr;
+    const int st = cuda_status(launch_gather(gp, true, s));
+    if (st != TP_OK) return st;
+  }
+  return TP_OK;
 }
 
 }  // namespace
@@ -781,6 +876,20 @@ size_t tp_workspace_bytes(const tp_problem* p, double keep_ratio, int64_t budget
   const bool sel = budget >= 0 || (keep_ratio >= 0.0 && keep_ratio <= 1.0);
   if (make_plan(p, keep_ratio, budget, sel, &P) != TP_OK) return 0;
   return P.ws_total;
+}
+
+size_t tp_workspace_bytes_stack(const tp_problem* p, double keep_ratio, int64_t budget, int n_layers) {
+  Plan P;
+  const bool sel = budget >= 0 || (keep_ratio >= 0.0 && keep_ratio <= 1.0);
+  if (n_layers < 0 || make_plan(p, keep_ratio, budget, sel, &P) != TP_OK) return 0;
+  return P.ws_total + size_t(stack_slots(P, n_layers) - 1) * slot_bytes(P);
+}
+
+int tp_stack_layers_per_selection(const tp_problem* p, double keep_ratio, int64_t budget,
+                                  int n_layers, size_t ws_bytes) {
+  Plan P;
+  if (n_layers < 1 || make_plan(p, keep_ratio, budget, true, &P) != TP_OK) return -1;
+  return stack_group(P, p->flags, n_layers, ws_bytes);
 }
 
 int tp_quantize_v(const tp_problem* p, const void* v, int8_t* vq, float* gamma, void* stream) {
@@ -998,34 +1107,21 @@ int tp_compress_layers(const tp_problem* p, int n_layers, const void* const* q,
   if (n_layers == 0) return TP_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  float* g = reinterpret_cast<float*>(w + P.ws_gamma);
   // one reset for the whole stack: pass 1 leaves its counters zero again
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
-  for (int l = 0; l < n_layers; ++l) {
-    // layer l's pass 1 is a dependent of layer l - 1's compaction (or of its
-    // selection when nothing is kept): its prologue overlaps that kernel's tail
-    if ((st = run_scoring(P, q[l], k[l], v[l], g, w, s, nullptr, l > 0)) != TP_OK) return st;
-    SelectParams sp;
-    fill_select(P, w, &sp);
-    sp.pool_kernel = p->pool_kernel;
-    sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
-    sp.blend = blend_of(p->flags);
-    sp.skey = reinterpret_cast<const float*>(w + P.ws_skey);
-    sp.gamma = g;
-    sp.idx = idx ? idx[l] : nullptr;
-    if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
-    if (P.cap == 0) continue;
-    GatherParams gp;
-    fill_gather(P, &gp);
-    gp.k = static_cast<const uint16_t*>(k[l]);
-    gp.v = static_cast<const uint16_t*>(v[l]);
-    gp.gamma = g;
-    gp.idx = idx[l];
-    gp.kc = kc ? static_cast<uint16_t*>(kc[l]) : nullptr;
-    gp.vc = vc ? static_cast<uint16_t*>(vc[l]) : nullptr;
-    gp.vqc = vqc ? vqc[l] : nullptr;
-    gp.gammac = gammac ? gammac[l] : nullptr;
-    if ((st = cuda_status(launch_gather(gp, true, s))) != TP_OK) return st;
+  const int group = stack_group(P, p->flags, n_layers, ws_bytes);
+  for (int l0 = 0; l0 < n_layers; l0 += group) {
+    const int gl = std::min(group, n_layers - l0);
+    for (int i = 0; i < gl; ++i) {
+      // each layer's pass 1 is a dependent of the kernel before it (the
+      // previous layer's pass 2, compaction or selection): its prologue
+      // overlaps that kernel's tail, and it waits for it before its first store
+      const Slot sl = stack_slot(P, w, i);
+      const int l = l0 + i;
+      if ((st = run_scoring(P, q[l], k[l], v[l], sl.gamma, w, s, nullptr, l > 0, sl.skey)) != TP_OK)
+        return st;
+    }
+    if ((st = stack_tail(P, p, l0, gl, k, v, idx, kc, vc, vqc, gammac, w, s)) != TP_OK) return st;
   }
   return TP_OK;
 }
@@ -1054,56 +1150,42 @@ int tp_compress_layers_lse(const tp_problem* p, int n_layers, const void* const*
   if (n_layers == 0) return TP_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  float* const g = reinterpret_cast<float*>(w + P.ws_gamma);
-  float* const skey = reinterpret_cast<float*>(w + P.ws_skey);
   int* const status = reinterpret_cast<int*>(w + P.ws_status);
   const bool scored = P.n_total > 0 && P.grid_x > 0;
   if ((st = zero_head(P, w, s)) != TP_OK) return st;
   // Per layer: the key scores with the Eq. 2 scales (one kernel on CTA pairs),
-  // the selection, the compaction, each a programmatic dependent of the
-  // kernel before it.  Layer l + 1's scoring kernel loads and scores while
-  // layer l's compaction finishes and waits for it only before its first
-  // store; that compaction completes after layer l's selection (it waited for
-  // it), which was the last reader of the key scores, and is itself the last
-  // reader of the scales, so one buffer of each serves every layer.  Without
-  // resident pairs each layer runs the quantiser and pass 2 instead.
-  for (int l = 0; l < n_layers; ++l) {
-    if (scored && P.blocks > 1) {
-      // a long guide: plain stream order (layer l's compaction has finished)
-      if ((st = run_scoring_blocks(P, q[l], k[l], v[l], g, lse[l], nullptr, w, s)) != TP_OK) return st;
-    } else if (scored) {
-      st = run_keyscore_scales(P, q[l], k[l], v[l], lse[l], skey, g, status, l > 0, s);
+  // then the selection and the compaction, each a programmatic dependent of
+  // the kernel before it.  A layer's scoring kernel loads and scores while the
+  // kernel before it finishes and waits for it only before its first store;
+  // the compaction completes after its selection (it waited for it), which
+  // was the last reader of the key scores, and is itself the last reader of
+  // the scales, so one buffer of each serves every group of layers.  Without
+  // resident pairs a layer runs the quantiser and pass 2 instead.
+  const int group = stack_group(P, p->flags, n_layers, ws_bytes);
+  for (int l0 = 0; l0 < n_layers; l0 += group) {
+    const int gl = std::min(group, n_layers - l0);
+    for (int i = 0; scored && i < gl; ++i) {
+      const Slot sl = stack_slot(P, w, i);
+      const int l = l0 + i;
+      if (P.blocks > 1) {
+        // a long guide: plain stream order
+        if ((st = run_scoring_blocks(P, q[l], k[l], v[l], sl.gamma, lse[l], nullptr, w, s, sl.skey)) !=
+            TP_OK)
+          return st;
+        continue;
+      }
+      st = run_keyscore_scales(P, q[l], k[l], v[l], lse[l], sl.skey, sl.gamma, status, l > 0, s);
       if (st == kNoFusedScales) {
-        if (launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, g, int64_t(P.hkv) * P.n_total,
-                          P.d, P.qmax, P.bits, num_sms(), s) != cudaSuccess)
+        if (launch_vquant(static_cast<const uint16_t*>(v[l]), nullptr, sl.gamma,
+                          int64_t(P.hkv) * P.n_total, P.d, P.qmax, P.bits, num_sms(), s) != cudaSuccess)
           return TP_ERR_CUDA;
         CUtensorMap tmk, tmq;
         if (!encode_maps(P, q[l], k[l], &tmk, &tmq)) return TP_ERR_CUDA;
-        st = run_keyscore(P, tmk, q[l], lse[l], skey, status, true, s);
+        st = run_keyscore(P, tmk, q[l], lse[l], sl.skey, status, true, s);
       }
       if (st != TP_OK) return st;
     }
-    SelectParams sp;
-    fill_select(P, w, &sp);
-    sp.pool_kernel = p->pool_kernel;
-    sp.key_only = (p->flags & TP_SCORE_KEY_ONLY) ? 1 : 0;
-    sp.blend = blend_of(p->flags);
-    sp.skey = skey;
-    sp.gamma = g;
-    sp.idx = idx ? idx[l] : nullptr;
-    if (launch_select(sp, true, s) != cudaSuccess) return TP_ERR_CUDA;
-    if (P.cap == 0) continue;
-    GatherParams gp;
-    fill_gather(P, &gp);
-    gp.k = static_cast<const uint16_t*>(k[l]);
-    gp.v = static_cast<const uint16_t*>(v[l]);
-    gp.gamma = g;
-    gp.idx = idx[l];
-    gp.kc = kc ? static_cast<uint16_t*>(kc[l]) : nullptr;
-    gp.vc = vc ? static_cast<uint16_t*>(vc[l]) : nullptr;
-    gp.vqc = vqc ? vqc[l] : nullptr;
-    gp.gammac = gammac ? gammac[l] : nullptr;
-    if ((st = cuda_status(launch_gather(gp, true, s))) != TP_OK) return st;
+    if ((st = stack_tail(P, p, l0, gl, k, v, idx, kc, vc, vqc, gammac, w, s)) != TP_OK) return st;
   }
   return TP_OK;
 }

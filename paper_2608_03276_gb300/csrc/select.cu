@@ -183,8 +183,17 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   const int rank = static_cast<int>(cluster.block_rank());
   // clusters launch in blockIdx.y order: the longest documents' units first,
   // so that a second wave holds the shortest ones
-  const int b = p.order[blockIdx.y / p.n_heads_kv], h = blockIdx.y % p.n_heads_kv;
+  // with several layers in one launch, units are layer-major
+  const int per_layer = p.batch * p.n_heads_kv;
+  const int layer = static_cast<int>(blockIdx.y) / per_layer;
+  const int yl = static_cast<int>(blockIdx.y) - layer * per_layer;
+  const int b = p.order[yl / p.n_heads_kv], h = yl % p.n_heads_kv;
   const int unit = b * p.n_heads_kv + h;
+  const bool merged = p.layers > 1;
+  const float* const skey_in = merged ? p.skey_l[layer] : p.skey;
+  const float* const gamma_in = merged ? p.gamma_l[layer] : p.gamma;
+  uint32_t* const keys_g = merged ? p.keys_l[layer] : p.keys;
+  int32_t* const idx_out = merged ? p.idx_l[layer] : p.idx;
   const int64_t lo = p.off[b];
   const int n = static_cast<int>(p.off[b + 1] - lo);
   const int k = p.kept[b];
@@ -194,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   const int s0 = min(rank * per_cta, n), s1 = min(s0 + per_cta, n);
   // the slice's keys: in shared memory when they fit, else in the global scratch
   const bool in_smem = (s1 - s0 <= kSliceKeys);
-  uint32_t* const keys_base = in_smem ? sm.keys : p.keys + row;
+  uint32_t* const keys_base = in_smem ? sm.keys : keys_g + row;
   // key of token i: keys_base[kpos(i)].  In shared memory every 16 keys are
   // followed by a padding word, so the compaction's runs of 16 consecutive
   // keys per thread start 17 words apart and its reads hit distinct banks.
@@ -226,12 +235,12 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
       // memory (cp.async, 16-byte groups where aligned): the key scores with
       // their halo and the scales (or given scores).  Halo positions outside
       // the document are zero.  One global round trip per sub-slice.
-      const float* vsrc = p.scores_in ? p.scores_in : (p.key_only ? nullptr : p.gamma);
+      const float* vsrc = p.scores_in ? p.scores_in : (p.key_only ? nullptr : gamma_in);
       const int64_t g0 = static_cast<int64_t>(row);  // global index of token 0
       const int64_t sref = (g0 + c0 - half) & ~int64_t(3), vref = (g0 + c0) & ~int64_t(3);
       if (fused) {
         const int ia = max(c0 - half, 0), ib = min(c1 + half, n);  // halo inside the document
-        stage_floats(sm.strip, p.skey, g0 + ia, g0 + ib, sref);
+        stage_floats(sm.strip, skey_in, g0 + ia, g0 + ib, sref);
         for (int i = c0 - half + static_cast<int>(threadIdx.x); i < c1 + half; i += kThreads)
           if (i < ia || i >= ib) sm.strip[g0 + i - sref] = 0.f;
       }
@@ -309,7 +318,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
   const int64_t unit_slot0 = static_cast<int64_t>(unit) * p.cap;
   const int kk = max(0, min(k, n));
   if (rank == 0)
-    for (int64_t t = kk + threadIdx.x; t < p.cap; t += kThreads) p.idx[unit_slot0 + t] = -1;
+    for (int64_t t = kk + threadIdx.x; t < p.cap; t += kThreads) idx_out[unit_slot0 + t] = -1;
   cluster.sync();  // histograms of phase A complete everywhere
 
   uint32_t thr = 0;
@@ -426,7 +435,7 @@ __global__ void __launch_bounds__(kThreads, 1) tp_select_kernel(const __grid_con
       const bool is_eq = !is_gt && kv[e] == thr;
       if (is_gt || (is_eq && eq_rank < need_eq)) {
         const int slot = gt_rank + (need_eq < 0 ? 0 : min(eq_rank, need_eq));
-        p.idx[unit_slot0 + slot] = j;
+        idx_out[unit_slot0 + slot] = j;
       }
       gt_rank += is_gt;
       eq_rank += is_eq;
@@ -521,8 +530,9 @@ int select_max_clusters(size_t smem, int slot) {
 }
 
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s) {
-  const int units = p.batch * p.n_heads_kv;
+  const int units = p.batch * p.n_heads_kv * (p.layers > 1 ? p.layers : 1);
   if (units <= 0) return cudaSuccess;
+  if (p.layers > kMaxSelectLayers) return cudaErrorInvalidValue;
   if (p.pool_kernel / 2 > kMaxHalf) return cudaErrorInvalidValue;
   const size_t smem = sizeof(SelectSmem);
   int dev = 0, sms = 148;
@@ -542,10 +552,21 @@ cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s)
     if (per_cta > 16 * kThreads) return launch_select_blend<12, 22>(p, units, smem, dependent, s, 56);
     return launch_select_blend<12>(p, units, smem, dependent, s, 21);
   }
+  // Several layers in one launch: four-CTA clusters, which the caller checked
+  // are all resident at once (select_merge_layers).
+  if (p.layers > 1 && (n_max + 3) / 4 <= kSliceKeys)
+    return launch_select_blend<4>(p, units, smem, dependent, s, 12);
   // Fewer, larger slices when eight CTAs per unit would need more than one wave.
   if (units * 8 > sms && (n_max + 3) / 4 <= kSliceKeys)
     return launch_select_blend<4>(p, units, smem, dependent, s, 12);
   return launch_select_blend<8>(p, units, smem, dependent, s, 15);
+}
+
+int select_merge_layers(int units_per_layer, int64_t n_max) {
+  if (units_per_layer <= 0 || (n_max + 3) / 4 > kSliceKeys) return 1;
+  const int clusters = select_max_clusters<4>(sizeof(SelectSmem), 12);
+  const int layers = clusters / units_per_layer;
+  return layers < 1 ? 1 : (layers > kMaxSelectLayers ? kMaxSelectLayers : layers);
 }
 
 }  // namespace tp

@@ -77,6 +77,9 @@ constexpr int kBlendProduct = 0;
 constexpr int kBlendNormAdd = 1;
 constexpr int kBlendHarmonic = 2;
 
+// Layers one selection launch may take at once (a stack of short documents).
+constexpr int kMaxSelectLayers = 8;
+
 struct SelectParams {
   int64_t off[kMaxBatch + 1];
   int32_t kept[kMaxBatch];   // k_b per document
@@ -96,6 +99,16 @@ struct SelectParams {
   float* scores_out;         // optional combined scores out (fused path)
   uint32_t* keys;            // [H_kv, N] scratch
   int32_t* idx;              // [batch, H_kv, cap]
+  // layers > 1: the selections of that many layers of one problem in one
+  // launch (units layer-major), each layer with its own key scores, scales,
+  // key scratch and kept indices; skey, gamma, keys and idx above are then
+  // unused.  Only the fused path with the product, harmonic or key-only score
+  // merges layers, and never with scores_in / scores_out.
+  int layers;
+  const float* skey_l[kMaxSelectLayers];
+  const float* gamma_l[kMaxSelectLayers];
+  uint32_t* keys_l[kMaxSelectLayers];
+  int32_t* idx_l[kMaxSelectLayers];
 };
 
 struct GatherParams {
@@ -167,6 +180,12 @@ int keyscore_pair_max_clusters(int head_dim, int rows_mma, size_t smem);
 // later block of guide rows added to the earlier blocks' sum.
 cudaError_t launch_add(float* acc, const float* x, int64_t n, int num_sms, cudaStream_t s);
 cudaError_t launch_select(const SelectParams& p, bool dependent, cudaStream_t s);
+// How many layers of a problem with `units_per_layer` (document, head) units
+// and documents of at most n_max tokens one selection launch can take with
+// every cluster resident at once and every slice in shared memory (four-CTA
+// clusters); 1 when merging layers would not fit (or the device is not asked:
+// no GPU, or the query is refused).
+int select_merge_layers(int units_per_layer, int64_t n_max);
 cudaError_t launch_gather(const GatherParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_prefix(const PrefixParams& p, bool dependent, cudaStream_t s);
 cudaError_t launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);

@@ -29,7 +29,7 @@ def declared_symbols():
 
 def test_exports_every_declared_symbol(lib):
     names = declared_symbols()
-    assert len(names) == 21, names
+    assert len(names) == 23, names
     assert sorted(lib.EXPORTS) == names
     cdll = lib.load()
     for n in names:
@@ -100,6 +100,33 @@ def test_long_guide_plan(lib):
     import torch
     if not torch.cuda.is_available():
         assert lib.tp_compress_kernel_count(p, 0.1, -1, lib.MODE_CALLER_LSE) == 4 + 2 * 2
+
+
+def test_stack_workspace(lib):
+    """tp_workspace_bytes_stack adds, for documents of at most 65536 tokens and
+    up to 7 further layers, one more layer's key scores, scales and selection
+    scratch (3 x 4 bytes per token and head, each array 256-byte aligned);
+    above 65536 tokens, or for one layer, it is tp_workspace_bytes.  The
+    grouping query answers 1 where the workspace has no room, for the
+    normalised-add score, and without a device to ask."""
+    offs = [0, 1000, 3000]
+    p = _prob(lib, offs)
+    base = lib.tp_workspace_bytes(p, 0.25, -1)
+    slot = 3 * ((4 * 2 * 3000 + 255) // 256 * 256)
+    assert lib.tp_workspace_bytes_stack(p, 0.25, -1, 1) == base
+    assert lib.tp_workspace_bytes_stack(p, 0.25, -1, 4) == base + 3 * slot
+    assert lib.tp_workspace_bytes_stack(p, 0.25, -1, 40) == base + 7 * slot
+    long_doc = _prob(lib, [0, 65537])
+    assert lib.tp_workspace_bytes_stack(long_doc, 0.25, -1, 4) == lib.tp_workspace_bytes(long_doc, 0.25, -1)
+    assert lib.load().tp_workspace_bytes_stack(p.ref(), 0.25, -1, -1) == 0
+    assert lib.tp_stack_layers_per_selection(p, 0.25, -1, 4, base) == 1
+    nadd = _prob(lib, offs, flags=lib.TP_SCORE_NORM_ADD)
+    assert lib.tp_stack_layers_per_selection(nadd, 0.25, -1, 4, base + 3 * slot) == 1
+    import torch
+    if not torch.cuda.is_available():
+        assert lib.tp_stack_layers_per_selection(p, 0.25, -1, 4, base + 3 * slot) == 1
+    with pytest.raises(lib.TaskPressError):
+        lib.tp_stack_layers_per_selection(p, 0.25, -1, 0, base)
 
 
 def test_rejects_bad_offsets(lib):

@@ -294,6 +294,52 @@ def test_lse_stack_matches_single_layers(cuda_lib, name, bits, nl):
                      bits=bits)
 
 
+GROUPED = [("c2-llama-4133", None, 6, 4), ("c1-tiny-2k", "harmonic", 9, 8),
+           ("c2-llama-4133", "key_only", 3, 3), ("c2-llama-4133", "normadd", 3, 1),
+           ("c5-ragged", None, 3, 1)]
+
+
+@pytest.mark.parametrize("name,mode,nl,group", GROUPED)
+def test_stack_grouped_selection(cuda_lib, name, mode, nl, group):
+    """With a tp_workspace_bytes_stack workspace the stacks select several
+    layers per launch (four-CTA clusters, all resident): 8 units per layer on
+    a 152-SM GB300 give groups of 4, 2 units groups of 8 (the last group of
+    one layer), the ragged batch's 40 units no grouping, the normalised-add
+    score none.  Both stacks equal one call per layer bit for bit, and the
+    oracle on every layer."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = SMALL[name]
+    flags = {None: 0, "harmonic": binding.TP_SCORE_HARMONIC, "normadd": binding.TP_SCORE_NORM_ADD,
+             "key_only": binding.TP_SCORE_KEY_ONLY}[mode]
+    xs = _stack(w, nl)
+    p = _problem(binding, w, xs[0].doc_offsets, flags=flags)
+    ws = torch.empty(binding.tp_workspace_bytes_stack(p, w.keep_ratio, w.budget, nl), dtype=torch.uint8,
+                     device="cuda")
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    got = binding.tp_stack_layers_per_selection(p, w.keep_ratio, w.budget, nl, ws.numel())
+    if sms == 152:
+        assert got == group, (got, group)
+    dev = [tuple(parity.to_device_bf16(t) for t in (x.q, x.k, x.v)) for x in xs]
+    lses = [torch.tensor(_context_lse(w, x), device="cuda") for x in xs]
+    for caller_lse in (False, True):
+        outs = [binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda") for _ in xs]
+        if caller_lse:
+            binding.tp_compress_layers_lse(p, dev, lses, w.keep_ratio, w.budget, outs, ws)
+        else:
+            binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, ws)
+        assert binding.tp_check_status(ws) == 0
+        for l, x in enumerate(xs):
+            single = binding.CompressOutputs(p, w.keep_ratio, w.budget, "cuda")
+            binding.compress(p, *dev[l], w.keep_ratio, w.budget, single,
+                             lse=lses[l] if caller_lse else None)
+            _outputs_equal(outs[l], single, f"layer {l} (caller lse {caller_lse})")
+            if not caller_lse:
+                ref = _oracle(w, x, combine_mode=mode) if mode in BLENDS else \
+                    _oracle(w, x, key_only=mode == "key_only")
+                _check_layer(w, x, single, ref, key_only=mode == "key_only")
+
+
 def test_full_size_lse_stack(cuda_lib):
     """Three 128K layers through tp_compress_layers_lse, the benchmark's
     caller-normaliser leg: each equals a single tp_compress_layer_lse call bit
