@@ -121,6 +121,27 @@ def pin_key_scores_total_mass(O):
         assert abs(s.sum() - lt) <= 1e-11 * max(1, lt), (s.sum(), lt)
 
 
+def pin_rows_independent_and_additive(O):
+    """Each guide row's normaliser involves that row alone, and the key score
+    is additive over rows: the normalisers of any block of rows equal the
+    whole set's for those rows, and the per-head score of a group is the
+    mean of its heads' scores, each head's a sum over its own rows.  (A
+    guide longer than one scoring block is scored block by block on these two
+    facts.)"""
+    for seed, (g, lt, n, d) in enumerate([(4, 7, 40, 8), (3, 5, 23, 16)]):
+        q = _rand(seed, (g, lt, d)) * 2
+        k = _rand(seed + 11, (n, d))
+        rows = q.reshape(g * lt, d)
+        whole = O.guide_lse(rows, k, 0.35)
+        for a, b in [(0, 1), (3, g * lt), (5, 11)]:
+            part = O.guide_lse(rows[a:b], k, 0.35)
+            assert np.allclose(part, whole[a:b], rtol=0, atol=1e-12), (a, b)
+        heads = [O.key_scores(q[i:i + 1], k, 0.35) for i in range(g)]
+        for i in range(g):  # one head: its scores sum to its L_t rows' total mass
+            assert abs(heads[i].sum() - lt) <= 1e-11 * lt
+        assert np.allclose(O.key_scores(q, k, 0.35), sum(heads) / g, rtol=1e-12, atol=0)
+
+
 def pin_uniform_attention(O):
     """Q = 0 (or identical keys) gives A = 1/n exactly, so s_key_i = L_t / n."""
     for g, lt, n, d in [(1, 1, 5, 4), (4, 16, 64, 8), (3, 5, 7, 2)]:

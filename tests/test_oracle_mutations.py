@@ -19,6 +19,7 @@ MUTATIONS = {
     "scale 1/d instead of 1/sqrt(d)": ("1.0 / math.sqrt(d)\n    gamma", "1.0 / d\n    gamma"),
     "no max subtraction": ("e = np.exp(x - m)", "e = np.exp(x)"),
     "row normaliser drops the max": ("return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))", "return np.log(np.sum(np.exp(x), axis=1))"),
+    "row normaliser summed over every row": ("return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))", "return m + np.log(np.sum(np.exp(x - m[:, None])))"),
     "row normaliser log2": ("return m + np.log(np.sum(np.exp(x - m[:, None]), axis=1))", "return m + np.log2(np.sum(np.exp(x - m[:, None]), axis=1))"),
     "sum over the GQA group": ("return a.sum(axis=0) / g", "return a.sum(axis=0)"),
     "mean over guide tokens": ("return a.sum(axis=0) / g", "return a.mean(axis=0)"),
