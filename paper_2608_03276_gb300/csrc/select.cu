@@ -11,7 +11,8 @@
 // One thread-block cluster of CL CTAs (8; 12 for documents of 64K tokens or
 // more when every unit's cluster is resident at once; 4 when 8 per unit would
 // not fit in one wave and every slice still fits in shared memory) handles one
-// (document, head):
+// (document, head) -- or one (layer, document, head) when a stack of short
+// layers is selected in one launch (four-CTA clusters, all resident):
 // CTA r owns a contiguous slice of the tokens.  Histograms and per-slice
 // counts live in each CTA's shared memory and are summed across the cluster
 // through distributed shared memory, separated by hardware cluster barriers,
