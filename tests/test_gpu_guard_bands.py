@@ -3,7 +3,9 @@ memory sanitizer): each buffer the library writes sits between two 4 KiB bands
 of a known byte, and after the call every band must be untouched.  Covers the
 fused layer (both blend kernels, 8- and 4-bit codes, ragged documents with an
 empty one), the caller-normaliser and literal-normaliser layers, the stack of
-layers, and the stand-alone selection and compaction."""
+layers (also with the stack workspace, whose short layers are selected four
+per launch, and with a guide longer than one 512-row block), and the
+stand-alone selection and compaction."""
 import numpy as np
 import pytest
 
@@ -113,3 +115,30 @@ def test_stack_and_stages_stay_in_bounds(cuda_lib):
     binding.tp_select(p, scores, w.keep_ratio, w.budget, o.idx, o.ws)
     binding.tp_compact(p, k, v, gamma, o.idx, w.keep_ratio, w.budget, o.kc, o.vc, o.vqc, o.gammac)
     gd.check("stand-alone stages")
+
+
+@pytest.mark.parametrize("lt", [64, 160])
+def test_grouped_and_long_guide_stacks_stay_in_bounds(cuda_lib, lt):
+    """Both stacks with the stack workspace (the later layers' key scores,
+    scales and selection scratch in slots after the single-layer workspace):
+    guide 64 (256 rows) selects layers several per launch, guide 160 (640
+    rows) also scores in blocks of 512 rows."""
+    import torch
+    from paper_2608_03276_gb300 import binding
+    w = synth.small_variant(synth.WORKLOADS[2], [3001]).with_(guide_len=lt)
+    nl = 5
+    xs = [synth.make_layer(w, l) for l in range(nl)]
+    p = binding.Problem(w.n_heads_q, w.n_heads_kv, w.head_dim, w.guide_len, xs[0].doc_offsets)
+    gd = Guarded()
+    dev = [tuple(parity.to_device_bf16(t) for t in (y.q, y.k, y.v)) for y in xs]
+    ws = gd.make((binding.tp_workspace_bytes_stack(p, w.keep_ratio, w.budget, nl),), torch.uint8)
+    outs = [_outputs(binding, gd, p, w, w.keep_ratio, w.budget, scores=False) for _ in xs]
+    binding.tp_compress_layers(p, dev, w.keep_ratio, w.budget, outs, ws)
+    assert binding.tp_check_status(ws) == 0
+    gd.check(f"tp_compress_layers, stack workspace, guide {lt}")
+    lses = [gd.make((w.batch, w.n_heads_kv, w.rows), torch.float32) for _ in xs]
+    for (q, k, _), lse in zip(dev, lses):
+        binding.tp_guide_lse(p, q, k, lse, outs[0].ws)
+    binding.tp_compress_layers_lse(p, dev, lses, w.keep_ratio, w.budget, outs, ws)
+    assert binding.tp_check_status(ws) == 0
+    gd.check(f"tp_compress_layers_lse, stack workspace, guide {lt}")
