@@ -11,8 +11,11 @@
  * Conventions shared by every call
  * --------------------------------
  *  - All tensor pointers are DEVICE pointers to contiguous row-major memory,
- *    owned by the caller.  The library allocates nothing and keeps no state
- *    between calls apart from a cache of TMA descriptors (guarded by a mutex).
+ *    owned by the caller.  The library allocates nothing (tp_guide_lse_static's
+ *    fixed device array aside) and keeps no state between calls apart from
+ *    small per-CUDA-context caches, each guarded by a mutex: kernel attributes
+ *    already set, the device's answers to cluster co-residency queries, and
+ *    that array's device address.  TMA descriptors are encoded on every call.
  *  - bf16 tensors are passed as `const void*` (IEEE bfloat16 bit patterns).
  *  - Shapes (d = head_dim, N = total tokens = doc_offsets[batch]):
  *        Q guide   [batch, H_q, L_t, d]   bf16, post-RoPE guide queries
