@@ -40,6 +40,21 @@ int main(void) {
   CHECK(tp_kept_capacity(&p, 0.0, 2048) == 1500);
   CHECK(tp_workspace_bytes(&p, 0.1, -1) > 0);
 
+  /* the stack workspace: short documents get room for up to 7 more layers'
+   * key scores, scales and selection scratch; one layer needs none */
+  CHECK(tp_workspace_bytes_stack(&p, 0.1, -1, 1) == tp_workspace_bytes(&p, 0.1, -1));
+  CHECK(tp_workspace_bytes_stack(&p, 0.1, -1, 4) > tp_workspace_bytes(&p, 0.1, -1));
+  CHECK(tp_stack_layers_per_selection(&p, 0.1, -1, 4, tp_workspace_bytes(&p, 0.1, -1)) == 1);
+  CHECK(tp_stack_layers_per_selection(&p, 0.1, -1, 0, 0) == -1);
+
+  /* a 256-token guide at G = 4 (1024 stacked rows) is taken in blocks; one
+   * above TP_MAX_GUIDE_ROWS is not */
+  p.guide_len = 256;
+  CHECK(tp_workspace_bytes(&p, 0.1, -1) > 0);
+  p.guide_len = TP_MAX_GUIDE_ROWS / 4 + 1;
+  CHECK(tp_workspace_bytes(&p, 0.1, -1) == 0);
+  p.guide_len = 64;
+
   p.head_dim = 96; /* unsupported head size */
   CHECK(tp_kept_capacity(&p, 0.1, -1) == -1);
   p.head_dim = 128;
