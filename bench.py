@@ -44,13 +44,11 @@ import argparse
 import datetime
 import hashlib
 import json
-import math
 import os
 import statistics
 import subprocess
 import sys
 import tempfile
-import threading
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))

@@ -11,10 +11,9 @@ import subprocess
 import numpy as np
 import pytest
 
-from oracle import taskpress_oracle as O
 from paper_2608_03276_gb300 import synth
 from tests import parity
-from tests.test_gpu_parity import SMALL, _oracle, _problem, _run_compress
+from tests.test_gpu_parity import SMALL, _oracle, _run_compress
 
 pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
