@@ -36,6 +36,18 @@ def test_exports_every_declared_symbol(lib):
         assert hasattr(cdll, n), n
 
 
+def test_missing_library_fails_loudly(tmp_path):
+    """The binding has no fallback: without the built library every call
+    raises (a fresh copy of the module, pointed at a path with no library)."""
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "binding_copy", os.path.join(ROOT, "paper_2608_03276_gb300", "binding.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    with pytest.raises(RuntimeError, match="not built"):
+        mod.load(str(tmp_path / "libtaskpress.so"))
+
+
 def test_budget_matches_oracle_and_exact_decimals(lib):
     for r in ["0", "0.05", "0.07", "0.1", "0.2", "0.25", "0.33", "0.5", "0.9", "1"]:
         for n in [0, 1, 2, 7, 100, 129, 2048, 32768, 65536, 131072, 294912]:
